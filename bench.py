@@ -1,0 +1,406 @@
+#!/usr/bin/env python3
+"""Throughput of one LoCA Stage-II pass on GB300: tokens/s/block at the Qwen2.5-7B shape.
+
+A step is one pass of the whole hot path over one batch of synthetic inputs resident in HBM:
+  loca_error -> loca_targets -> loca_batch_step -> loca_gram_cross -> loca_ridge_solve
+(head error, feedback targets, scale-normalised step, Gram / cross statistics on the tensor
+cores, projected ridge solves for every block and every candidate lambda).
+
+value     = N * L / (seconds per step)            tokens per second per block (higher is better)
+e2e       = the same metric with the inputs copied from pinned host memory and the adapters
+            copied back inside every timed step
+roofline  = the Gram / cross kernel (the dominant one): useful flops per launch
+            L * (2 N d^2 + N d (d + 1)) over its CUDA-event duration, against the measured
+            sustained bf16 peak
+cpu_baseline = the fp64 oracle on the host cores on a bounded sample (one block, a prefix of
+            the tokens)
+
+Inputs (X is 26 GB at 7B) are far larger than the 129 MB L2, so no flush is needed between
+steps.  --impl reference times the oracle itself (the reference arm of this comparison).
+Multi-GPU: the method needs one GPU; --gpus N runs N independent replicas (weak scaling),
+with a barrier and the max step time over ranks.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "LoCA fit tokens/s/block at Qwen2.5-7B shape, 1 GB300; % bf16 tensor-core peak"
+UNIT = "tokens/s/block"
+FALLBACK_SUSTAINED_TFLOPS = 1700.0  # profiling recipe's sustained figure, used if no measured file
+
+# dram bytes per launch of k_gram_cross_tc from an ncu capture (see profiles/), valid only for
+# the kernel source whose sha256 prefix is given; otherwise traffic is reported as null
+GRAM_TC_TRAFFIC = {"sha256": None, "bytes_per_unit": None, "unit": None}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--workload", default="qwen2.5-7b")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            mp = json.load(f)
+        return float(mp["bf16_tflops_sustained"]), "measured"
+    return FALLBACK_SUSTAINED_TFLOPS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples (200 ms) of SM clock and throttle reasons during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid):
+        self.uuid = uuid
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            args = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200"]
+            if self.uuid:
+                args += ["-i", self.uuid]
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(args, stdout=self.out, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.out.close()
+
+    def summary(self):
+        if self.proc is None or self.path is None:
+            return None
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, flags in rows for i, v in enumerate(flags) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+def dist_setup(args):
+    import torch
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend=backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+def max_over_ranks(world, value):
+    if world == 1:
+        return value
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([value], dtype=torch.float64, device="cuda" if torch.cuda.is_available() else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ----------------------------------------------------------------------------- oracle timing
+
+def oracle_sample(w, tokens, host):
+    """One oracle pass on a bounded sample: block 0, the first `tokens` tokens."""
+    import numpy as np
+
+    from oracle import loca_oracle as O
+
+    X = host["X0"][:tokens][None].astype(np.float64)
+    t0 = time.perf_counter()
+    O.loca_pass(host["z"][:tokens], host["label_cols"], host["y"][:tokens], X, host["P"][:1], host["Q"][:1],
+                host["A"][:1], w.eta, w.lambda_rel, t_feed="bf16" if w.act_dtype == "bf16" else None)
+    return time.perf_counter() - t0
+
+
+def host_sample(w, seed=0, tokens=None):
+    """Host-side inputs for the oracle sample (block 0 drawn with the same recipe)."""
+    import numpy as np
+
+    from synth import inputs as S
+
+    f = S.host_factors(w, seed)
+    n = tokens or w.N
+    ws = S.scaled(w, L=1, N=n)
+    X0 = S.host_X(ws, seed)[0]
+    if w.V == w.C:
+        z = (X0.astype(np.float64) @ f["W_head"].astype(np.float64)).astype(np.float32)
+    else:
+        z = S.host_logits(S.scaled(w, N=n), None, seed)
+    return dict(X0=X0, z=z, y=f["y"][:n], label_cols=f["label_cols"], P=f["P"], Q=f["Q"], A=f["A"])
+
+
+def run_reference(args, w):
+    host = host_sample(w, tokens=4096)
+    tokens = 2048
+    for _ in range(args.warmup):
+        oracle_sample(w, tokens, host)
+    times = [oracle_sample(w, tokens, host) for _ in range(args.steps)]
+    sec = sum(times) / len(times)
+    value = tokens / sec
+    cores = os.cpu_count()
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "L": w.L, "d": w.d, "N": w.N, "C": w.C, "r": w.r, "k": w.k,
+                   "sample": f"block 0, first {tokens} tokens"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": f"one block (of {w.L}), first {tokens} of {w.N} tokens, full d={w.d}; numpy fp64"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+def main():
+    args = parse()
+    from synth import inputs as S
+
+    w = S.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        rank = int(os.environ.get("RANK", "0"))
+        if rank == 0:
+            run_reference(args, w)
+        return
+
+    import numpy as np
+    import torch
+
+    world, rank, local = dist_setup(args)
+    import __graft_entry__
+
+    __graft_entry__.build()
+    from paper_2608_03020_gb300 import loca as lc
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    inp = S.device_inputs(w, seed=rank, device=dev)
+    X, z, y, cols, P, Q, A = (inp[k] for k in ("X", "z", "y", "label_cols", "P", "Q", "A"))
+    L, N, d, C, r, k = w.L, w.N, w.d, w.C, w.r, w.k
+    nl = len(w.lambda_rel)
+    act = X.dtype
+    f32 = dict(dtype=torch.float32, device=dev)
+    E = torch.empty((N, C), **f32)
+    ce = torch.empty((N,), **f32)
+    T = torch.empty((L, N, d), dtype=act, device=dev)
+    tsq = torch.empty((L,), dtype=torch.float64, device=dev)
+    xsq = torch.empty((L,), dtype=torch.float64, device=dev)
+    alpha = torch.empty((L,), **f32)
+    gram = torch.empty((L, d, d), **f32)
+    cross = torch.empty((L, d, d), **f32)
+    B = torch.empty((nl, L, d, k), **f32)
+    info = torch.empty((nl, L), dtype=torch.int32, device=dev)
+    ws_t = torch.empty(lc.targets_workspace_size(N, L, d), dtype=torch.uint8, device=dev)
+    ws_b = torch.empty(lc.batch_step_workspace_size(L), dtype=torch.uint8, device=dev)
+    ws_g = torch.empty(lc.gram_cross_workspace_size(), dtype=torch.uint8, device=dev)
+    ws_s = torch.empty(lc.ridge_solve_workspace_size(L, d, k), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    launches_per_step = 1 + 2 + 2 + 1 + 2  # error; targets+reduce; sumsq+step; gram/cross; project+solve
+
+    def step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        lc.loca_error(z, cols, y, E, ce=ce, stream=stream)
+        if ev is not None:
+            ev[1].record(stream)
+        lc.loca_targets(E, P, Q, T, tsq=tsq, workspace=ws_t, stream=stream)
+        if ev is not None:
+            ev[2].record(stream)
+        lc.loca_batch_step(X, tsq, w.eta, xsq, alpha, zero_first=True, workspace=ws_b, stream=stream)
+        if ev is not None:
+            ev[3].record(stream)
+        lc.loca_gram_cross(X, T, alpha, gram, cross, zero_first=True, workspace=ws_g, stream=stream)
+        if ev is not None:
+            ev[4].record(stream)
+        lc.loca_ridge_solve(gram, cross, A, w.lambda_rel, B, info, xsq_total=xsq, workspace=ws_s, stream=stream)
+        if ev is not None:
+            ev[5].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    status = lc.loca_device_status()
+    if status != 0:
+        raise SystemExit(f"device status {status} after warm-up")
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(dev).uuid)
+        uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        uuid = None
+    barrier(world)
+    torch.cuda.synchronize()
+    with ClockSampler(uuid) as clk:
+        t_start = torch.cuda.Event(enable_timing=True)
+        t_end = torch.cuda.Event(enable_timing=True)
+        t_start.record(stream)
+        for i in range(args.steps):
+            step(evs[i])
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    ms_total = t_start.elapsed_time(t_end)
+    ms_total = max_over_ranks(world, ms_total)
+    ms_step = ms_total / args.steps
+    stage_names = ["error", "targets", "batch_step", "gram_cross", "ridge_solve"]
+    stages = {n: statistics.mean(e[i].elapsed_time(e[i + 1]) for e in evs) for i, n in enumerate(stage_names)}
+    status = lc.loca_device_status()
+    if status != 0:
+        raise SystemExit(f"device status {status} after the timed steps")
+    if int(info.abs().sum().item()) != 0:
+        raise SystemExit("a ridge system was not positive definite")
+    value = world * N * L / (ms_step / 1e3)
+
+    # roofline of the Gram / cross kernel
+    peak, peak_kind = peaks()
+    flops = L * (2.0 * N * d * d + N * d * (d + 1.0))
+    achieved = flops / (stages["gram_cross"] / 1e3) / 1e12
+    src = open(os.path.join(ROOT, "paper_2608_03020_gb300", "csrc", "gram_tc.cu"), "rb").read()
+    sha = hashlib.sha256(src).hexdigest()[:16]
+    traffic = None
+    if GRAM_TC_TRAFFIC["sha256"] == sha and GRAM_TC_TRAFFIC["bytes_per_unit"] is not None:
+        traffic = GRAM_TC_TRAFFIC["bytes_per_unit"] * L  # bytes per launch
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "traffic": traffic, "kernel": "k_gram_cross_tc",
+                "peak_kind": f"bf16 dense sustained, {peak_kind}", "flops_per_launch": flops}
+
+    # end to end through the public API: host inputs copied in, adapters copied out, per step
+    e2e = None
+    if not args.no_e2e:
+        pin = dict(pin_memory=True)
+        hX = torch.empty(X.shape, dtype=X.dtype, **pin)
+        hX.copy_(X)
+        hz = torch.empty(z.shape, dtype=z.dtype, **pin)
+        hz.copy_(z)
+        small = {kk: torch.empty(v.shape, dtype=v.dtype, **pin).copy_(v) for kk, v in
+                 (("y", y), ("cols", cols), ("P", P), ("Q", Q), ("A", A))}
+        hB = torch.empty(B.shape, dtype=B.dtype, **pin)
+        hinfo = torch.empty(info.shape, dtype=info.dtype, **pin)
+        h2d = sum(t.numel() * t.element_size() for t in [hX, hz, *small.values()])
+        d2h = hB.numel() * hB.element_size() + hinfo.numel() * hinfo.element_size()
+
+        def e2e_step():
+            X.copy_(hX, non_blocking=True)
+            z.copy_(hz, non_blocking=True)
+            y.copy_(small["y"], non_blocking=True)
+            cols.copy_(small["cols"], non_blocking=True)
+            P.copy_(small["P"], non_blocking=True)
+            Q.copy_(small["Q"], non_blocking=True)
+            A.copy_(small["A"], non_blocking=True)
+            step()
+            hB.copy_(B, non_blocking=True)
+            hinfo.copy_(info, non_blocking=True)
+
+        e2e_steps = max(1, min(args.steps, 5))
+        e2e_step()
+        torch.cuda.synchronize()
+        barrier(world)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(e2e_steps):
+            e2e_step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        ms_e2e = max_over_ranks(world, a.elapsed_time(b)) / e2e_steps
+        e2e = {"value": world * N * L / (ms_e2e / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e, "steps": e2e_steps}
+        del hX, hz
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        tokens = 8192
+        host = host_sample(w, tokens=tokens)
+        oracle_sample(w, 512, host)
+        sec = oracle_sample(w, tokens, host)
+        cpu = {"value": tokens / sec, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+               "sample": f"one block (of {L}), first {tokens} of {N} tokens, full d={d}, C={C}, r={r}, k={k}; "
+                         f"numpy fp64, {sec:.1f} s"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": w.name, "L": L, "d": d, "N": N, "C": C, "r": r, "k": k,
+                       "lambda_rel": list(w.lambda_rel), "eta": w.eta, "parallelism": f"replicas{world}",
+                       "l2": "inputs larger than L2 (X is %.1f GB)" % (X.numel() * X.element_size() / 1e9)},
+            "stages_ms": stages,
+            "solve_ms": stages["ridge_solve"],
+            "roofline": roofline,
+            "gpu_launches": launches_per_step * args.steps,
+            "e2e": e2e,
+            "cpu_baseline": cpu,
+            "clocks": clk.summary(),
+        }
+        print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,219 @@
+/*
+ * loca.h — C ABI of the LoCA forward-only adaptation hot path on one GB300 (sm_103a).
+ *
+ * LoCA (Local Credit Assignment, arXiv 2608.03020) tunes the low-rank adapters
+ * H_l = Hbar_l + B_l A_l H_{l-1} of a frozen transformer (Eq. 1) without further
+ * backpropagation after one calibration.  One Stage-II outer iteration (S13) is, after
+ * the forward pass:
+ *
+ *   loca_error        top-layer error at the frozen head             (Eq. 4, Lemma S3)
+ *   loca_targets      tokenwise feedback predictions T_l = E P_l Q_l  (S3, S11)
+ *   loca_accumulate   streamed Gram / cross statistics with the
+ *                     scale-normalised step                          (Eqs. 6, 9, 10; S7, S8)
+ *   loca_ridge_solve  projected statistics and positive-definite
+ *                     solves B* = C (G + lambda I)^-1 for all blocks
+ *                     and all ridge candidates                       (Eq. 8, Theorem S6, S7)
+ *
+ * and, once before Stage II, loca_calib_fit fits each block's rank-r feedback map from
+ * probe-backward pairs (Eq. 5, S5).
+ *
+ * Notation: the paper's adapter rank (r) is k here and its feedback rank (k) is r here.
+ * The head W_u restricted to the C label columns is folded into P_l, so the error E has
+ * C columns and the paper's F_l e becomes the row  e^T P_l Q_l  (F_l^T = P_l Q_l).
+ *
+ * Conventions for every entry point:
+ *  - All array arguments are DEVICE pointers owned by the caller, contiguous row-major,
+ *    unless the argument's comment says "host".  The library allocates no memory; entry
+ *    points that need scratch take a caller-provided device workspace whose size the
+ *    matching *_workspace_size function returns (workspace may be NULL when that size
+ *    is 0).  The workspace must not be shared by calls that may overlap on the GPU.
+ *  - Work is enqueued asynchronously on `stream` (a cudaStream_t; NULL = the legacy
+ *    default stream).  The return value reports host-side validation and launch errors
+ *    only; conditions detected on the device (a bounded wait that gave up, see
+ *    loca_device_status; a system that is not positive definite, see `info`) are written
+ *    to device memory.
+ *  - No exception crosses the ABI and nothing is printed.  loca_last_error_string()
+ *    describes the last non-OK status of the calling thread.
+ *  - Pointers to 16-bit or 32-bit data must be aligned to their element size; the bf16
+ *    statistics path additionally needs 16-byte aligned X and T and d % 8 == 0 (its rows
+ *    are fed to the tensor cores by TMA, which reads 16-byte rows).
+ */
+#ifndef LOCA_H_
+#define LOCA_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes. */
+typedef enum loca_status {
+  LOCA_OK = 0,
+  LOCA_ERR_INVALID_ARG = 1,        /* null pointer where one is required, bad flag or value */
+  LOCA_ERR_SHAPE = 2,              /* a size is out of range or inconsistent */
+  LOCA_ERR_ALIGNMENT = 3,          /* a pointer or a row pitch is misaligned */
+  LOCA_ERR_UNSUPPORTED_DTYPE = 4,  /* dtype code not accepted by this entry point */
+  LOCA_ERR_CUDA = 5,               /* a CUDA runtime call or launch failed */
+  LOCA_ERR_TIMEOUT = 6,            /* a device wait gave up (reported by loca_device_status) */
+  LOCA_ERR_WORKSPACE = 7,          /* workspace missing or smaller than required */
+  LOCA_ERR_UNSUPPORTED = 8         /* valid request outside what this build supports */
+} loca_status;
+
+/* Element type codes. */
+enum { LOCA_F32 = 0, LOCA_BF16 = 1 };
+
+/* Library ABI version (major * 10000 + minor * 100 + patch). */
+int loca_version(void);
+
+/* Message for the last non-OK status returned to the calling thread ("" if none). */
+const char* loca_last_error_string(void);
+
+/*
+ * loca_device_status — read and clear the library's device status word on the current
+ * device.  Kernels whose waits are bounded (the tensor-core statistics kernel) write
+ * LOCA_ERR_TIMEOUT there when a wait gives up instead of hanging; their outputs are
+ * then undefined.  Synchronises `stream`.  *host_status receives LOCA_OK or the code.
+ */
+int loca_device_status(int32_t* host_status /* host */, void* stream);
+
+/*
+ * loca_error — top-layer error at the frozen head (Eq. 4; Lemma "Top-layer error", S3).
+ *
+ *   lse_n   = log sum_{j in S} exp(z[n, j])       S = full row (normaliser 0, the paper's
+ *                                                 softmax over the vocabulary) or the
+ *                                                 label columns (normaliser 1)
+ *   E[n, c] = w_n (exp(z[n, label_cols[c]] - lse_n) - [y_n == c])
+ *   ce[n]   = w_n (lse_n - z[n, label_cols[y_n]])
+ *
+ * logits      N x V, row pitch ldz elements (ldz >= V), LOCA_F32 or LOCA_BF16
+ * label_cols  C int32 column indices in [0, V), C in [1, 1024]
+ * y           N int32 labels in [0, C), or -1 for a masked position (weight 0, E row = 0)
+ * w           N float loss weights w_n >= 0, or NULL for all ones
+ * E           N x C float output
+ * ce          N float output, or NULL
+ * Arithmetic in fp32; one warp per row, single pass (running max and rescaled sum).
+ */
+int loca_error(const void* logits, int logit_dtype, int64_t N, int64_t V, int64_t ldz,
+               const int32_t* label_cols, int32_t C, const int32_t* y, const float* w,
+               int normaliser, float* E, float* ce, void* stream);
+
+/*
+ * loca_targets — tokenwise feedback predictions of every block (S3: Q_l := F_l E;
+ * applied through the low-rank factors as in S11):  T_l = (E P_l) Q_l.
+ *
+ * E    N x C float (from loca_error)
+ * P    L x C x r float, Q  L x r x d float (feedback factors, e.g. from loca_calib_fit)
+ * T    L x N x d output, t_dtype LOCA_BF16 (the tensor-core feed) or LOCA_F32;
+ *      each value is computed in fp32 and rounded once (round to nearest even)
+ * tsq  L double output ||T_l||_F^2 of the unrounded fp32 values, or NULL
+ *      (then no workspace is needed)
+ * r in [1, 64], C in [1, 1024].  Deterministic: partial sums are reduced in a fixed order.
+ */
+int loca_targets_workspace_size(int64_t N, int32_t L, int64_t d, size_t* bytes /* host */);
+int loca_targets(const float* E, int64_t N, int32_t C, const float* P, const float* Q,
+                 int32_t L, int32_t r, int64_t d, void* T, int t_dtype, double* tsq,
+                 void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * loca_accumulate — add one mini-batch of N tokens to the sufficient statistics of every
+ * block (Eqs. 6 and 9; additivity over mini-batches, S7; one step per block and
+ * mini-batch, Eq. 10 and S8):
+ *
+ *   xsq_b[l]  = ||X_l||_F^2                              (this batch)
+ *   alpha_l   = -eta sqrt(xsq_b[l] / tsq[l]), 0 if tsq[l] == 0
+ *               (= -eta_bar: eta RMS(X_l) / RMS(T_l), both N x d)
+ *   gram_l   += X_l^T X_l                                (d x d, symmetric, both halves written)
+ *   cross_l  += alpha_l T_l^T X_l                        (d x d; row = output channel i,
+ *                                                        column = input channel j)
+ *   xsq_total[l] += xsq_b[l]
+ *
+ * With zero_first != 0 the three outputs are overwritten instead of accumulated.
+ * X, T  L x N x d, both of `dtype`:
+ *   LOCA_BF16  tcgen05 tensor-core GEMM, bf16 operands, fp32 accumulation in tensor
+ *              memory; needs d % 8 == 0 and 16-byte aligned X and T
+ *   LOCA_F32   exact-input path: fp32 operands, fp64 accumulation (slow; small shapes)
+ * tsq   L double (from loca_targets, over the same tokens)
+ * gram, cross  L x d x d float;  xsq_total  L double.
+ * Deterministic: every output element is produced by one thread in a fixed order.
+ */
+int loca_accumulate_workspace_size(int32_t L, int64_t N, int64_t d, int dtype,
+                                   size_t* bytes /* host */);
+int loca_accumulate(const void* X, const void* T, int dtype, int32_t L, int64_t N, int64_t d,
+                    const double* tsq, float eta, int zero_first, float* gram, float* cross,
+                    double* xsq_total, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * loca_batch_step and loca_gram_cross — the two halves of loca_accumulate, for callers that
+ * schedule them separately (for example to time the tensor-core kernel on its own).
+ *
+ * loca_batch_step (Eq. 10; S8): xsq_b[l] = ||X_l||_F^2, alpha[l] = -eta sqrt(xsq_b[l] / tsq[l])
+ *   (0 if tsq[l] == 0), xsq_total[l] = (zero_first ? 0 : xsq_total[l]) + xsq_b[l].
+ *   alpha: L float device output.  Workspace: loca_batch_step_workspace_size.
+ * loca_gram_cross (Eq. 9; S7): gram_l (+)= X_l^T X_l, cross_l (+)= alpha[l] T_l^T X_l with the
+ *   alpha of loca_batch_step.  Workspace: loca_gram_cross_workspace_size (256 bytes; holds a
+ *   launch-local flag).  Arguments, layouts, dtypes and determinism as loca_accumulate.
+ */
+int loca_batch_step_workspace_size(int32_t L, size_t* bytes /* host */);
+int loca_batch_step(const void* X, int dtype, int32_t L, int64_t N, int64_t d, const double* tsq,
+                    float eta, int zero_first, double* xsq_total, float* alpha, void* workspace,
+                    size_t workspace_bytes, void* stream);
+int loca_gram_cross_workspace_size(size_t* bytes /* host */);
+int loca_gram_cross(const void* X, const void* T, int dtype, int32_t L, int64_t N, int64_t d,
+                    const float* alpha, int zero_first, float* gram, float* cross, void* workspace,
+                    size_t workspace_bytes, void* stream);
+
+/*
+ * loca_ridge_solve — closed-form block minimisers for every block l and every ridge
+ * candidate j (Eq. 8; Theorem S6; positive-definite solve without an inverse, S7):
+ *
+ *   G_l   = A_l^T gram_l A_l                              (k x k, Eq. 9 with p = A_l^T x)
+ *   C_l   = B_prev,l G_l + cross_l A_l                    (d x k; = sum_n rho_n p_n^T with
+ *                                                         rho = B^(t) p - eta_bar q, Eq. 6)
+ *   lam   = lambda_rel[j] * xsq_total[l] / d              (xsq_total != NULL; = tr(gram_l)/d)
+ *         = lambda_rel[j]                                 (xsq_total == NULL: absolute)
+ *   B[j, l] = C_l (G_l + lam I)^-1   via Cholesky (fp64) and two triangular substitutions
+ *
+ * gram, cross   L x d x d float;  A  L x d x k float;  B_prev  L x d x k float or NULL (0)
+ * lambda_rel    HOST array of nl > 0 positive floats, nl <= 16
+ * B             nl x L x d x k float output;  info  nl x L int32 output: 0, or p > 0 when
+ *               the p-th pivot of G_l + lam I is not positive (B[j, l] is then zero)
+ * G_out         L x k x k float output or NULL;  C_out  L x d x k float output or NULL
+ * k in [1, 64].
+ */
+int loca_ridge_solve_workspace_size(int32_t L, int64_t d, int32_t k, size_t* bytes /* host */);
+int loca_ridge_solve(const float* gram, const float* cross, const double* xsq_total,
+                     const float* A, const float* B_prev, const float* lambda_rel /* host */,
+                     int32_t nl, int32_t L, int64_t d, int32_t k, float* B, int32_t* info,
+                     float* G_out, float* C_out, void* workspace, size_t workspace_bytes,
+                     void* stream);
+
+/*
+ * loca_calib_fit — one-shot reduced-rank fit of every block's feedback map from
+ * probe-backward pairs (Eq. 5; Theorem "Feedback ridge solution" and Lemma
+ * "Rank-truncation error", S5).  Token-major:
+ *
+ *   F_hat_l^T = (E_probe^T E_probe + beta I_m)^-1 E_probe^T G_probe_l      (m x d)
+ *   F_hat_l^T = U S V^T  (thin SVD),  P_l = U_r S_r (m x r),  Q_l = V_r^T (r x d)
+ *
+ * so that loca_targets with (P_l, Q_l) applies the rank-r map F_l = (P_l Q_l)^T.  Signs:
+ * the entry of largest magnitude in each row of Q_l is positive.  Singular values that
+ * are zero (r > rank) give zero rows of Q_l and zero columns of P_l.
+ *
+ * E_probe  Np x m float; G_probe  L x Np x d float; beta > 0; 1 <= r <= m <= 64
+ * P        L x m x r float; Q  L x r x d float; sigma  L x r float or NULL
+ * Arithmetic: the m x m and m x d products in fp64, Cholesky solve and Jacobi
+ * eigen-decomposition of the m x m matrix F_hat^T F_hat... (one thread block per block l).
+ */
+int loca_calib_fit_workspace_size(int64_t Np, int32_t m, int64_t d, int32_t L, int32_t r,
+                                  size_t* bytes /* host */);
+int loca_calib_fit(const float* E_probe, const float* G_probe, int64_t Np, int32_t m, int64_t d,
+                   int32_t L, float beta, int32_t r, float* P, float* Q, float* sigma,
+                   void* workspace, size_t workspace_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LOCA_H_ */

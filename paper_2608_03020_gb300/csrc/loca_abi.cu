@@ -1,0 +1,390 @@
+// C ABI entry points: host-side validation, workspace layout, and dispatch to the kernels.
+// See include/loca.h for the contract of each function.
+#include <cuda_runtime.h>
+
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "loca_internal.h"
+
+namespace loca {
+namespace {
+
+thread_local char g_msg[512] = "";
+
+int fail(int code, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_msg, sizeof(g_msg), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+int cuda_fail(cudaError_t e, const char* where) {
+  return fail(LOCA_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+__device__ int32_t g_status_word = 0;
+
+constexpr int kMaxDevices = 64;
+
+}  // namespace
+
+int sm_count() {
+  static int cache[kMaxDevices] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 148;
+  if (cache[dev] == 0) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0)
+      v = 148;
+    cache[dev] = v;
+  }
+  return cache[dev];
+}
+
+int32_t* device_status_word() {
+  static int32_t* cache[kMaxDevices] = {};
+  static std::mutex mu;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lock(mu);
+  if (cache[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
+    cache[dev] = static_cast<int32_t*>(p);
+  }
+  return cache[dev];
+}
+
+}  // namespace loca
+
+using namespace loca;
+
+namespace {
+
+// ---- workspace layouts (offsets are 256-byte aligned)
+struct TargetsWs {
+  size_t partials, total;
+};
+TargetsWs targets_ws(int64_t N, int32_t L, int64_t d) {
+  TargetsWs w{};
+  w.partials = 0;
+  w.total = align256(sizeof(double) * size_t(L) * size_t(targets_num_partials(N, d)));
+  return w;
+}
+
+struct AccumWs {
+  size_t partials, alpha, abort_flag, total;
+};
+AccumWs accum_ws(int32_t L) {
+  AccumWs w{};
+  w.partials = 0;
+  w.alpha = align256(sizeof(double) * size_t(L) * size_t(sumsq_num_partials()));
+  w.abort_flag = w.alpha + align256(sizeof(float) * size_t(L));
+  w.total = w.abort_flag + 256;
+  return w;
+}
+
+struct SolveWs {
+  size_t ga, ca, total;
+};
+SolveWs solve_ws(int32_t L, int64_t d, int32_t k) {
+  SolveWs w{};
+  const size_t one = align256(sizeof(float) * size_t(L) * size_t(d) * size_t(k));
+  w.ga = 0;
+  w.ca = one;
+  w.total = 2 * one;
+  return w;
+}
+
+int check_ws(void* ws, size_t have, size_t need) {
+  if (need == 0) return LOCA_OK;
+  if (ws == nullptr) return fail(LOCA_ERR_WORKSPACE, "workspace is NULL but %zu bytes are required", need);
+  if (have < need)
+    return fail(LOCA_ERR_WORKSPACE, "workspace of %zu bytes is smaller than the %zu required", have, need);
+  if (!aligned(ws, 256)) return fail(LOCA_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  return LOCA_OK;
+}
+
+char* ws_at(void* ws, size_t off) { return static_cast<char*>(ws) + off; }
+
+}  // namespace
+
+extern "C" {
+
+int loca_version(void) { return 100; }
+
+const char* loca_last_error_string(void) { return g_msg; }
+
+int loca_device_status(int32_t* host_status, void* stream) {
+  if (host_status == nullptr) return fail(LOCA_ERR_INVALID_ARG, "host_status is NULL");
+  int32_t* w = device_status_word();
+  if (w == nullptr) return fail(LOCA_ERR_CUDA, "cannot resolve the device status word");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaMemcpyAsync(host_status, w, sizeof(int32_t), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(w, 0, sizeof(int32_t), s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "loca_device_status");
+  return LOCA_OK;
+}
+
+int loca_error(const void* logits, int logit_dtype, int64_t N, int64_t V, int64_t ldz,
+               const int32_t* label_cols, int32_t C, const int32_t* y, const float* w,
+               int normaliser, float* E, float* ce, void* stream) {
+  g_msg[0] = 0;
+  if (N < 0 || V < 1 || ldz < V) return fail(LOCA_ERR_SHAPE, "need N >= 0, V >= 1, ldz >= V (N=%lld V=%lld ldz=%lld)", (long long)N, (long long)V, (long long)ldz);
+  if (C < 1 || C > 1024 || C > V) return fail(LOCA_ERR_SHAPE, "need 1 <= C <= min(V, 1024), got C=%d", C);
+  if (logit_dtype != LOCA_F32 && logit_dtype != LOCA_BF16)
+    return fail(LOCA_ERR_UNSUPPORTED_DTYPE, "logit_dtype must be LOCA_F32 or LOCA_BF16");
+  if (normaliser != 0 && normaliser != 1) return fail(LOCA_ERR_INVALID_ARG, "normaliser must be 0 or 1");
+  if (N == 0) return LOCA_OK;
+  if (!logits || !label_cols || !y || !E) return fail(LOCA_ERR_INVALID_ARG, "logits, label_cols, y and E are required");
+  const size_t es = logit_dtype == LOCA_BF16 ? 2 : 4;
+  if (!aligned(logits, es) || !aligned(label_cols, 4) || !aligned(y, 4) || !aligned(E, 4) ||
+      (w && !aligned(w, 4)) || (ce && !aligned(ce, 4)))
+    return fail(LOCA_ERR_ALIGNMENT, "pointers must be aligned to their element size");
+  cudaError_t e = launch_head_error(logits, logit_dtype, N, V, ldz, label_cols, C, y, w, normaliser,
+                                    E, ce, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "loca_error launch");
+  return LOCA_OK;
+}
+
+int loca_targets_workspace_size(int64_t N, int32_t L, int64_t d, size_t* bytes) {
+  if (!bytes) return fail(LOCA_ERR_INVALID_ARG, "bytes is NULL");
+  if (N < 0 || L < 1 || d < 1) return fail(LOCA_ERR_SHAPE, "need N >= 0, L >= 1, d >= 1");
+  *bytes = targets_ws(N, L, d).total;
+  return LOCA_OK;
+}
+
+int loca_targets(const float* E, int64_t N, int32_t C, const float* P, const float* Q, int32_t L,
+                 int32_t r, int64_t d, void* T, int t_dtype, double* tsq, void* workspace,
+                 size_t workspace_bytes, void* stream) {
+  g_msg[0] = 0;
+  if (N < 0 || L < 1 || L > 65535 || d < 1) return fail(LOCA_ERR_SHAPE, "need N >= 0, 1 <= L <= 65535, d >= 1");
+  if (C < 1 || C > 1024) return fail(LOCA_ERR_SHAPE, "need 1 <= C <= 1024");
+  if (r < 1 || r > 64) return fail(LOCA_ERR_SHAPE, "need 1 <= r <= 64, got %d", r);
+  if (t_dtype != LOCA_F32 && t_dtype != LOCA_BF16)
+    return fail(LOCA_ERR_UNSUPPORTED_DTYPE, "t_dtype must be LOCA_F32 or LOCA_BF16");
+  if ((N > 0 && (!E || !T)) || !P || !Q) return fail(LOCA_ERR_INVALID_ARG, "E, P, Q and T are required");
+  const size_t es = t_dtype == LOCA_BF16 ? 2 : 4;
+  if (!aligned(E, 4) || !aligned(P, 4) || !aligned(Q, 4) || !aligned(T, 16) || (tsq && !aligned(tsq, 8)))
+    return fail(LOCA_ERR_ALIGNMENT, "E, P, Q need 4-byte, T 16-byte and tsq 8-byte alignment");
+  (void)es;
+  if (tsq) {
+    const int rc = check_ws(workspace, workspace_bytes, targets_ws(N, L, d).total);
+    if (rc != LOCA_OK) return rc;
+  }
+  cudaError_t e = launch_targets(E, N, C, P, Q, L, r, d, T, t_dtype, tsq,
+                                 tsq ? reinterpret_cast<double*>(ws_at(workspace, 0)) : nullptr,
+                                 static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "loca_targets launch");
+  return LOCA_OK;
+}
+
+}  // extern "C"
+
+namespace {
+
+int validate_stats_inputs(const void* X, const void* T, int dtype, int32_t L, int64_t N, int64_t d,
+                          bool need_T) {
+  if (L < 1 || L > 255 || N < 0 || d < 1) return fail(LOCA_ERR_SHAPE, "need 1 <= L <= 255, N >= 0, d >= 1");
+  if (dtype != LOCA_F32 && dtype != LOCA_BF16)
+    return fail(LOCA_ERR_UNSUPPORTED_DTYPE, "dtype must be LOCA_F32 or LOCA_BF16");
+  if (N > 0 && (!X || (need_T && !T))) return fail(LOCA_ERR_INVALID_ARG, "X and T are required");
+  if (dtype == LOCA_BF16) {
+    if (d % 8 != 0) return fail(LOCA_ERR_SHAPE, "the bf16 path needs d %% 8 == 0 (16-byte rows), got d=%lld", (long long)d);
+    if (d > 65536 || N > 2147483647LL) return fail(LOCA_ERR_SHAPE, "the bf16 path needs d <= 65536 and N < 2^31");
+    if (N > 0 && (!aligned(X, 16) || (need_T && !aligned(T, 16))))
+      return fail(LOCA_ERR_ALIGNMENT, "the bf16 path needs 16-byte aligned X and T");
+  } else {
+    if (N > 0 && (!aligned(X, 4) || (need_T && !aligned(T, 4)))) return fail(LOCA_ERR_ALIGNMENT, "X and T need 4-byte alignment");
+  }
+  return LOCA_OK;
+}
+
+int run_batch_step(const void* X, int dtype, int32_t L, int64_t N, int64_t d, const double* tsq,
+                   float eta, int zero_first, double* xsq_total, float* alpha, double* partials,
+                   cudaStream_t s) {
+  cudaError_t e = launch_sumsq_and_step(X, dtype, L, N, d, tsq, eta, zero_first, xsq_total, partials, alpha, s);
+  if (e != cudaSuccess) return cuda_fail(e, "batch step: sum of squares");
+  return LOCA_OK;
+}
+
+int run_gram_cross(const void* X, const void* T, int dtype, int32_t L, int64_t N, int64_t d,
+                   const float* alpha, int zero_first, float* gram, float* cross, int32_t* abort_flag,
+                   cudaStream_t s) {
+  cudaError_t e = cudaSuccess;
+  if (N == 0) {
+    if (zero_first) {
+      e = cudaMemsetAsync(gram, 0, sizeof(float) * size_t(L) * size_t(d) * size_t(d), s);
+      if (e == cudaSuccess) e = cudaMemsetAsync(cross, 0, sizeof(float) * size_t(L) * size_t(d) * size_t(d), s);
+      if (e != cudaSuccess) return cuda_fail(e, "Gram/cross: zeroing");
+    }
+    return LOCA_OK;
+  }
+  if (dtype == LOCA_BF16) {
+    int32_t* status = device_status_word();
+    if (!status) return fail(LOCA_ERR_CUDA, "cannot resolve the device status word");
+    e = launch_gram_cross_tc(X, T, L, N, d, alpha, zero_first, gram, cross, status, abort_flag, s);
+  } else {
+    e = launch_gram_cross_f32(static_cast<const float*>(X), static_cast<const float*>(T), L, N, d,
+                              alpha, zero_first, gram, cross, s);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "Gram/cross launch");
+  return LOCA_OK;
+}
+
+size_t batch_step_ws(int32_t L) { return align256(sizeof(double) * size_t(L) * size_t(sumsq_num_partials())); }
+constexpr size_t kGramCrossWs = 256;
+
+}  // namespace
+
+extern "C" {
+
+int loca_batch_step_workspace_size(int32_t L, size_t* bytes) {
+  if (!bytes) return fail(LOCA_ERR_INVALID_ARG, "bytes is NULL");
+  if (L < 1) return fail(LOCA_ERR_SHAPE, "need L >= 1");
+  *bytes = batch_step_ws(L);
+  return LOCA_OK;
+}
+
+int loca_batch_step(const void* X, int dtype, int32_t L, int64_t N, int64_t d, const double* tsq,
+                    float eta, int zero_first, double* xsq_total, float* alpha, void* workspace,
+                    size_t workspace_bytes, void* stream) {
+  g_msg[0] = 0;
+  int rc = validate_stats_inputs(X, nullptr, dtype, L, N, d, false);
+  if (rc != LOCA_OK) return rc;
+  if (!(eta >= 0.f)) return fail(LOCA_ERR_INVALID_ARG, "eta must be >= 0");
+  if (!tsq || !xsq_total || !alpha) return fail(LOCA_ERR_INVALID_ARG, "tsq, xsq_total and alpha are required");
+  if (!aligned(tsq, 8) || !aligned(xsq_total, 8) || !aligned(alpha, 4))
+    return fail(LOCA_ERR_ALIGNMENT, "tsq and xsq_total need 8-byte, alpha 4-byte alignment");
+  rc = check_ws(workspace, workspace_bytes, batch_step_ws(L));
+  if (rc != LOCA_OK) return rc;
+  return run_batch_step(X, dtype, L, N, d, tsq, eta, zero_first, xsq_total, alpha,
+                        reinterpret_cast<double*>(workspace), static_cast<cudaStream_t>(stream));
+}
+
+int loca_gram_cross_workspace_size(size_t* bytes) {
+  if (!bytes) return fail(LOCA_ERR_INVALID_ARG, "bytes is NULL");
+  *bytes = kGramCrossWs;
+  return LOCA_OK;
+}
+
+int loca_gram_cross(const void* X, const void* T, int dtype, int32_t L, int64_t N, int64_t d,
+                    const float* alpha, int zero_first, float* gram, float* cross, void* workspace,
+                    size_t workspace_bytes, void* stream) {
+  g_msg[0] = 0;
+  int rc = validate_stats_inputs(X, T, dtype, L, N, d, true);
+  if (rc != LOCA_OK) return rc;
+  if (!alpha || !gram || !cross) return fail(LOCA_ERR_INVALID_ARG, "alpha, gram and cross are required");
+  if (!aligned(gram, 16) || !aligned(cross, 16) || !aligned(alpha, 4))
+    return fail(LOCA_ERR_ALIGNMENT, "gram and cross need 16-byte, alpha 4-byte alignment");
+  rc = check_ws(workspace, workspace_bytes, kGramCrossWs);
+  if (rc != LOCA_OK) return rc;
+  return run_gram_cross(X, T, dtype, L, N, d, alpha, zero_first, gram, cross,
+                        reinterpret_cast<int32_t*>(workspace), static_cast<cudaStream_t>(stream));
+}
+
+int loca_accumulate_workspace_size(int32_t L, int64_t N, int64_t d, int dtype, size_t* bytes) {
+  (void)N;
+  (void)d;
+  (void)dtype;
+  if (!bytes) return fail(LOCA_ERR_INVALID_ARG, "bytes is NULL");
+  if (L < 1) return fail(LOCA_ERR_SHAPE, "need L >= 1");
+  *bytes = accum_ws(L).total;
+  return LOCA_OK;
+}
+
+int loca_accumulate(const void* X, const void* T, int dtype, int32_t L, int64_t N, int64_t d,
+                    const double* tsq, float eta, int zero_first, float* gram, float* cross,
+                    double* xsq_total, void* workspace, size_t workspace_bytes, void* stream) {
+  g_msg[0] = 0;
+  int rc = validate_stats_inputs(X, T, dtype, L, N, d, true);
+  if (rc != LOCA_OK) return rc;
+  if (!(eta >= 0.f)) return fail(LOCA_ERR_INVALID_ARG, "eta must be >= 0");
+  if (!tsq || !gram || !cross || !xsq_total)
+    return fail(LOCA_ERR_INVALID_ARG, "tsq, gram, cross and xsq_total are required");
+  if (!aligned(gram, 16) || !aligned(cross, 16) || !aligned(tsq, 8) || !aligned(xsq_total, 8))
+    return fail(LOCA_ERR_ALIGNMENT, "gram and cross need 16-byte, tsq and xsq_total 8-byte alignment");
+  const AccumWs lay = accum_ws(L);
+  rc = check_ws(workspace, workspace_bytes, lay.total);
+  if (rc != LOCA_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  float* alpha = reinterpret_cast<float*>(ws_at(workspace, lay.alpha));
+  rc = run_batch_step(X, dtype, L, N, d, tsq, eta, zero_first, xsq_total, alpha,
+                      reinterpret_cast<double*>(ws_at(workspace, lay.partials)), s);
+  if (rc != LOCA_OK) return rc;
+  return run_gram_cross(X, T, dtype, L, N, d, alpha, zero_first, gram, cross,
+                        reinterpret_cast<int32_t*>(ws_at(workspace, lay.abort_flag)), s);
+}
+
+int loca_ridge_solve_workspace_size(int32_t L, int64_t d, int32_t k, size_t* bytes) {
+  if (!bytes) return fail(LOCA_ERR_INVALID_ARG, "bytes is NULL");
+  if (L < 1 || d < 1 || k < 1) return fail(LOCA_ERR_SHAPE, "need L, d, k >= 1");
+  *bytes = solve_ws(L, d, k).total;
+  return LOCA_OK;
+}
+
+int loca_ridge_solve(const float* gram, const float* cross, const double* xsq_total, const float* A,
+                     const float* B_prev, const float* lambda_rel, int32_t nl, int32_t L, int64_t d,
+                     int32_t k, float* B, int32_t* info, float* G_out, float* C_out,
+                     void* workspace, size_t workspace_bytes, void* stream) {
+  g_msg[0] = 0;
+  if (L < 1 || L > 65535 || d < 1) return fail(LOCA_ERR_SHAPE, "need 1 <= L <= 65535, d >= 1");
+  if (k < 1 || k > 32 || k > d) return fail(LOCA_ERR_SHAPE, "need 1 <= k <= min(d, 32), got k=%d", k);
+  if (nl < 1 || nl > 16) return fail(LOCA_ERR_SHAPE, "need 1 <= nl <= 16, got nl=%d", nl);
+  if (!gram || !cross || !A || !lambda_rel || !B || !info)
+    return fail(LOCA_ERR_INVALID_ARG, "gram, cross, A, lambda_rel, B and info are required");
+  for (int j = 0; j < nl; ++j)
+    if (!(lambda_rel[j] > 0.f)) return fail(LOCA_ERR_INVALID_ARG, "lambda_rel[%d] must be > 0", j);
+  if (!aligned(gram, 4) || !aligned(cross, 4) || !aligned(A, 4) || !aligned(B, 4) ||
+      !aligned(info, 4) || (B_prev && !aligned(B_prev, 4)) || (xsq_total && !aligned(xsq_total, 8)) ||
+      (G_out && !aligned(G_out, 4)) || (C_out && !aligned(C_out, 4)))
+    return fail(LOCA_ERR_ALIGNMENT, "pointers must be aligned to their element size");
+  const SolveWs lay = solve_ws(L, d, k);
+  int rc = check_ws(workspace, workspace_bytes, lay.total);
+  if (rc != LOCA_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  float* GA = reinterpret_cast<float*>(ws_at(workspace, lay.ga));
+  float* CA = reinterpret_cast<float*>(ws_at(workspace, lay.ca));
+  cudaError_t e = launch_project_rows(gram, cross, A, L, d, k, GA, CA, s);
+  if (e != cudaSuccess) return cuda_fail(e, "loca_ridge_solve: projection");
+  e = launch_chol_solve(GA, CA, A, B_prev, xsq_total, lambda_rel, nl, L, d, k, B, info, G_out, C_out, s);
+  if (e != cudaSuccess) return cuda_fail(e, "loca_ridge_solve: solve");
+  return LOCA_OK;
+}
+
+int loca_calib_fit_workspace_size(int64_t Np, int32_t m, int64_t d, int32_t L, int32_t r, size_t* bytes) {
+  if (!bytes) return fail(LOCA_ERR_INVALID_ARG, "bytes is NULL");
+  if (Np < 1 || m < 1 || m > 64 || d < 1 || L < 1 || r < 1 || r > m)
+    return fail(LOCA_ERR_SHAPE, "need Np >= 1, 1 <= r <= m <= 64, d >= 1, L >= 1");
+  *bytes = calib_workspace_bytes(Np, m, d, L, r);
+  return LOCA_OK;
+}
+
+int loca_calib_fit(const float* E_probe, const float* G_probe, int64_t Np, int32_t m, int64_t d,
+                   int32_t L, float beta, int32_t r, float* P, float* Q, float* sigma,
+                   void* workspace, size_t workspace_bytes, void* stream) {
+  g_msg[0] = 0;
+  if (Np < 1 || m < 1 || m > 64 || d < 1 || L < 1 || L > 65535 || r < 1 || r > m)
+    return fail(LOCA_ERR_SHAPE, "need Np >= 1, 1 <= r <= m <= 64, d >= 1, 1 <= L <= 65535");
+  if (!(beta > 0.f)) return fail(LOCA_ERR_INVALID_ARG, "beta must be > 0");
+  if (!E_probe || !G_probe || !P || !Q) return fail(LOCA_ERR_INVALID_ARG, "E_probe, G_probe, P and Q are required");
+  if (!aligned(E_probe, 4) || !aligned(G_probe, 4) || !aligned(P, 4) || !aligned(Q, 4) ||
+      (sigma && !aligned(sigma, 4)))
+    return fail(LOCA_ERR_ALIGNMENT, "pointers must be 4-byte aligned");
+  int rc = check_ws(workspace, workspace_bytes, calib_workspace_bytes(Np, m, d, L, r));
+  if (rc != LOCA_OK) return rc;
+  cudaError_t e = launch_calib_fit(E_probe, G_probe, Np, m, d, L, beta, r, P, Q, sigma, workspace,
+                                   static_cast<cudaStream_t>(stream));
+  if (e == cudaErrorNotSupported) return fail(LOCA_ERR_UNSUPPORTED, "calibration fit is not built");
+  if (e != cudaSuccess) return cuda_fail(e, "loca_calib_fit launch");
+  return LOCA_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,64 @@
+// Internal declarations shared by the library's translation units (host side).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/loca.h"
+
+namespace loca {
+
+// Number of SMs of the current device (cached per device).
+int sm_count();
+
+// Device address of the library's status word on the current device (see
+// loca_device_status); resolved once per device with that device current.
+int32_t* device_status_word();
+
+// Bytes needed to round `n` up to a 256-byte boundary.
+inline size_t align256(size_t n) { return (n + 255) & ~size_t(255); }
+
+// ---- head error (error.cu)
+cudaError_t launch_head_error(const void* z, int dtype, int64_t N, int64_t V, int64_t ldz,
+                              const int32_t* cols, int C, const int32_t* y, const float* w,
+                              int normaliser, float* E, float* ce, cudaStream_t s);
+
+// ---- feedback targets (targets.cu)
+// Grid geometry used by launch_targets; partial sums of ||T_l||^2 live in
+// `partials` (L x targets_num_partials(N, d) doubles).
+int64_t targets_num_partials(int64_t N, int64_t d);
+cudaError_t launch_targets(const float* E, int64_t N, int C, const float* P, const float* Q,
+                           int L, int r, int64_t d, void* T, int t_dtype, double* tsq,
+                           double* partials, cudaStream_t s);
+
+// ---- statistics (stats.cu, gram_tc.cu)
+// Sum of squares of X (per block) and the step alpha_l; partials: L x sumsq_num_partials().
+int sumsq_num_partials();
+cudaError_t launch_sumsq_and_step(const void* X, int dtype, int L, int64_t N, int64_t d,
+                                  const double* tsq, float eta, int zero_first, double* xsq_total,
+                                  double* partials, float* alpha, cudaStream_t s);
+// fp32-input Gram / cross (fp64 accumulation).
+cudaError_t launch_gram_cross_f32(const float* X, const float* T, int L, int64_t N, int64_t d,
+                                  const float* alpha, int zero_first, float* gram, float* cross,
+                                  cudaStream_t s);
+// bf16-input Gram / cross on tcgen05 tensor cores.
+cudaError_t launch_gram_cross_tc(const void* X, const void* T, int L, int64_t N, int64_t d,
+                                 const float* alpha, int zero_first, float* gram, float* cross,
+                                 int32_t* status, int32_t* abort_flag, cudaStream_t s);
+
+// ---- ridge solve (solve.cu)
+cudaError_t launch_project_rows(const float* gram, const float* cross, const float* A, int L,
+                                int64_t d, int k, float* GA, float* CA, cudaStream_t s);
+cudaError_t launch_chol_solve(const float* GA, const float* CA, const float* A, const float* B_prev,
+                              const double* xsq_total, const float* lambda_rel, int nl, int L,
+                              int64_t d, int k, float* B, int32_t* info, float* G_out,
+                              float* C_out, cudaStream_t s);
+
+// ---- calibration (calib.cu)
+size_t calib_workspace_bytes(int64_t Np, int m, int64_t d, int L, int r);
+cudaError_t launch_calib_fit(const float* E_probe, const float* G_probe, int64_t Np, int m,
+                             int64_t d, int L, float beta, int r, float* P, float* Q, float* sigma,
+                             void* workspace, cudaStream_t s);
+
+}  // namespace loca

@@ -1,0 +1,281 @@
+// Projected statistics and batched positive-definite solves (Eqs. 8 and 9; Theorem S6; S7).
+//
+// k_project_rows  GA_l = Gram_l A_l, CA_l = Cross_l A_l (d x k each).  One thread per row of the
+//                 stacked [Gram_l; Cross_l]; each thread streams its row with 32-byte loads while
+//                 the block shares A_l through shared memory (broadcast reads).  Bound: the HBM
+//                 read of Gram and Cross (8 d^2 bytes per block), k fp32 FMAs per element read.
+// k_chol_solve    one thread block per (ridge candidate j, block l):
+//                 G_l = A_l^T GA_l (k x k), lambda from the trace, Cholesky of G_l + lambda I in
+//                 fp64 in shared memory, then every row i of C_l = B_prev,l G_l + CA_l is solved
+//                 by a forward and a back substitution:  B[j, l, i] = C_l[i] (G_l + lambda I)^-1.
+//                 k is padded to a compile-time size with an identity block (its solution
+//                 columns are zero), so each row's solve stays in registers.
+#include "loca_internal.h"
+
+namespace loca {
+namespace {
+
+constexpr int PR_THREADS = 256;
+constexpr int PR_JC = 128;  // columns of A staged per step
+
+template <int KM>
+__global__ void __launch_bounds__(PR_THREADS) k_project_rows(const float* __restrict__ gram,
+                                                            const float* __restrict__ cross,
+                                                            const float* __restrict__ A, int64_t d,
+                                                            int k, float* __restrict__ GA,
+                                                            float* __restrict__ CA) {
+  __shared__ float As[PR_JC][KM];
+  const int l = blockIdx.y;
+  const int64_t row = int64_t(blockIdx.x) * PR_THREADS + threadIdx.x;  // in [0, 2d)
+  const bool active = row < 2 * d;
+  const bool is_gram = row < d;
+  const int64_t i = is_gram ? row : row - d;
+  const float* M = (is_gram ? gram : cross) + int64_t(l) * d * d + (active ? i * d : 0);
+  const float* Al = A + int64_t(l) * d * k;
+  const bool vec = (d % 4 == 0);
+  float acc[KM];
+#pragma unroll
+  for (int s = 0; s < KM; ++s) acc[s] = 0.f;
+  for (int64_t j0 = 0; j0 < d; j0 += PR_JC) {
+    __syncthreads();
+    for (int e = threadIdx.x; e < PR_JC * KM; e += PR_THREADS) {
+      const int jj = e / KM, s = e % KM;
+      As[jj][s] = (j0 + jj < d && s < k) ? Al[(j0 + jj) * k + s] : 0.f;
+    }
+    __syncthreads();
+    if (!active) continue;
+    const int64_t jn = (d - j0) < PR_JC ? (d - j0) : PR_JC;
+    if (vec && jn == PR_JC) {
+#pragma unroll 2
+      for (int jj = 0; jj < PR_JC; jj += 8) {
+        const float4 m0 = __ldg(reinterpret_cast<const float4*>(M + j0 + jj));
+        const float4 m1 = __ldg(reinterpret_cast<const float4*>(M + j0 + jj + 4));
+        const float m[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+#pragma unroll
+          for (int s = 0; s < KM; ++s) acc[s] = fmaf(m[u], As[jj + u][s], acc[s]);
+      }
+    } else {
+      for (int jj = 0; jj < jn; ++jj) {
+        const float m = M[j0 + jj];
+#pragma unroll
+        for (int s = 0; s < KM; ++s) acc[s] = fmaf(m, As[jj][s], acc[s]);
+      }
+    }
+  }
+  if (!active) return;
+  float* out = (is_gram ? GA : CA) + (int64_t(l) * d + i) * k;
+#pragma unroll
+  for (int s = 0; s < KM; ++s)
+    if (s < k) out[s] = acc[s];
+}
+
+constexpr int CS_THREADS = 256;
+constexpr int CS_ROWS = 64;  // rows of A / GA staged per step when forming G
+
+template <int KM>
+__global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
+    const float* __restrict__ GA, const float* __restrict__ CA, const float* __restrict__ A,
+    const float* __restrict__ B_prev, const double* __restrict__ xsq_total, int64_t d, int k, int L,
+    float l0, float l1, float l2, float l3, float l4, float l5, float l6, float l7, float l8,
+    float l9, float l10, float l11, float l12, float l13, float l14, float l15,
+    float* __restrict__ B, int32_t* __restrict__ info, float* __restrict__ G_out,
+    float* __restrict__ C_out) {
+  __shared__ float As[CS_ROWS][KM];
+  __shared__ float Gs[CS_ROWS][KM];
+  __shared__ float Gf[KM][KM];   // G_l (fp32, symmetrised), padded with identity
+  __shared__ double Md[KM][KM];  // G_l + lambda I, then its Cholesky factor (lower)
+  __shared__ float Lf[KM][KM];
+  __shared__ float Linv[KM];
+  __shared__ int s_info;
+  const int j = blockIdx.x, l = blockIdx.y;
+  const float lam_rel[16] = {l0, l1, l2, l3, l4, l5, l6, l7, l8, l9, l10, l11, l12, l13, l14, l15};
+  const float* Al = A + int64_t(l) * d * k;
+  const float* GAl = GA + int64_t(l) * d * k;
+  const float* CAl = CA + int64_t(l) * d * k;
+
+  // G_l = A_l^T GA_l: thread owns entries e = t, t + 256, ... of the KM x KM matrix
+  constexpr int PER = (KM * KM + CS_THREADS - 1) / CS_THREADS;
+  float g[PER];
+#pragma unroll
+  for (int p = 0; p < PER; ++p) g[p] = 0.f;
+  for (int64_t i0 = 0; i0 < d; i0 += CS_ROWS) {
+    __syncthreads();
+    for (int e = threadIdx.x; e < CS_ROWS * KM; e += CS_THREADS) {
+      const int ii = e / KM, s = e % KM;
+      const bool ok = (i0 + ii < d) && s < k;
+      As[ii][s] = ok ? Al[(i0 + ii) * k + s] : 0.f;
+      Gs[ii][s] = ok ? GAl[(i0 + ii) * k + s] : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int p = 0; p < PER; ++p) {
+      const int e = threadIdx.x + p * CS_THREADS;
+      if (e < KM * KM) {
+        const int a = e / KM, b = e % KM;
+        float acc = g[p];
+        for (int ii = 0; ii < CS_ROWS; ++ii) acc = fmaf(As[ii][a], Gs[ii][b], acc);
+        g[p] = acc;
+      }
+    }
+  }
+#pragma unroll
+  for (int p = 0; p < PER; ++p) {
+    const int e = threadIdx.x + p * CS_THREADS;
+    if (e < KM * KM) Gf[e / KM][e % KM] = g[p];
+  }
+  __syncthreads();
+  const double lam =
+      double(lam_rel[j]) * (xsq_total != nullptr ? xsq_total[l] / double(d) : 1.0);
+  for (int e = threadIdx.x; e < KM * KM; e += CS_THREADS) {
+    const int a = e / KM, b = e % KM;
+    double v;
+    if (a < k && b < k) {
+      v = 0.5 * (double(Gf[a][b]) + double(Gf[b][a]));
+      if (a == b) v += lam;
+    } else {
+      v = (a == b) ? 1.0 : 0.0;
+    }
+    Md[a][b] = v;
+  }
+  __syncthreads();
+  if (G_out != nullptr && j == 0) {
+    for (int e = threadIdx.x; e < k * k; e += CS_THREADS) {
+      const int a = e / k, b = e % k;
+      G_out[(int64_t(l) * k + a) * k + b] = float(0.5 * (double(Gf[a][b]) + double(Gf[b][a])));
+    }
+  }
+  // Cholesky, lower factor, column by column (warp 0; lanes over rows)
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
+    int inf = 0;
+    for (int c = 0; c < KM; ++c) {
+      double diag = Md[c][c];
+      for (int t = 0; t < c; ++t) diag -= Md[c][t] * Md[c][t];
+      if (!(diag > 0.0)) {
+        inf = c + 1;
+        break;
+      }
+      const double lcc = sqrt(diag);
+      __syncwarp();
+      for (int r = c + 1 + lane; r < KM; r += 32) {
+        double v = Md[r][c];
+        for (int t = 0; t < c; ++t) v -= Md[r][t] * Md[c][t];
+        Md[r][c] = v / lcc;
+      }
+      __syncwarp();
+      if (lane == 0) Md[c][c] = lcc;
+      __syncwarp();
+    }
+    if (lane == 0) s_info = inf;
+  }
+  __syncthreads();
+  const int inf = s_info;
+  if (threadIdx.x == 0) info[int64_t(j) * L + l] = inf;
+  for (int e = threadIdx.x; e < KM * KM; e += CS_THREADS) {
+    const int a = e / KM, b = e % KM;
+    Lf[a][b] = (b <= a) ? float(Md[a][b]) : 0.f;
+  }
+  for (int a = threadIdx.x; a < KM; a += CS_THREADS) Linv[a] = float(1.0 / Md[a][a]);
+  __syncthreads();
+
+  float* Bj = B + (int64_t(j) * L + l) * d * k;
+  const float* Bp = B_prev ? B_prev + int64_t(l) * d * k : nullptr;
+  for (int64_t i = threadIdx.x; i < d; i += CS_THREADS) {
+    float c[KM];
+#pragma unroll
+    for (int s = 0; s < KM; ++s) c[s] = (s < k) ? CAl[i * k + s] : 0.f;
+    if (Bp != nullptr) {
+      float b[KM];
+#pragma unroll
+      for (int s = 0; s < KM; ++s) b[s] = (s < k) ? Bp[i * k + s] : 0.f;
+#pragma unroll
+      for (int s = 0; s < KM; ++s) {
+        float a = c[s];
+#pragma unroll
+        for (int t = 0; t < KM; ++t) a = fmaf(b[t], Gf[t][s], a);
+        c[s] = (s < k) ? a : 0.f;
+      }
+    }
+    if (C_out != nullptr && j == 0) {
+#pragma unroll
+      for (int s = 0; s < KM; ++s)
+        if (s < k) C_out[(int64_t(l) * d + i) * k + s] = c[s];
+    }
+    if (inf != 0) {
+#pragma unroll
+      for (int s = 0; s < KM; ++s)
+        if (s < k) Bj[i * k + s] = 0.f;
+      continue;
+    }
+    // forward: Lf y = c
+#pragma unroll
+    for (int s = 0; s < KM; ++s) {
+      float a = c[s];
+#pragma unroll
+      for (int t = 0; t < s; ++t) a = fmaf(-Lf[s][t], c[t], a);
+      c[s] = a * Linv[s];
+    }
+    // back: Lf^T x = y
+#pragma unroll
+    for (int s = KM - 1; s >= 0; --s) {
+      float a = c[s];
+#pragma unroll
+      for (int t = s + 1; t < KM; ++t) a = fmaf(-Lf[t][s], c[t], a);
+      c[s] = a * Linv[s];
+    }
+#pragma unroll
+    for (int s = 0; s < KM; ++s)
+      if (s < k) Bj[i * k + s] = c[s];
+  }
+}
+
+template <int KM>
+cudaError_t project_t(const float* gram, const float* cross, const float* A, int L, int64_t d,
+                      int k, float* GA, float* CA, cudaStream_t s) {
+  const dim3 grid = dim3(unsigned((2 * d + PR_THREADS - 1) / PR_THREADS), unsigned(L));
+  k_project_rows<KM><<<grid, PR_THREADS, 0, s>>>(gram, cross, A, d, k, GA, CA);
+  return cudaGetLastError();
+}
+
+template <int KM>
+cudaError_t solve_t(const float* GA, const float* CA, const float* A, const float* B_prev,
+                    const double* xsq_total, const float* lr, int nl, int L, int64_t d, int k,
+                    float* B, int32_t* info, float* G_out, float* C_out, cudaStream_t s) {
+  float v[16] = {};
+  for (int i = 0; i < nl && i < 16; ++i) v[i] = lr[i];
+  const dim3 grid = dim3(unsigned(nl), unsigned(L));
+  k_chol_solve<KM><<<grid, CS_THREADS, 0, s>>>(GA, CA, A, B_prev, xsq_total, d, k, L, v[0], v[1],
+                                               v[2], v[3], v[4], v[5], v[6], v[7], v[8], v[9],
+                                               v[10], v[11], v[12], v[13], v[14], v[15], B, info,
+                                               G_out, C_out);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_project_rows(const float* gram, const float* cross, const float* A, int L,
+                                int64_t d, int k, float* GA, float* CA, cudaStream_t s) {
+  if (k <= 4) return project_t<4>(gram, cross, A, L, d, k, GA, CA, s);
+  if (k <= 8) return project_t<8>(gram, cross, A, L, d, k, GA, CA, s);
+  if (k <= 16) return project_t<16>(gram, cross, A, L, d, k, GA, CA, s);
+  if (k <= 32) return project_t<32>(gram, cross, A, L, d, k, GA, CA, s);
+  return project_t<64>(gram, cross, A, L, d, k, GA, CA, s);
+}
+
+cudaError_t launch_chol_solve(const float* GA, const float* CA, const float* A, const float* B_prev,
+                              const double* xsq_total, const float* lambda_rel, int nl, int L,
+                              int64_t d, int k, float* B, int32_t* info, float* G_out,
+                              float* C_out, cudaStream_t s) {
+#define LOCA_SOLVE(KM)                                                                          \
+  return solve_t<KM>(GA, CA, A, B_prev, xsq_total, lambda_rel, nl, L, d, k, B, info, G_out, C_out, \
+                     s)
+  if (k <= 4) LOCA_SOLVE(4);
+  if (k <= 8) LOCA_SOLVE(8);
+  if (k <= 16) LOCA_SOLVE(16);
+  LOCA_SOLVE(32);
+#undef LOCA_SOLVE
+}
+
+}  // namespace loca

@@ -1,0 +1,363 @@
+"""Python binding of ``libloca.so`` (argument marshalling only).
+
+Every function here has the name of the C entry point it calls (``include/loca.h``), checks
+the tensors it is given (device, dtype, shape, contiguity), passes their device pointers and
+the current torch stream, and raises :class:`LocaError` on a non-OK status.  All arithmetic
+of the hot path runs in the library's CUDA kernels; PyTorch only provides device memory and
+streams.  There is no CPU fallback: importing works without a GPU, calling needs one.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libloca.so")
+
+LOCA_F32 = 0
+LOCA_BF16 = 1
+
+STATUS_NAMES = {
+    0: "LOCA_OK", 1: "LOCA_ERR_INVALID_ARG", 2: "LOCA_ERR_SHAPE", 3: "LOCA_ERR_ALIGNMENT",
+    4: "LOCA_ERR_UNSUPPORTED_DTYPE", 5: "LOCA_ERR_CUDA", 6: "LOCA_ERR_TIMEOUT",
+    7: "LOCA_ERR_WORKSPACE", 8: "LOCA_ERR_UNSUPPORTED",
+}
+
+# (name, restype, argtypes) of every exported entry point
+_P = ctypes.c_void_p
+_I32 = ctypes.c_int32
+_I64 = ctypes.c_int64
+_SZ = ctypes.c_size_t
+_F = ctypes.c_float
+SIGNATURES = [
+    ("loca_version", ctypes.c_int, []),
+    ("loca_last_error_string", ctypes.c_char_p, []),
+    ("loca_device_status", ctypes.c_int, [ctypes.POINTER(_I32), _P]),
+    ("loca_error", ctypes.c_int, [_P, ctypes.c_int, _I64, _I64, _I64, _P, _I32, _P, _P, ctypes.c_int, _P, _P, _P]),
+    ("loca_targets_workspace_size", ctypes.c_int, [_I64, _I32, _I64, ctypes.POINTER(_SZ)]),
+    ("loca_targets", ctypes.c_int, [_P, _I64, _I32, _P, _P, _I32, _I32, _I64, _P, ctypes.c_int, _P, _P, _SZ, _P]),
+    ("loca_accumulate_workspace_size", ctypes.c_int, [_I32, _I64, _I64, ctypes.c_int, ctypes.POINTER(_SZ)]),
+    ("loca_accumulate", ctypes.c_int,
+     [_P, _P, ctypes.c_int, _I32, _I64, _I64, _P, _F, ctypes.c_int, _P, _P, _P, _P, _SZ, _P]),
+    ("loca_batch_step_workspace_size", ctypes.c_int, [_I32, ctypes.POINTER(_SZ)]),
+    ("loca_batch_step", ctypes.c_int, [_P, ctypes.c_int, _I32, _I64, _I64, _P, _F, ctypes.c_int, _P, _P, _P, _SZ, _P]),
+    ("loca_gram_cross_workspace_size", ctypes.c_int, [ctypes.POINTER(_SZ)]),
+    ("loca_gram_cross", ctypes.c_int,
+     [_P, _P, ctypes.c_int, _I32, _I64, _I64, _P, ctypes.c_int, _P, _P, _P, _SZ, _P]),
+    ("loca_ridge_solve_workspace_size", ctypes.c_int, [_I32, _I64, _I32, ctypes.POINTER(_SZ)]),
+    ("loca_ridge_solve", ctypes.c_int,
+     [_P, _P, _P, _P, _P, ctypes.POINTER(_F), _I32, _I32, _I64, _I32, _P, _P, _P, _P, _P, _SZ, _P]),
+    ("loca_calib_fit_workspace_size", ctypes.c_int, [_I64, _I32, _I64, _I32, _I32, ctypes.POINTER(_SZ)]),
+    ("loca_calib_fit", ctypes.c_int,
+     [_P, _P, _I64, _I32, _I64, _I32, _F, _I32, _P, _P, _P, _P, _SZ, _P]),
+]
+
+
+class LocaError(RuntimeError):
+    def __init__(self, status: int, where: str, message: str):
+        self.status = status
+        super().__init__(f"{where}: {STATUS_NAMES.get(status, status)}: {message}")
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load ``libloca.so`` (built in-tree by ``_build.build()``); fails loudly if missing."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is not built: run __graft_entry__.build() (nvcc, sm_103a)")
+        h = ctypes.CDLL(LIB_PATH)
+        for name, res, args in SIGNATURES:
+            fn = getattr(h, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = h
+    return _lib
+
+
+def _check(rc: int, where: str):
+    if rc != 0:
+        msg = lib().loca_last_error_string().decode(errors="replace")
+        raise LocaError(rc, where, msg)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dev(t, name, dtype=None, ndim=None):
+    if t is None:
+        return
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype not in (dtype if isinstance(dtype, tuple) else (dtype,)):
+        raise TypeError(f"{name} has dtype {t.dtype}, expected {dtype}")
+    if ndim is not None and t.dim() != ndim:
+        raise ValueError(f"{name} must have {ndim} dimensions, got {tuple(t.shape)}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+def _code(dtype) -> int:
+    if dtype == torch.float32:
+        return LOCA_F32
+    if dtype == torch.bfloat16:
+        return LOCA_BF16
+    raise TypeError(f"unsupported dtype {dtype}")
+
+
+def _workspace(nbytes: int, device, given=None):
+    if nbytes == 0:
+        return None
+    if given is not None:
+        if given.numel() * given.element_size() < nbytes:
+            raise ValueError(f"workspace has {given.numel() * given.element_size()} bytes, need {nbytes}")
+        return given
+    return torch.empty(nbytes, dtype=torch.uint8, device=device)
+
+
+def loca_version() -> int:
+    return lib().loca_version()
+
+
+def loca_device_status(stream=None) -> int:
+    """Read and clear the device status word (LOCA_OK or LOCA_ERR_TIMEOUT)."""
+    out = ctypes.c_int32(0)
+    _check(lib().loca_device_status(ctypes.byref(out), _stream(stream)), "loca_device_status")
+    return out.value
+
+
+def loca_error(logits, label_cols, y, E, w=None, ce=None, normaliser=0, stream=None):
+    """Top-layer error at the head: fills ``E`` (N x C float) and optionally ``ce`` (N)."""
+    _dev(logits, "logits", (torch.float32, torch.bfloat16))
+    if logits.dim() != 2 or logits.stride(1) != 1:
+        raise ValueError("logits must be a 2-D row-major tensor (unit column stride)")
+    _dev(label_cols, "label_cols", torch.int32, 1)
+    _dev(y, "y", torch.int32, 1)
+    _dev(E, "E", torch.float32, 2)
+    _dev(w, "w", torch.float32, 1)
+    _dev(ce, "ce", torch.float32, 1)
+    N, V = logits.shape
+    C = label_cols.numel()
+    if E.shape != (N, C) or y.numel() != N:
+        raise ValueError("E must be N x C and y must have N entries")
+    rc = lib().loca_error(_ptr(logits), _code(logits.dtype), N, V, logits.stride(0), _ptr(label_cols), C,
+                          _ptr(y), _ptr(w), int(normaliser), _ptr(E), _ptr(ce), _stream(stream))
+    _check(rc, "loca_error")
+
+
+def targets_workspace_size(N, L, d) -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib().loca_targets_workspace_size(N, L, d, ctypes.byref(out)), "loca_targets_workspace_size")
+    return out.value
+
+
+def loca_targets(E, P, Q, T, tsq=None, workspace=None, stream=None):
+    """Feedback targets ``T_l = (E P_l) Q_l`` into ``T`` (L x N x d, bf16 or f32) and
+    ``tsq`` (L, float64, optional)."""
+    _dev(E, "E", torch.float32, 2)
+    _dev(P, "P", torch.float32, 3)
+    _dev(Q, "Q", torch.float32, 3)
+    _dev(T, "T", (torch.float32, torch.bfloat16), 3)
+    _dev(tsq, "tsq", torch.float64, 1)
+    N, C = E.shape
+    L, C2, r = P.shape
+    L2, r2, d = Q.shape
+    if C2 != C or L2 != L or r2 != r or tuple(T.shape) != (L, N, d):
+        raise ValueError("shape mismatch among E (N x C), P (L x C x r), Q (L x r x d), T (L x N x d)")
+    ws = None
+    nbytes = 0
+    if tsq is not None:
+        nbytes = targets_workspace_size(N, L, d)
+        ws = _workspace(nbytes, E.device, workspace)
+    rc = lib().loca_targets(_ptr(E), N, C, _ptr(P), _ptr(Q), L, r, d, _ptr(T), _code(T.dtype), _ptr(tsq),
+                            _ptr(ws), nbytes, _stream(stream))
+    _check(rc, "loca_targets")
+
+
+def accumulate_workspace_size(L, N, d, dtype) -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib().loca_accumulate_workspace_size(L, N, d, _code(dtype), ctypes.byref(out)),
+           "loca_accumulate_workspace_size")
+    return out.value
+
+
+def loca_accumulate(X, T, tsq, eta, gram, cross, xsq_total, zero_first, workspace=None, stream=None):
+    """Add one mini-batch to the Gram / cross statistics of every block."""
+    _dev(X, "X", (torch.float32, torch.bfloat16), 3)
+    _dev(T, "T", X.dtype, 3)
+    _dev(tsq, "tsq", torch.float64, 1)
+    _dev(gram, "gram", torch.float32, 3)
+    _dev(cross, "cross", torch.float32, 3)
+    _dev(xsq_total, "xsq_total", torch.float64, 1)
+    L, N, d = X.shape
+    if tuple(T.shape) != (L, N, d) or tuple(gram.shape) != (L, d, d) or tuple(cross.shape) != (L, d, d):
+        raise ValueError("shape mismatch among X, T (L x N x d) and gram, cross (L x d x d)")
+    nbytes = accumulate_workspace_size(L, N, d, X.dtype)
+    ws = _workspace(nbytes, X.device, workspace)
+    rc = lib().loca_accumulate(_ptr(X), _ptr(T), _code(X.dtype), L, N, d, _ptr(tsq), float(eta), int(bool(zero_first)),
+                               _ptr(gram), _ptr(cross), _ptr(xsq_total), _ptr(ws), nbytes, _stream(stream))
+    _check(rc, "loca_accumulate")
+
+
+def batch_step_workspace_size(L) -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib().loca_batch_step_workspace_size(L, ctypes.byref(out)), "loca_batch_step_workspace_size")
+    return out.value
+
+
+def loca_batch_step(X, tsq, eta, xsq_total, alpha, zero_first, workspace=None, stream=None):
+    """Step of Eq. 10 for one mini-batch: ``alpha[l] = -eta ||X_l|| / sqrt(tsq[l])``; updates
+    ``xsq_total``."""
+    _dev(X, "X", (torch.float32, torch.bfloat16), 3)
+    _dev(tsq, "tsq", torch.float64, 1)
+    _dev(xsq_total, "xsq_total", torch.float64, 1)
+    _dev(alpha, "alpha", torch.float32, 1)
+    L, N, d = X.shape
+    nbytes = batch_step_workspace_size(L)
+    ws = _workspace(nbytes, X.device, workspace)
+    rc = lib().loca_batch_step(_ptr(X), _code(X.dtype), L, N, d, _ptr(tsq), float(eta), int(bool(zero_first)),
+                               _ptr(xsq_total), _ptr(alpha), _ptr(ws), nbytes, _stream(stream))
+    _check(rc, "loca_batch_step")
+
+
+def gram_cross_workspace_size() -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib().loca_gram_cross_workspace_size(ctypes.byref(out)), "loca_gram_cross_workspace_size")
+    return out.value
+
+
+def loca_gram_cross(X, T, alpha, gram, cross, zero_first, workspace=None, stream=None):
+    """Statistics of Eq. 9 for one mini-batch with the step ``alpha`` of loca_batch_step."""
+    _dev(X, "X", (torch.float32, torch.bfloat16), 3)
+    _dev(T, "T", X.dtype, 3)
+    _dev(alpha, "alpha", torch.float32, 1)
+    _dev(gram, "gram", torch.float32, 3)
+    _dev(cross, "cross", torch.float32, 3)
+    L, N, d = X.shape
+    if tuple(T.shape) != (L, N, d) or tuple(gram.shape) != (L, d, d) or tuple(cross.shape) != (L, d, d):
+        raise ValueError("shape mismatch among X, T (L x N x d) and gram, cross (L x d x d)")
+    nbytes = gram_cross_workspace_size()
+    ws = _workspace(nbytes, X.device, workspace)
+    rc = lib().loca_gram_cross(_ptr(X), _ptr(T), _code(X.dtype), L, N, d, _ptr(alpha), int(bool(zero_first)),
+                               _ptr(gram), _ptr(cross), _ptr(ws), nbytes, _stream(stream))
+    _check(rc, "loca_gram_cross")
+
+
+def ridge_solve_workspace_size(L, d, k) -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib().loca_ridge_solve_workspace_size(L, d, k, ctypes.byref(out)), "loca_ridge_solve_workspace_size")
+    return out.value
+
+
+def loca_ridge_solve(gram, cross, A, lambda_rel, B, info, xsq_total=None, B_prev=None, G_out=None, C_out=None,
+                     workspace=None, stream=None):
+    """Closed-form adapters ``B[j, l] = C_l (G_l + lambda_j I)^-1`` for every block and candidate."""
+    _dev(gram, "gram", torch.float32, 3)
+    _dev(cross, "cross", torch.float32, 3)
+    _dev(A, "A", torch.float32, 3)
+    _dev(B, "B", torch.float32, 4)
+    _dev(info, "info", torch.int32, 2)
+    _dev(xsq_total, "xsq_total", torch.float64, 1)
+    _dev(B_prev, "B_prev", torch.float32, 3)
+    _dev(G_out, "G_out", torch.float32, 3)
+    _dev(C_out, "C_out", torch.float32, 3)
+    L, d, k = A.shape
+    lam = [float(v) for v in lambda_rel]
+    nl = len(lam)
+    if tuple(B.shape) != (nl, L, d, k) or tuple(info.shape) != (nl, L):
+        raise ValueError("B must be nl x L x d x k and info nl x L")
+    lam_arr = (ctypes.c_float * max(nl, 1))(*lam)
+    nbytes = ridge_solve_workspace_size(L, d, k)
+    ws = _workspace(nbytes, A.device, workspace)
+    rc = lib().loca_ridge_solve(_ptr(gram), _ptr(cross), _ptr(xsq_total), _ptr(A), _ptr(B_prev), lam_arr, nl, L, d,
+                                k, _ptr(B), _ptr(info), _ptr(G_out), _ptr(C_out), _ptr(ws), nbytes, _stream(stream))
+    _check(rc, "loca_ridge_solve")
+
+
+def calib_fit_workspace_size(Np, m, d, L, r) -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib().loca_calib_fit_workspace_size(Np, m, d, L, r, ctypes.byref(out)), "loca_calib_fit_workspace_size")
+    return out.value
+
+
+def loca_calib_fit(E_probe, G_probe, beta, r, P, Q, sigma=None, workspace=None, stream=None):
+    """Rank-r feedback factors ``P`` (L x m x r), ``Q`` (L x r x d) from probe pairs."""
+    _dev(E_probe, "E_probe", torch.float32, 2)
+    _dev(G_probe, "G_probe", torch.float32, 3)
+    _dev(P, "P", torch.float32, 3)
+    _dev(Q, "Q", torch.float32, 3)
+    _dev(sigma, "sigma", torch.float32, 2)
+    Np, m = E_probe.shape
+    L, Np2, d = G_probe.shape
+    if Np2 != Np or tuple(P.shape) != (L, m, r) or tuple(Q.shape) != (L, r, d):
+        raise ValueError("shape mismatch among E_probe, G_probe, P, Q")
+    nbytes = calib_fit_workspace_size(Np, m, d, L, r)
+    ws = _workspace(nbytes, E_probe.device, workspace)
+    rc = lib().loca_calib_fit(_ptr(E_probe), _ptr(G_probe), Np, m, d, L, float(beta), r, _ptr(P), _ptr(Q),
+                              _ptr(sigma), _ptr(ws), nbytes, _stream(stream))
+    _check(rc, "loca_calib_fit")
+
+
+class Pass:
+    """Device buffers and workspaces for repeated Stage-II outer iterations of one shape.
+
+    ``run()`` enqueues loca_error -> (loca_targets -> loca_accumulate per mini-batch) ->
+    loca_ridge_solve on the current stream and allocates nothing.
+    """
+
+    def __init__(self, L, N, d, C, r, k, act_dtype, lambda_rel, eta, micro_batches=1, device="cuda",
+                 t_dtype=None):
+        self.L, self.N, self.d, self.C, self.r, self.k = L, N, d, C, r, k
+        self.eta = float(eta)
+        self.lambda_rel = [float(v) for v in lambda_rel]
+        self.mb = int(micro_batches)
+        self.nb = -(-N // self.mb)
+        dev = torch.device(device)
+        t_dtype = act_dtype if t_dtype is None else t_dtype
+        f32 = dict(dtype=torch.float32, device=dev)
+        self.E = torch.empty((N, C), **f32)
+        self.ce = torch.empty((N,), **f32)
+        self.T = torch.empty((L, self.nb, d), dtype=t_dtype, device=dev)
+        self.tsq = torch.empty((L,), dtype=torch.float64, device=dev)
+        self.gram = torch.empty((L, d, d), **f32)
+        self.cross = torch.empty((L, d, d), **f32)
+        self.xsq = torch.empty((L,), dtype=torch.float64, device=dev)
+        nl = len(self.lambda_rel)
+        self.B = torch.empty((nl, L, d, k), **f32)
+        self.info = torch.empty((nl, L), dtype=torch.int32, device=dev)
+        self.ws_t = _workspace(targets_workspace_size(self.nb, L, d), dev)
+        self.ws_a = _workspace(accumulate_workspace_size(L, self.nb, d, act_dtype), dev)
+        self.ws_s = _workspace(ridge_solve_workspace_size(L, d, k), dev)
+
+    def run(self, logits, label_cols, y, X, P, Q, A, B_prev=None, normaliser=0, stream=None):
+        """``X``: one ``L x N x d`` tensor, or a list of per-mini-batch ``L x N_m x d`` tensors
+        (contiguous token ranges of ``ceil(N / micro_batches)`` tokens, in order)."""
+        loca_error(logits, label_cols, y, self.E, ce=self.ce, normaliser=normaliser, stream=stream)
+        batches = X if isinstance(X, (list, tuple)) else [X]
+        if len(batches) != self.mb:
+            raise ValueError(f"expected {self.mb} mini-batches of X, got {len(batches)}")
+        n0 = 0
+        for m, Xm in enumerate(batches):
+            nm = Xm.shape[1]
+            Tm = self.T.view(-1)[: self.L * nm * self.d].view(self.L, nm, self.d)
+            loca_targets(self.E[n0:n0 + nm], P, Q, Tm, tsq=self.tsq, workspace=self.ws_t, stream=stream)
+            loca_accumulate(Xm, Tm, self.tsq, self.eta, self.gram, self.cross, self.xsq, zero_first=(m == 0),
+                            workspace=self.ws_a, stream=stream)
+            n0 += nm
+        if n0 != self.N:
+            raise ValueError(f"mini-batches hold {n0} tokens, expected {self.N}")
+        loca_ridge_solve(self.gram, self.cross, A, self.lambda_rel, self.B, self.info, xsq_total=self.xsq,
+                         B_prev=B_prev, workspace=self.ws_s, stream=stream)
+        return self.B

@@ -1,0 +1,114 @@
+"""Host-side checks of the C ABI (no GPU needed): the library builds and loads, exports every
+symbol ``include/loca.h`` declares, the binding knows every one of them, and argument
+validation rejects bad calls with the documented status codes before any CUDA call."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "loca.h")
+
+
+def _declared():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(loca_[a-z0-9_]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2608_03020_gb300 import _build
+    from paper_2608_03020_gb300 import loca
+
+    _build.build()
+    return loca.lib()
+
+
+def test_header_declares_the_five_hot_path_calls():
+    names = _declared()
+    for n in ("loca_calib_fit", "loca_error", "loca_targets", "loca_accumulate", "loca_ridge_solve"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(L):
+    for name in _declared():
+        assert hasattr(L, name), name
+
+
+def test_binding_covers_every_declared_symbol():
+    from paper_2608_03020_gb300 import loca
+
+    assert sorted(n for n, _, _ in loca.SIGNATURES) == _declared()
+
+
+def test_version(L):
+    assert L.loca_version() == 100
+
+
+def _ws(fn, *args):
+    out = ctypes.c_size_t(0)
+    rc = fn(*args, ctypes.byref(out))
+    return rc, out.value
+
+
+def test_workspace_sizes(L):
+    rc, n = _ws(L.loca_targets_workspace_size, 131072, 28, 3584)
+    assert rc == 0 and n >= 8 * 28 * (131072 // 64) * 14 and n % 256 == 0
+    rc, n = _ws(L.loca_accumulate_workspace_size, 28, 131072, 3584, 1)
+    assert rc == 0 and n > 0
+    rc, n = _ws(L.loca_ridge_solve_workspace_size, 28, 3584, 16)
+    assert rc == 0 and n >= 2 * 4 * 28 * 3584 * 16
+    rc, _ = _ws(L.loca_ridge_solve_workspace_size, 0, 3584, 16)
+    assert rc == 2  # LOCA_ERR_SHAPE
+    assert L.loca_targets_workspace_size(1, 1, 1, None) == 1  # NULL out pointer
+
+
+def test_validation_codes(L):
+    # every call below is rejected on the host before any CUDA call
+    P = ctypes.c_void_p
+    fake = P(256)  # never dereferenced: validation fails first
+    # bad dtype code
+    assert L.loca_error(fake, 7, 4, 4, 4, fake, 4, fake, None, 0, fake, None, None) == 4
+    # C > V
+    assert L.loca_error(fake, 0, 4, 4, 4, fake, 5, fake, None, 0, fake, None, None) == 2
+    # normaliser out of range
+    assert L.loca_error(fake, 0, 4, 4, 4, fake, 4, fake, None, 2, fake, None, None) == 1
+    # missing E
+    assert L.loca_error(fake, 0, 4, 4, 4, fake, 4, fake, None, 0, None, None, None) == 1
+    # N == 0 is a no-op
+    assert L.loca_error(None, 0, 0, 4, 4, None, 4, None, None, 0, None, None, None) == 0
+    msg = L.loca_last_error_string()
+    assert msg == b""
+    # r out of range
+    assert L.loca_targets(fake, 8, 4, fake, fake, 2, 65, 64, fake, 1, None, None, 0, None) == 2
+    # misaligned T (T must be 16-byte aligned)
+    assert L.loca_targets(fake, 8, 4, fake, fake, 2, 4, 64, P(258), 1, None, None, 0, None) == 3
+    # tsq requested but no workspace
+    assert L.loca_targets(fake, 8, 4, fake, fake, 2, 4, 64, fake, 1, fake, None, 0, None) == 7
+    # bf16 statistics need d % 8 == 0
+    assert L.loca_accumulate(fake, fake, 1, 2, 64, 60, fake, ctypes.c_float(0.01), 1, fake, fake, fake,
+                             fake, 1 << 20, None) == 2
+    # negative eta
+    assert L.loca_accumulate(fake, fake, 1, 2, 64, 64, fake, ctypes.c_float(-1.0), 1, fake, fake, fake,
+                             fake, 1 << 20, None) == 1
+    # workspace too small
+    assert L.loca_accumulate(fake, fake, 1, 2, 64, 64, fake, ctypes.c_float(0.01), 1, fake, fake, fake,
+                             fake, 16, None) == 7
+    assert b"workspace" in L.loca_last_error_string()
+    # lambda_rel must be positive
+    lam = (ctypes.c_float * 2)(1e-3, 0.0)
+    assert L.loca_ridge_solve(fake, fake, None, fake, None, lam, 2, 2, 64, 4, fake, fake, None, None,
+                              fake, 1 << 24, None) == 1
+    # k above the supported maximum
+    lam = (ctypes.c_float * 1)(1e-3)
+    assert L.loca_ridge_solve(fake, fake, None, fake, None, lam, 1, 2, 64, 33, fake, fake, None, None,
+                              fake, 1 << 24, None) == 2
+    # calibration: r > m
+    assert L.loca_calib_fit(fake, fake, 16, 4, 64, 2, ctypes.c_float(0.1), 5, fake, fake, None, fake,
+                            1 << 20, None) == 2
+    # calibration: beta <= 0
+    assert L.loca_calib_fit(fake, fake, 16, 4, 64, 2, ctypes.c_float(0.0), 2, fake, fake, None, fake,
+                            1 << 20, None) == 1
