@@ -58,7 +58,9 @@ typedef enum loca_status {
   LOCA_ERR_CUDA = 5,               /* a CUDA runtime call or launch failed */
   LOCA_ERR_TIMEOUT = 6,            /* a device wait gave up (reported by loca_device_status) */
   LOCA_ERR_WORKSPACE = 7,          /* workspace missing or smaller than required */
-  LOCA_ERR_UNSUPPORTED = 8         /* valid request outside what this build supports */
+  LOCA_ERR_UNSUPPORTED = 8,        /* valid request outside what this build supports */
+  LOCA_ERR_NUMERIC = 9             /* device: a system that should be positive definite was not
+                                      in floating point (reported by loca_device_status) */
 } loca_status;
 
 /* Element type codes. */
@@ -203,8 +205,13 @@ int loca_ridge_solve(const float* gram, const float* cross, const double* xsq_to
  *
  * E_probe  Np x m float; G_probe  L x Np x d float; beta > 0; 1 <= r <= m <= 64
  * P        L x m x r float; Q  L x r x d float; sigma  L x r float or NULL
- * Arithmetic: the m x m and m x d products in fp64, Cholesky solve and Jacobi
- * eigen-decomposition of the m x m matrix F_hat^T F_hat... (one thread block per block l).
+ * Arithmetic: E^T E and E^T G_l from fp32 products summed in fp32 over 32-token chunks and in
+ * fp64 across chunks; Cholesky solve (fp64) for F_hat^T; cyclic Jacobi eigen-decomposition
+ * (fp64) of the m x m matrix F_hat^T F_hat, whose eigenvectors are U and whose eigenvalues are
+ * S^2; Q_l = S_r^-1 U_r^T F_hat^T.  Singular values below 1e-12 sigma_1 count as zero.  If
+ * E^T E + beta I is not positive definite in floating point (beta below the rounding level
+ * of E^T E), LOCA_ERR_NUMERIC is written to the device status word and that block's P, Q and
+ * sigma are zero.
  */
 int loca_calib_fit_workspace_size(int64_t Np, int32_t m, int64_t d, int32_t L, int32_t r,
                                   size_t* bytes /* host */);

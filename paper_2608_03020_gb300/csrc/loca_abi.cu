@@ -380,9 +380,10 @@ int loca_calib_fit(const float* E_probe, const float* G_probe, int64_t Np, int32
     return fail(LOCA_ERR_ALIGNMENT, "pointers must be 4-byte aligned");
   int rc = check_ws(workspace, workspace_bytes, calib_workspace_bytes(Np, m, d, L, r));
   if (rc != LOCA_OK) return rc;
+  int32_t* status = device_status_word();
+  if (!status) return fail(LOCA_ERR_CUDA, "cannot resolve the device status word");
   cudaError_t e = launch_calib_fit(E_probe, G_probe, Np, m, d, L, beta, r, P, Q, sigma, workspace,
-                                   static_cast<cudaStream_t>(stream));
-  if (e == cudaErrorNotSupported) return fail(LOCA_ERR_UNSUPPORTED, "calibration fit is not built");
+                                   status, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "loca_calib_fit launch");
   return LOCA_OK;
 }

@@ -59,6 +59,6 @@ cudaError_t launch_chol_solve(const float* GA, const float* CA, const float* A, 
 size_t calib_workspace_bytes(int64_t Np, int m, int64_t d, int L, int r);
 cudaError_t launch_calib_fit(const float* E_probe, const float* G_probe, int64_t Np, int m,
                              int64_t d, int L, float beta, int r, float* P, float* Q, float* sigma,
-                             void* workspace, cudaStream_t s);
+                             void* workspace, int32_t* status, cudaStream_t s);
 
 }  // namespace loca

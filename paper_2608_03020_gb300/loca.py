@@ -23,7 +23,7 @@ LOCA_BF16 = 1
 STATUS_NAMES = {
     0: "LOCA_OK", 1: "LOCA_ERR_INVALID_ARG", 2: "LOCA_ERR_SHAPE", 3: "LOCA_ERR_ALIGNMENT",
     4: "LOCA_ERR_UNSUPPORTED_DTYPE", 5: "LOCA_ERR_CUDA", 6: "LOCA_ERR_TIMEOUT",
-    7: "LOCA_ERR_WORKSPACE", 8: "LOCA_ERR_UNSUPPORTED",
+    7: "LOCA_ERR_WORKSPACE", 8: "LOCA_ERR_UNSUPPORTED", 9: "LOCA_ERR_NUMERIC",
 }
 
 # (name, restype, argtypes) of every exported entry point
@@ -140,9 +140,12 @@ def loca_device_status(stream=None) -> int:
 
 def loca_error(logits, label_cols, y, E, w=None, ce=None, normaliser=0, stream=None):
     """Top-layer error at the head: fills ``E`` (N x C float) and optionally ``ce`` (N)."""
-    _dev(logits, "logits", (torch.float32, torch.bfloat16))
-    if logits.dim() != 2 or logits.stride(1) != 1:
-        raise ValueError("logits must be a 2-D row-major tensor (unit column stride)")
+    if not isinstance(logits, torch.Tensor) or not logits.is_cuda:
+        raise TypeError("logits must be a CUDA tensor")
+    if logits.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError(f"logits has dtype {logits.dtype}, expected float32 or bfloat16")
+    if logits.dim() != 2 or logits.stride(1) != 1 or logits.stride(0) < logits.shape[1]:
+        raise ValueError("logits must be 2-D with unit column stride and row pitch >= V")
     _dev(label_cols, "label_cols", torch.int32, 1)
     _dev(y, "y", torch.int32, 1)
     _dev(E, "E", torch.float32, 2)

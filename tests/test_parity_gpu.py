@@ -180,7 +180,9 @@ def test_accumulate_parity(lc, dtype, L, d, batches):
     rg, rc = _rel(_np(gram), g_ref), _rel(_np(cross), c_ref)
     print(f"rel err gram {rg:.3e} cross {rc:.3e}")
     assert rg <= tol and rc <= tol
-    assert np.allclose(_np(xsq), x_ref, rtol=1e-12, atol=0)
+    # f32 path: fp64 sums (1e-12).  bf16 path: exact squares summed in fp32 partials of at most
+    # 32 terms, partials summed in fp64: relative error <= 32 * 2^-24 < 2e-6.
+    assert np.allclose(_np(xsq), x_ref, rtol=1e-12 if dtype == "f32" else 2e-6, atol=0)
     gg = _np(gram)
     assert np.array_equal(gg, np.transpose(gg, (0, 2, 1)))  # both halves written, identical
     if dtype == "bf16":
@@ -329,5 +331,5 @@ def test_end_to_end_bf16_small(lc, batches, prev):
     rb = max(_rel(_np(ps.B)[j, l], ref["B"][j, l]) for j in range(len(w.lambda_rel)) for l in range(w.L))
     print(f"rel err gram {rg:.2e} cross {rc:.2e} B {rb:.2e}")
     assert rg < 2e-3 and rc < 2e-3 and rb < 2e-3
-    assert np.allclose(_np(ps.xsq), ref["xsq_total"], rtol=1e-12)
+    assert np.allclose(_np(ps.xsq), ref["xsq_total"], rtol=2e-6)
     assert lc.loca_device_status() == 0
