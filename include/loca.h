@@ -167,6 +167,31 @@ int loca_gram_cross(const void* X, const void* T, int dtype, int32_t L, int64_t 
                     size_t workspace_bytes, void* stream);
 
 /*
+ * loca_accumulate_noalloc — loca_accumulate for callers that cannot provide device scratch
+ * memory.  The paper has no counterpart: it concerns only how this library obtains scratch.
+ *
+ * Some callers cannot allocate device memory when they call the library: a program whose
+ * device memory is reserved up front by another owner (an inference server, a plugin host
+ * that exposes no allocator), or a caller that must not call cudaMalloc on its hot loop
+ * because the call can synchronise the device and take an unbounded time.  This entry point
+ * allocates nothing: its scratch (partial sums of ||X_l||^2, the steps alpha_l and a wait
+ * flag; 524,800 bytes) is a fixed array in the library's device memory that every GPU which
+ * loads the library holds until the process exits.  Arguments, outputs and results are
+ * those of loca_accumulate, without the workspace.
+ *
+ * Limits and use:
+ *  - L <= 64 blocks; a larger L is rejected with LOCA_ERR_SHAPE (use loca_accumulate).
+ *  - The first call on each device looks up the array's device address (cudaGetSymbolAddress,
+ *    with that device current) and caches it; make that first call before any stream capture.
+ *  - Every call reuses the same array.  Calls whose work may overlap on the GPU (different
+ *    streams, or threads without ordering between them) race on it: serialise them.
+ *  - Calls no cudaMalloc, cudaFree or other allocating routine.
+ */
+int loca_accumulate_noalloc(const void* X, const void* T, int dtype, int32_t L, int64_t N, int64_t d,
+                            const double* tsq, float eta, int zero_first, float* gram, float* cross,
+                            double* xsq_total, void* stream);
+
+/*
  * loca_ridge_solve — closed-form block minimisers for every block l and every ridge
  * candidate j (Eq. 8; Theorem S6; positive-definite solve without an inverse, S7):
  *

@@ -34,6 +34,14 @@ constexpr int kMaxDevices = 64;
 
 }  // namespace
 
+int set_error_message(int code, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_msg, sizeof(g_msg), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
 int sm_count() {
   static int cache[kMaxDevices] = {};
   int dev = 0;

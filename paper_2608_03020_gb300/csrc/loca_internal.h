@@ -16,6 +16,9 @@ int sm_count();
 // loca_device_status); resolved once per device with that device current.
 int32_t* device_status_word();
 
+// Record the message loca_last_error_string() returns for the calling thread; returns `code`.
+int set_error_message(int code, const char* fmt, ...);
+
 // Bytes needed to round `n` up to a 256-byte boundary.
 inline size_t align256(size_t n) { return (n + 255) & ~size_t(255); }
 

@@ -42,6 +42,8 @@ SIGNATURES = [
     ("loca_accumulate_workspace_size", ctypes.c_int, [_I32, _I64, _I64, ctypes.c_int, ctypes.POINTER(_SZ)]),
     ("loca_accumulate", ctypes.c_int,
      [_P, _P, ctypes.c_int, _I32, _I64, _I64, _P, _F, ctypes.c_int, _P, _P, _P, _P, _SZ, _P]),
+    ("loca_accumulate_noalloc", ctypes.c_int,
+     [_P, _P, ctypes.c_int, _I32, _I64, _I64, _P, _F, ctypes.c_int, _P, _P, _P, _P]),
     ("loca_batch_step_workspace_size", ctypes.c_int, [_I32, ctypes.POINTER(_SZ)]),
     ("loca_batch_step", ctypes.c_int, [_P, ctypes.c_int, _I32, _I64, _I64, _P, _F, ctypes.c_int, _P, _P, _P, _SZ, _P]),
     ("loca_gram_cross_workspace_size", ctypes.c_int, [ctypes.POINTER(_SZ)]),
@@ -212,6 +214,25 @@ def loca_accumulate(X, T, tsq, eta, gram, cross, xsq_total, zero_first, workspac
     rc = lib().loca_accumulate(_ptr(X), _ptr(T), _code(X.dtype), L, N, d, _ptr(tsq), float(eta), int(bool(zero_first)),
                                _ptr(gram), _ptr(cross), _ptr(xsq_total), _ptr(ws), nbytes, _stream(stream))
     _check(rc, "loca_accumulate")
+
+
+def loca_accumulate_noalloc(X, T, tsq, eta, gram, cross, xsq_total, zero_first, stream=None):
+    """loca_accumulate without a workspace, for callers that cannot allocate device memory when
+    they call the library; its scratch is a fixed array inside the library (L <= 64 blocks).
+    Calls that may overlap on the GPU share that array and must be serialised."""
+    _dev(X, "X", (torch.float32, torch.bfloat16), 3)
+    _dev(T, "T", X.dtype, 3)
+    _dev(tsq, "tsq", torch.float64, 1)
+    _dev(gram, "gram", torch.float32, 3)
+    _dev(cross, "cross", torch.float32, 3)
+    _dev(xsq_total, "xsq_total", torch.float64, 1)
+    L, N, d = X.shape
+    if tuple(T.shape) != (L, N, d) or tuple(gram.shape) != (L, d, d) or tuple(cross.shape) != (L, d, d):
+        raise ValueError("shape mismatch among X, T (L x N x d) and gram, cross (L x d x d)")
+    rc = lib().loca_accumulate_noalloc(_ptr(X), _ptr(T), _code(X.dtype), L, N, d, _ptr(tsq), float(eta),
+                                       int(bool(zero_first)), _ptr(gram), _ptr(cross), _ptr(xsq_total),
+                                       _stream(stream))
+    _check(rc, "loca_accumulate_noalloc")
 
 
 def batch_step_workspace_size(L) -> int:
