@@ -53,6 +53,8 @@ def parse():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--workload", default="qwen2.5-7b")
+    ap.add_argument("--L", type=int, default=None, help="override the workload's block count")
+    ap.add_argument("--N", type=int, default=None, help="override the workload's token count")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -217,6 +219,8 @@ def main():
     from synth import inputs as S
 
     w = S.WORKLOADS[args.workload]
+    if args.L is not None or args.N is not None:
+        w = S.scaled(w, L=args.L or w.L, N=args.N or w.N)
     if args.impl == "reference":
         rank = int(os.environ.get("RANK", "0"))
         if rank == 0:
