@@ -111,7 +111,8 @@ int loca_error(const void* logits, int logit_dtype, int64_t N, int64_t V, int64_
  *      each value is computed in fp32 and rounded once (round to nearest even)
  * tsq  L double output ||T_l||_F^2 of the unrounded fp32 values, or NULL
  *      (then no workspace is needed)
- * r in [1, 64], C in [1, 1024].  Deterministic: partial sums are reduced in a fixed order.
+ * r in [1, 64], C in [1, 64].  Deterministic: partial sums are reduced in a fixed order;
+ * ||T_l||^2 is formed as sum_n u_n^T (Q_l Q_l^T) u_n with u_n = E[n] P_l.
  */
 int loca_targets_workspace_size(int64_t N, int32_t L, int64_t d, size_t* bytes /* host */);
 int loca_targets(const float* E, int64_t N, int32_t C, const float* P, const float* Q,

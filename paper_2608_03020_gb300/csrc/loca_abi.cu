@@ -80,9 +80,10 @@ struct TargetsWs {
   size_t partials, total;
 };
 TargetsWs targets_ws(int64_t N, int32_t L, int64_t d) {
+  (void)d;
   TargetsWs w{};
   w.partials = 0;
-  w.total = align256(sizeof(double) * size_t(L) * size_t(targets_num_partials(N, d)));
+  w.total = targets_workspace_bytes(N, L, 64);  // sized for the largest feedback rank
   return w;
 }
 
@@ -174,7 +175,7 @@ int loca_targets(const float* E, int64_t N, int32_t C, const float* P, const flo
                  size_t workspace_bytes, void* stream) {
   g_msg[0] = 0;
   if (N < 0 || L < 1 || L > 65535 || d < 1) return fail(LOCA_ERR_SHAPE, "need N >= 0, 1 <= L <= 65535, d >= 1");
-  if (C < 1 || C > 1024) return fail(LOCA_ERR_SHAPE, "need 1 <= C <= 1024");
+  if (C < 1 || C > targets_max_C()) return fail(LOCA_ERR_SHAPE, "need 1 <= C <= %d, got C=%d", targets_max_C(), C);
   if (r < 1 || r > 64) return fail(LOCA_ERR_SHAPE, "need 1 <= r <= 64, got %d", r);
   if (t_dtype != LOCA_F32 && t_dtype != LOCA_BF16)
     return fail(LOCA_ERR_UNSUPPORTED_DTYPE, "t_dtype must be LOCA_F32 or LOCA_BF16");
@@ -187,8 +188,7 @@ int loca_targets(const float* E, int64_t N, int32_t C, const float* P, const flo
     const int rc = check_ws(workspace, workspace_bytes, targets_ws(N, L, d).total);
     if (rc != LOCA_OK) return rc;
   }
-  cudaError_t e = launch_targets(E, N, C, P, Q, L, r, d, T, t_dtype, tsq,
-                                 tsq ? reinterpret_cast<double*>(ws_at(workspace, 0)) : nullptr,
+  cudaError_t e = launch_targets(E, N, C, P, Q, L, r, d, T, t_dtype, tsq, tsq ? workspace : nullptr,
                                  static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "loca_targets launch");
   return LOCA_OK;

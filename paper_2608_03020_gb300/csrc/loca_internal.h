@@ -28,12 +28,14 @@ cudaError_t launch_head_error(const void* z, int dtype, int64_t N, int64_t V, in
                               int normaliser, float* E, float* ce, cudaStream_t s);
 
 // ---- feedback targets (targets.cu)
-// Grid geometry used by launch_targets; partial sums of ||T_l||^2 live in
-// `partials` (L x targets_num_partials(N, d) doubles).
+// Workspace: partial sums of ||T_l||^2 (L x targets_num_partials(N, d) doubles) followed by
+// M_l = Q_l Q_l^T (L x r x r floats); targets_workspace_bytes gives the total.
 int64_t targets_num_partials(int64_t N, int64_t d);
+size_t targets_workspace_bytes(int64_t N, int L, int r);
+int targets_max_C();
 cudaError_t launch_targets(const float* E, int64_t N, int C, const float* P, const float* Q,
                            int L, int r, int64_t d, void* T, int t_dtype, double* tsq,
-                           double* partials, cudaStream_t s);
+                           void* workspace, cudaStream_t s);
 
 // ---- statistics (stats.cu, gram_tc.cu)
 // Sum of squares of X (per block) and the step alpha_l; partials: L x sumsq_num_partials().

@@ -56,7 +56,7 @@ def _ws(fn, *args):
 
 def test_workspace_sizes(L):
     rc, n = _ws(L.loca_targets_workspace_size, 131072, 28, 3584)
-    assert rc == 0 and n >= 8 * 28 * (131072 // 64) * 14 and n % 256 == 0
+    assert rc == 0 and n >= 8 * 28 * (131072 // 1024) + 4 * 28 * 64 * 64 and n % 256 == 0
     rc, n = _ws(L.loca_accumulate_workspace_size, 28, 131072, 3584, 1)
     assert rc == 0 and n > 0
     rc, n = _ws(L.loca_ridge_solve_workspace_size, 28, 3584, 16)
