@@ -43,7 +43,8 @@ FALLBACK_SUSTAINED_TFLOPS = 1700.0  # profiling recipe's sustained figure, used 
 
 # dram bytes per launch of k_gram_cross_tc from an ncu capture (see profiles/), valid only for
 # the kernel source whose sha256 prefix is given; otherwise traffic is reported as null
-GRAM_TC_TRAFFIC = {"sha256": None, "bytes_per_unit": None, "unit": None}
+GRAM_TC_TRAFFIC = {"sha256": "4c359b83e81645d7", "read_per_token_block": 39725.0,
+                   "write_per_block": 91.047e6, "source": "profiles/gram_cross_tc_qwen2.5-7b.md"}
 
 
 def parse():
@@ -324,8 +325,9 @@ def main():
     src = open(os.path.join(ROOT, "paper_2608_03020_gb300", "csrc", "gram_tc.cu"), "rb").read()
     sha = hashlib.sha256(src).hexdigest()[:16]
     traffic = None
-    if GRAM_TC_TRAFFIC["sha256"] == sha and GRAM_TC_TRAFFIC["bytes_per_unit"] is not None:
-        traffic = GRAM_TC_TRAFFIC["bytes_per_unit"] * L  # bytes per launch
+    if GRAM_TC_TRAFFIC["sha256"] == sha:
+        # dram bytes per launch, scaled from a smaller ncu capture of the same kernel source
+        traffic = GRAM_TC_TRAFFIC["read_per_token_block"] * L * N + GRAM_TC_TRAFFIC["write_per_block"] * L
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "traffic": traffic, "kernel": "k_gram_cross_tc",
                 "peak_kind": f"bf16 dense sustained, {peak_kind}", "flops_per_launch": flops}
