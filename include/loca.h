@@ -107,12 +107,12 @@ int loca_error(const void* logits, int logit_dtype, int64_t N, int64_t V, int64_
  *
  * E    N x C float (from loca_error)
  * P    L x C x r float, Q  L x r x d float (feedback factors, e.g. from loca_calib_fit)
- * T    L x N x d output, t_dtype LOCA_BF16 (the tensor-core feed) or LOCA_F32;
- *      each value is computed in fp32 and rounded once (round to nearest even)
- * tsq  L double output ||T_l||_F^2 of the unrounded fp32 values, or NULL
- *      (then no workspace is needed)
- * r in [1, 64], C in [1, 64].  Deterministic: partial sums are reduced in a fixed order;
- * ||T_l||^2 is formed as sum_n u_n^T (Q_l Q_l^T) u_n with u_n = E[n] P_l.
+ * T    L x N x d output, t_dtype LOCA_BF16 (the tensor-core feed) or LOCA_F32; 16-byte aligned
+ * tsq  L double output ||T_l||_F^2 of the fp32 values before rounding, or NULL
+ * Arithmetic: u = E[n] P_l in fp32; U Q_l on the tensor cores (tcgen05, kind::tf32) as
+ * hi*hi + hi*lo + lo*hi of tf32 splits with fp32 accumulation (fp32-accurate); one rounding
+ * to the output type.  r in [1, 32], C in [1, 64].  A workspace is always required (it also
+ * holds a launch-local wait flag).  Deterministic: partial sums are reduced in a fixed order.
  */
 int loca_targets_workspace_size(int64_t N, int32_t L, int64_t d, size_t* bytes /* host */);
 int loca_targets(const float* E, int64_t N, int32_t C, const float* P, const float* Q,

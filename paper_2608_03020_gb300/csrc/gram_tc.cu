@@ -25,6 +25,7 @@
 #include <mutex>
 
 #include "loca_internal.h"
+#include "tc_ptx.cuh"
 
 namespace loca {
 namespace {
@@ -42,121 +43,9 @@ constexpr int NUM_THREADS = 192;
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /* align slack */ + 256 /* barriers */;
 
 // Instruction descriptor (kind::f16): D fp32, A bf16, B bf16, A and B MN-major, N, M.
-constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | (1u << 16) |
-                           (uint32_t(BN >> 3) << 17) | (uint32_t(BM >> 4) << 24);
+constexpr uint32_t IDESC = tc::idesc(1, 1, 1, 1, BM, BN);
 
-// ------------------------------------------------------------------ PTX wrappers
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ uint64_t globaltimer() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-      " selp.u32 %0, 1, 0, p;\n}\n"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
-struct WaitCtl {
-  int32_t* status;               // library status word (sticky error code)
-  volatile int32_t* abort_flag;  // launch-local: set by the first CTA that gives up
-  uint64_t limit_ns;
-};
-
-// Bounded wait for the phase of parity `parity` of barrier `bar`.  Returns false when the wait
-// gave up (time limit reached, or another waiter of this launch gave up).
-__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const WaitCtl& w) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer();
-  for (uint32_t it = 1;; ++it) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 255u) == 0) {
-      if (*w.abort_flag != 0) return false;
-      if (globaltimer() - t0 > w.limit_ns) {
-        atomicExch(w.status, int32_t(LOCA_ERR_TIMEOUT));
-        *w.abort_flag = 1;
-        __threadfence();
-        return false;
-      }
-    }
-  }
-}
-
-__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
-                                            int c0, int c1, int c2) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2)
-      : "memory");
-}
-
-// Shared-memory matrix descriptor, 128-byte swizzle, MN-major canonical layout:
-// LBO = byte distance between 64-element MN blocks, SBO = byte distance between 8-row K groups.
-__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
-  uint64_t d = 0;
-  d |= uint64_t((saddr >> 4) & 0x3FFFu);
-  d |= uint64_t((lbo >> 4) & 0x3FFFu) << 16;
-  d |= uint64_t((sbo >> 4) & 0x3FFFu) << 32;
-  d |= uint64_t(1) << 46;  // descriptor version for tcgen05
-  d |= uint64_t(2) << 61;  // 128-byte swizzle
-  return d;
-}
-
-__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
-                                          uint32_t accumulate) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
-      "l"(adesc), "l"(bdesc), "r"(IDESC), "r"(accumulate));
-}
-__device__ __forceinline__ void umma_commit(uint32_t bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                   bar)
-               : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-
-// 32 lanes x 32 consecutive fp32 columns: thread t of the warp gets row (lane base + t).
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
-      "%12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, "
-      "%30, %31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
-        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
-        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
+using namespace tc;
 
 // ------------------------------------------------------------------ work items
 struct Geo {
@@ -237,20 +126,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     mbar_init(acc_full, 1);
     mbar_init(acc_empty, 128);
     mbar_init(drain_bar, 1);
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmX)) : "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmT)) : "memory");
+    mbar_init_fence();
+    prefetch_tensormap(&tmX);
+    prefetch_tensormap(&tmT);
   }
-  if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                     smem_u32(tmem_slot)),
-                 "r"(TMEM_COLS)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-  }
-  tc_fence_before();
+  if (warp == 1) tmem_alloc(smem_u32(tmem_slot), TMEM_COLS);
+  fence_before();
   __syncthreads();
-  tc_fence_after();
+  fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const int nkb = (g.N + BK - 1) / BK;
 
@@ -307,31 +190,31 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       for (int it = blockIdx.x; it < total_items && ok; it += gridDim.x) {
         const Item w = decode(g, it);
         if (!mbar_wait(acc_empty, acc_phase ^ 1u, wc)) { ok = false; break; }
-        tc_fence_after();
+        fence_after();
         for (int kb = 0; kb < nkb; ++kb) {
           if (!mbar_wait(full_bar(stage), phase, wc)) { ok = false; break; }
-          tc_fence_after();
+          fence_after();
           const uint32_t st = smem_base + uint32_t(stage) * STAGE_BYTES;
           const uint32_t bsm = st + 2u * A_BYTES;
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk) {
-            const uint64_t bd = sdesc(bsm + uint32_t(kk) * 2048u, SUB_BYTES, 1024u);
+            const uint64_t bd = sdesc(bsm + uint32_t(kk) * 2048u, SUB_BYTES, 1024u, kSwizzle128B);
             for (int s = 0; s < w.nslots; ++s) {
               const uint64_t ad = sdesc(st + uint32_t(s) * A_BYTES + uint32_t(kk) * 2048u,
-                                        SUB_BYTES, 1024u);
-              umma_bf16(tmem_base + uint32_t(s) * BN, ad, bd, (kb | kk) != 0 ? 1u : 0u);
+                                        SUB_BYTES, 1024u, kSwizzle128B);
+              mma_f16(tmem_base + uint32_t(s) * BN, ad, bd, IDESC, (kb | kk) != 0 ? 1u : 0u);
             }
           }
           issued = true;
-          umma_commit(empty_bar(stage));  // frees the stage once these MMAs have read it
+          mma_commit(empty_bar(stage));  // frees the stage once these MMAs have read it
           if (++stage == STAGES) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
-        umma_commit(acc_full);  // accumulators complete
+        mma_commit(acc_full);  // accumulators complete
         acc_phase ^= 1u;
       }
       if (!ok && issued) {
-        umma_commit(drain_bar);
+        mma_commit(drain_bar);
         const uint64_t t0 = globaltimer();
         while (!mbar_try_wait(drain_bar, 0)) {
           if (globaltimer() - t0 > limit_ns) break;
@@ -348,7 +231,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const Item w = decode(g, it);
       const bool ok = mbar_wait(acc_full, acc_phase, wc);
       if (!__all_sync(0xffffffffu, ok)) break;  // warp-uniform decision, warp reconverged
-      tc_fence_after();
+      fence_after();
       const float al = alpha[w.l];
       for (int s = 0; s < w.nslots; ++s) {
         const bool is_gram = w.kind[s] == 0;
@@ -399,39 +282,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
         }
       }
-      tc_fence_before();
+      fence_before();
       mbar_arrive(acc_empty);
       acc_phase ^= 1u;
     }
   }
 
-  tc_fence_before();
+  fence_before();
   __syncthreads();
-  tc_fence_after();
-  if (warp == 1) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
-                 "r"(TMEM_COLS)
-                 : "memory");
-  }
+  fence_after();
+  if (warp == 1) tmem_dealloc(tmem_base, TMEM_COLS);
 }
 
 // ------------------------------------------------------------------ host side
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  });
-  return fn;
-}
-
 bool make_map(CUtensorMap* m, const void* base, int L, int64_t N, int64_t d) {
-  auto fn = encode_fn();
+  auto fn = tensor_map_encoder();
   if (!fn) return false;
   cuuint64_t dims[3] = {cuuint64_t(d), cuuint64_t(N), cuuint64_t(L)};
   cuuint64_t strides[2] = {cuuint64_t(d) * 2, cuuint64_t(N) * cuuint64_t(d) * 2};

@@ -34,6 +34,20 @@ constexpr int kMaxDevices = 64;
 
 }  // namespace
 
+TensorMapEncodeFn tensor_map_encoder() {
+  static TensorMapEncodeFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<TensorMapEncodeFn>(p);
+  });
+  return fn;
+}
+
 int set_error_message(int code, const char* fmt, ...) {
   va_list ap;
   va_start(ap, fmt);
@@ -80,10 +94,9 @@ struct TargetsWs {
   size_t partials, total;
 };
 TargetsWs targets_ws(int64_t N, int32_t L, int64_t d) {
-  (void)d;
   TargetsWs w{};
   w.partials = 0;
-  w.total = targets_workspace_bytes(N, L, 64);  // sized for the largest feedback rank
+  w.total = targets_workspace_bytes(N, L, d);
   return w;
 }
 
@@ -176,7 +189,7 @@ int loca_targets(const float* E, int64_t N, int32_t C, const float* P, const flo
   g_msg[0] = 0;
   if (N < 0 || L < 1 || L > 65535 || d < 1) return fail(LOCA_ERR_SHAPE, "need N >= 0, 1 <= L <= 65535, d >= 1");
   if (C < 1 || C > targets_max_C()) return fail(LOCA_ERR_SHAPE, "need 1 <= C <= %d, got C=%d", targets_max_C(), C);
-  if (r < 1 || r > 64) return fail(LOCA_ERR_SHAPE, "need 1 <= r <= 64, got %d", r);
+  if (r < 1 || r > targets_max_r()) return fail(LOCA_ERR_SHAPE, "need 1 <= r <= %d, got %d", targets_max_r(), r);
   if (t_dtype != LOCA_F32 && t_dtype != LOCA_BF16)
     return fail(LOCA_ERR_UNSUPPORTED_DTYPE, "t_dtype must be LOCA_F32 or LOCA_BF16");
   if ((N > 0 && (!E || !T)) || !P || !Q) return fail(LOCA_ERR_INVALID_ARG, "E, P, Q and T are required");
@@ -184,11 +197,11 @@ int loca_targets(const float* E, int64_t N, int32_t C, const float* P, const flo
   if (!aligned(E, 4) || !aligned(P, 4) || !aligned(Q, 4) || !aligned(T, 16) || (tsq && !aligned(tsq, 8)))
     return fail(LOCA_ERR_ALIGNMENT, "E, P, Q need 4-byte, T 16-byte and tsq 8-byte alignment");
   (void)es;
-  if (tsq) {
-    const int rc = check_ws(workspace, workspace_bytes, targets_ws(N, L, d).total);
-    if (rc != LOCA_OK) return rc;
-  }
-  cudaError_t e = launch_targets(E, N, C, P, Q, L, r, d, T, t_dtype, tsq, tsq ? workspace : nullptr,
+  const int rc = check_ws(workspace, workspace_bytes, targets_ws(N, L, d).total);
+  if (rc != LOCA_OK) return rc;
+  int32_t* status = device_status_word();
+  if (!status) return fail(LOCA_ERR_CUDA, "cannot resolve the device status word");
+  cudaError_t e = launch_targets(E, N, C, P, Q, L, r, d, T, t_dtype, tsq, workspace, status,
                                  static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "loca_targets launch");
   return LOCA_OK;

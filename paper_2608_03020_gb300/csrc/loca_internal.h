@@ -1,6 +1,7 @@
 // Internal declarations shared by the library's translation units (host side).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -16,6 +17,13 @@ int sm_count();
 // loca_device_status); resolved once per device with that device current.
 int32_t* device_status_word();
 
+// cuTensorMapEncodeTiled from the driver (looked up once), or nullptr.
+typedef CUresult (*TensorMapEncodeFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                      const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                      const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                      CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+TensorMapEncodeFn tensor_map_encoder();
+
 // Record the message loca_last_error_string() returns for the calling thread; returns `code`.
 int set_error_message(int code, const char* fmt, ...);
 
@@ -28,14 +36,15 @@ cudaError_t launch_head_error(const void* z, int dtype, int64_t N, int64_t V, in
                               int normaliser, float* E, float* ce, cudaStream_t s);
 
 // ---- feedback targets (targets.cu)
-// Workspace: partial sums of ||T_l||^2 (L x targets_num_partials(N, d) doubles) followed by
-// M_l = Q_l Q_l^T (L x r x r floats); targets_workspace_bytes gives the total.
+// Workspace: partial sums of ||T_l||^2 (L x targets_num_partials(N, d) doubles) and a
+// launch-local wait flag; targets_workspace_bytes gives the total.
 int64_t targets_num_partials(int64_t N, int64_t d);
-size_t targets_workspace_bytes(int64_t N, int L, int r);
+size_t targets_workspace_bytes(int64_t N, int L, int64_t d);
 int targets_max_C();
+int targets_max_r();
 cudaError_t launch_targets(const float* E, int64_t N, int C, const float* P, const float* Q,
                            int L, int r, int64_t d, void* T, int t_dtype, double* tsq,
-                           void* workspace, cudaStream_t s);
+                           void* workspace, int32_t* status, cudaStream_t s);
 
 // ---- statistics (stats.cu, gram_tc.cu)
 // Sum of squares of X (per block) and the step alpha_l; partials: L x sumsq_num_partials().

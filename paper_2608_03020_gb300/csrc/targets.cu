@@ -1,270 +1,453 @@
 // Tokenwise feedback predictions of every block (S3: Q_l := F_l E), applied through the
-// low-rank factors (S11: F e = U_k (S_k (V_k^T e))):  T_l = (E P_l) Q_l.
+// low-rank factors (S11: F e = U_k (S_k (V_k^T e))):  T_l = (E P_l) Q_l,  on the tensor cores.
 //
-// k_qqt        M_l = Q_l Q_l^T (r x r), so that ||T_l||^2 = sum_n u_n^T M_l u_n with u_n = E[n] P_l.
-// k_targets    persistent; a work item is (block l, 256-channel tile, 1024-token chunk).  The
-//              tile Q_l[:, j0:j0+256] stays in shared memory for the item; for each 64-token
-//              tile the E rows (prefetched into registers one tile ahead) give U = E P_l
-//              (64 x r) in shared memory, and each thread forms an 8 token x 8 channel register
-//              tile of T = U Q_l (fp32 FMA), rounds once to the output type and stores it (a
-//              warp writes two runs of 256 contiguous bytes per token row in bf16).  Items of
-//              channel tile 0 also
-//              reduce u^T M_l u over their tokens into one partial; a second kernel sums the
-//              partials in a fixed order (deterministic).
-// Bound: 2 r fp32 FMA-flops per output element and 2 (bf16) or 4 (fp32) output bytes: at
-// r = 16 with bf16 output the FMA pipe (~128 FMA/clk/SM) is the limit, not HBM.
+// The product U Q_l has inner dimension r (4..32), so it is a short tcgen05 MMA per output
+// tile; the kernel is bound by the HBM write of T (2 bytes per element in bf16).  Precision:
+// U and Q are split into tf32 pairs (hi = rna(x), lo = rna(x - hi)) and the tile is
+// hi*hi + hi*lo + lo*hi with fp32 accumulation (kind::tf32), ~2^-20 relative per product, so
+// the fp32 output matches an fp32 FMA evaluation.
+//
+// Persistent, one CTA per SM, 288 threads:
+//   warps 0-3   producers: per item load Q_l[:, 256-channel tile], split it into hi/lo K-major
+//               tiles (B); per 128-token tile, thread i forms u = E[n0 + i] P_l (fp32), splits
+//               it and writes its row of the A tiles (double-buffered).
+//   warp 8      owns 512 TMEM columns (two 128 x 256 fp32 accumulators) and issues the MMAs.
+//   warps 4-7   epilogue: tcgen05.ld, sum of squares of the fp32 values (||T_l||^2), rounding
+//               to the output type; in bf16 each warp stages its 32 token rows in shared
+//               memory (128-byte swizzled boxes) and writes them with TMA bulk tensor stores,
+//               so HBM sees whole lines; fp32 output uses plain stores (one row per thread).
+// Work item = (block l, 256-channel tile, 4096-token chunk); ||T_l||^2 partials are written
+// per item and epilogue warp and summed in a fixed order by k_reduce_partials
+// (deterministic).  All waits are bounded (see tc_ptx.cuh) and no warp waits on another
+// warp except through those bounded mbarrier waits.
 #include <cuda_bf16.h>
 
+#include <cstring>
+
 #include "loca_internal.h"
+#include "tc_ptx.cuh"
 
 namespace loca {
 namespace {
 
-constexpr int TN = 64;         // tokens per tile
-constexpr int TD = 256;        // channels per tile
-constexpr int CHUNK = 1024;    // tokens per work item
-constexpr int kMaxC = 64;      // label columns supported by the fused U stage
+using namespace tc;
+
+constexpr int TM = 128;           // tokens per tile (TMEM lanes)
+constexpr int TCH = 256;          // channels per tile (TMEM columns per accumulator)
+constexpr int CHUNK_TILES = 32;   // tiles per work item
+constexpr int CHUNK = TM * CHUNK_TILES;
+constexpr int kMaxC = 64;
+constexpr int kMaxRP = 32;        // padded feedback rank (multiple of 8)
+constexpr int NTHREADS = 288;
+constexpr uint32_t TMEM_COLS = 512;
+constexpr uint32_t ID_TF32 = idesc(2, 2, 0, 0, TM, TCH);
+
+constexpr uint32_t STAGE_WARP = 32 * TCH * 2;  // one epilogue warp's 32 x 256 bf16 rows (16 KB)
+
+struct Layout {
+  uint32_t stage, b_hi, b_lo, a_hi[2], a_lo[2], bars, total;
+};
+__host__ __device__ inline Layout layout_for(int rp) {
+  Layout o;
+  const uint32_t b = uint32_t(TCH) * rp * 4, a = uint32_t(TM) * rp * 4;
+  o.stage = 0;  // 4 x 16 KB, 1024-byte aligned (128-byte swizzled TMA boxes)
+  const uint32_t base = 4 * STAGE_WARP;
+  o.b_hi = base;
+  o.b_lo = base + b;
+  o.a_hi[0] = base + 2 * b;
+  o.a_lo[0] = base + 2 * b + a;
+  o.a_hi[1] = base + 2 * b + 2 * a;
+  o.a_lo[1] = base + 2 * b + 3 * a;
+  o.bars = base + 2 * b + 4 * a;
+  o.total = o.bars + 256 + 1024;  // + alignment slack
+  // at least 120 KB so that one CTA (which takes all 512 TMEM columns) sits on each SM
+  if (o.total < 120u * 1024u) o.total = 120u * 1024u;
+  return o;
+}
+
+// byte offset of element (row m, k s) in a K-major, no-swizzle canonical tile with rp columns:
+// 8-row x 16-byte core matrices, K-adjacent ones 128 bytes apart, 8-row groups rp*32 bytes apart
+__device__ __forceinline__ uint32_t kmaj_off(int m, int s, int rp) {
+  return uint32_t(m >> 3) * uint32_t(rp * 32) + uint32_t(s >> 2) * 128u + uint32_t(m & 7) * 16u +
+         uint32_t(s & 3) * 4u;
+}
+
+__device__ __forceinline__ uint32_t tf32_rna(float x) {
+  uint32_t y;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(y) : "f"(x));
+  return y;
+}
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
   return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-// M_l = Q_l Q_l^T, one thread block per block l.
-__global__ void __launch_bounds__(256) k_qqt(const float* __restrict__ Q, int r, int64_t d,
-                                             float* __restrict__ M) {
-  const int l = blockIdx.x;
-  const float* Ql = Q + int64_t(l) * r * d;
-  for (int e = threadIdx.x; e < r * r; e += 256) {
-    const int a = e / r, b = e % r;
-    if (b < a) continue;
-    const float* qa = Ql + int64_t(a) * d;
-    const float* qb = Ql + int64_t(b) * d;
-    double acc = 0.0;
-    float part = 0.f;
-    for (int64_t j = 0; j < d; ++j) {
-      part = fmaf(qa[j], qb[j], part);
-      if ((j & 63) == 63) { acc += part; part = 0.f; }
-    }
-    acc += part;
-    M[(int64_t(l) * r + a) * r + b] = float(acc);
-    M[(int64_t(l) * r + b) * r + a] = float(acc);
-  }
+struct Geo {
+  int64_t N, d;
+  int C, r, rp, L;
+  int64_t nd, nchunks, items;
+};
+
+__device__ __forceinline__ void decode(const Geo& g, int64_t it, int& l, int64_t& jt, int64_t& ck) {
+  l = int(it / (g.nd * g.nchunks));
+  const int64_t rem = it - int64_t(l) * g.nd * g.nchunks;
+  jt = rem / g.nchunks;
+  ck = rem - jt * g.nchunks;
 }
 
 template <bool kBF16>
-__global__ void __launch_bounds__(256, 2) k_targets(const float* __restrict__ E, int64_t N, int C,
-                                                    const float* __restrict__ P,
-                                                    const float* __restrict__ Q,
-                                                    const float* __restrict__ M, int r, int64_t d,
-                                                    int L, void* __restrict__ Tout,
-                                                    double* __restrict__ partials) {
-  extern __shared__ float smem[];
-  float* q_s = smem;                 // r x TD
-  float* u_s = q_s + r * TD;         // r x TN (transposed U tile)
-  float* e_s = u_s + TN * r;         // TN x C
-  float* p_s = e_s + TN * kMaxC;     // C x r
-  float* m_s = p_s + kMaxC * r;      // r x r
-  __shared__ double red[8];
-  const int t = threadIdx.x;
-  const int cg = t & 31, tg = t >> 5;
-  const int64_t nd = (d + TD - 1) / TD;
-  const int64_t nchunks = (N + CHUNK - 1) / CHUNK;
-  const int64_t items = int64_t(L) * nd * nchunks;
+__global__ void __launch_bounds__(NTHREADS, 1)
+    k_targets_tc(const float* __restrict__ E, const float* __restrict__ P, const float* __restrict__ Q,
+                 Geo g, void* __restrict__ Tout, const __grid_constant__ CUtensorMap tmT, int use_tma,
+                 double* __restrict__ partials, int32_t* status, int32_t* abort_flag,
+                 unsigned long long limit_ns) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  // 1024-byte aligned base: the 128-byte swizzle of the TMA boxes repeats every 1024 bytes
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const Layout lay = layout_for(g.rp);
+  const uint32_t sbase = smem_u32(smem);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + lay.bars);
+  // bars: a_full[2], a_empty[2], acc_full[2], acc_empty[2], b_full, b_empty, drain
+  const uint32_t bar0 = smem_u32(bars);
+  auto a_full = [&](int b) { return bar0 + 8u * b; };
+  auto a_empty = [&](int b) { return bar0 + 8u * (2 + b); };
+  auto acc_full = [&](int b) { return bar0 + 8u * (4 + b); };
+  auto acc_empty = [&](int b) { return bar0 + 8u * (6 + b); };
+  const uint32_t b_full = bar0 + 64, b_empty = bar0 + 72, drain_bar = bar0 + 80;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 11);
 
-  for (int64_t it = blockIdx.x; it < items; it += gridDim.x) {
-    const int l = int(it / (nd * nchunks));
-    const int64_t rem = it - int64_t(l) * nd * nchunks;
-    const int64_t jt = rem / nchunks;
-    const int64_t ck = rem - jt * nchunks;
-    const int64_t j0 = jt * TD;
-    const int64_t nbeg = ck * CHUNK;
-    const int64_t nend = (nbeg + CHUNK < N) ? nbeg + CHUNK : N;
-    const bool do_sq = (jt == 0) && partials != nullptr;
-    const float* Ql = Q + int64_t(l) * r * d;
-    const float* Pl = P + int64_t(l) * C * r;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const WaitCtl wc{status, abort_flag, limit_ns};
+  const int rp = g.rp, r = g.r, C = g.C;
 
-    __syncthreads();  // previous item's shared-memory readers are done
-    for (int e = t; e < r * TD; e += 256) {
-      const int s = e / TD, jj = e - s * TD;
-      q_s[e] = (j0 + jj < d) ? Ql[int64_t(s) * d + j0 + jj] : 0.f;
+  if (threadIdx.x == 0) {
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(a_full(b), 128);
+      mbar_init(a_empty(b), 1);
+      mbar_init(acc_full(b), 1);
+      mbar_init(acc_empty(b), 128);
     }
-    for (int e = t; e < C * r; e += 256) p_s[e] = Pl[e];
-    if (do_sq)
-      for (int e = t; e < r * r; e += 256) m_s[e] = M[int64_t(l) * r * r + e];
-    // E rows of the first tile
-    float ev[(TN * kMaxC) / 256];
-    const int nev = (TN * C + 255) / 256;
+    mbar_init(b_full, 128);
+    mbar_init(b_empty, 1);
+    mbar_init(drain_bar, 1);
+    mbar_init_fence();
+  }
+  if (warp == 8) tmem_alloc(smem_u32(tmem_slot), TMEM_COLS);
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp < 4) {
+    // ---------------- producers: thread i <-> tile row i
+    const int i = threadIdx.x;
+    uint32_t tcount = 0, icount = 0;
+    bool ok = true;
+    for (int64_t it = blockIdx.x; it < g.items && ok; it += gridDim.x, ++icount) {
+      int l;
+      int64_t jt, ck;
+      decode(g, it, l, jt, ck);
+      const int64_t j0 = jt * TCH;
+      const int64_t nbeg = ck * CHUNK;
+      const int64_t nend = (nbeg + CHUNK < g.N) ? nbeg + CHUNK : g.N;
+      if (!mbar_wait(b_empty, (icount & 1u) ^ 1u, wc)) { ok = false; break; }
+      // B = Q_l[:, j0 : j0 + 256] as hi/lo K-major tiles (channel = row, s = k)
+      const float* Ql = Q + int64_t(l) * r * g.d;
+      for (int h = 0; h < 2; ++h) {
+        const int j = i + 128 * h;
+        const bool jv = j0 + j < g.d;
+        for (int s4 = 0; s4 < rp; s4 += 4) {
+          uint32_t hi[4], lo[4];
 #pragma unroll
-    for (int i = 0; i < (TN * kMaxC) / 256; ++i) {
-      const int e = t + 256 * i;
-      ev[i] = (i < nev && e < TN * C && nbeg + e / C < nend) ? E[nbeg * C + e] : 0.f;
-    }
-    float sq = 0.f;
-    for (int64_t n0 = nbeg; n0 < nend; n0 += TN) {
-      // stage E tile, then U = E P_l
-#pragma unroll
-      for (int i = 0; i < (TN * kMaxC) / 256; ++i) {
-        const int e = t + 256 * i;
-        if (i < nev && e < TN * C) e_s[e] = ev[i];
-      }
-      __syncthreads();
-      for (int e = t; e < TN * r; e += 256) {
-        const int s = e / TN, nn = e - s * TN;
-        float u = 0.f;
-        for (int c = 0; c < C; ++c) u = fmaf(e_s[nn * C + c], p_s[c * r + s], u);
-        u_s[e] = u;  // transposed: u_s[s * TN + token]
-      }
-      // prefetch the next tile's E rows
-      const int64_t n1 = n0 + TN;
-#pragma unroll
-      for (int i = 0; i < (TN * kMaxC) / 256; ++i) {
-        const int e = t + 256 * i;
-        ev[i] = (i < nev && e < TN * C && n1 + e / C < nend) ? E[n1 * C + e] : 0.f;
-      }
-      __syncthreads();
-      if (do_sq && t < TN && n0 + t < nend) {
-        // ||t_n||^2 = u_n^T M_l u_n for this thread's token
-        float acc = 0.f;
-        for (int a = 0; a < r; ++a) {
-          float ma = 0.f;
-          for (int b = 0; b < r; ++b) ma = fmaf(m_s[a * r + b], u_s[b * TN + t], ma);
-          acc = fmaf(u_s[a * TN + t], ma, acc);
+          for (int u = 0; u < 4; ++u) {
+            const int s = s4 + u;
+            const float x = (jv && s < r) ? Ql[int64_t(s) * g.d + j0 + j] : 0.f;
+            hi[u] = tf32_rna(x);
+            lo[u] = tf32_rna(x - __uint_as_float(hi[u]));
+          }
+          const uint32_t off = kmaj_off(j, s4, rp);
+          *reinterpret_cast<uint4*>(smem + lay.b_hi + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+          *reinterpret_cast<uint4*>(smem + lay.b_lo + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
         }
-        sq += acc;
       }
-      // T tile: 8 tokens x 8 channels per thread
-      float acc[8][8];
+      fence_proxy_async_smem();
+      mbar_arrive(b_full);
+      const float* Pl = P + int64_t(l) * C * r;  // read by every producer thread (cached)
+      for (int64_t n0 = nbeg; n0 < nend; n0 += TM, ++tcount) {
+        const int buf = int(tcount & 1u);
+        const uint32_t ph = (tcount >> 1) & 1u;
+        const int64_t n = n0 + i;
+        float u[kMaxRP];
 #pragma unroll
-      for (int i = 0; i < 8; ++i)
+        for (int s = 0; s < kMaxRP; ++s) u[s] = 0.f;
+        if (n < nend) {
+          const float* er = E + n * C;
+          for (int c = 0; c < C; ++c) {
+            const float ec = er[c];
+            const float* pr = Pl + c * r;
 #pragma unroll
-        for (int jj = 0; jj < 8; ++jj) acc[i][jj] = 0.f;
-#pragma unroll 4
-      for (int s = 0; s < r; ++s) {
-        // this thread's 8 tokens: two broadcast 16-byte loads; its 8 channels: 4 at cg*4 and 4
-        // at 128 + cg*4 (a warp reads 2 x 512 consecutive bytes: no bank conflicts)
-        const float4 ua = *reinterpret_cast<const float4*>(u_s + s * TN + tg * 8);
-        const float4 ub = *reinterpret_cast<const float4*>(u_s + s * TN + tg * 8 + 4);
-        const float u[8] = {ua.x, ua.y, ua.z, ua.w, ub.x, ub.y, ub.z, ub.w};
-        const float4 qa = *reinterpret_cast<const float4*>(q_s + s * TD + cg * 4);
-        const float4 qb = *reinterpret_cast<const float4*>(q_s + s * TD + 128 + cg * 4);
-        const float q[8] = {qa.x, qa.y, qa.z, qa.w, qb.x, qb.y, qb.z, qb.w};
+            for (int s = 0; s < kMaxRP; ++s)
+              if (s < r) u[s] = fmaf(ec, __ldg(pr + s), u[s]);
+          }
+        }
+        if (!mbar_wait(a_empty(buf), ph ^ 1u, wc)) { ok = false; break; }
 #pragma unroll
-        for (int i = 0; i < 8; ++i)
+        for (int s4 = 0; s4 < kMaxRP; s4 += 4) {
+          if (s4 >= rp) break;
+          uint32_t hi[4], lo[4];
 #pragma unroll
-          for (int jj = 0; jj < 8; ++jj) acc[i][jj] = fmaf(u[i], q[jj], acc[i][jj]);
+          for (int v = 0; v < 4; ++v) {
+            hi[v] = tf32_rna(u[s4 + v]);
+            lo[v] = tf32_rna(u[s4 + v] - __uint_as_float(hi[v]));
+          }
+          const uint32_t off = kmaj_off(i, s4, rp);
+          *reinterpret_cast<uint4*>(smem + lay.a_hi[buf] + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+          *reinterpret_cast<uint4*>(smem + lay.a_lo[buf] + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+        }
+        fence_proxy_async_smem();
+        mbar_arrive(a_full(buf));
       }
-      // channels jA = j0 + cg*4 .. +3 (acc[i][0..3]) and jB = j0 + 128 + cg*4 .. +3 (acc[i][4..7])
-      const int64_t jA = j0 + cg * 4, jB = j0 + 128 + cg * 4;
-      const bool fullA = (jA + 4 <= d) && (d % 4 == 0), fullB = (jB + 4 <= d) && (d % 4 == 0);
+    }
+  } else if (warp == 8) {
+    // ---------------- MMA issuer
+    if (lane == 0) {
+      uint32_t tcount = 0, icount = 0;
+      bool ok = true, issued = false;
+      const uint32_t sbo = uint32_t(rp) * 32u;
+      for (int64_t it = blockIdx.x; it < g.items && ok; it += gridDim.x, ++icount) {
+        int l;
+        int64_t jt, ck;
+        decode(g, it, l, jt, ck);
+        const int64_t nbeg = ck * CHUNK;
+        const int64_t nend = (nbeg + CHUNK < g.N) ? nbeg + CHUNK : g.N;
+        if (!mbar_wait(b_full, icount & 1u, wc)) { ok = false; break; }
+        fence_after();
+        for (int64_t n0 = nbeg; n0 < nend; n0 += TM, ++tcount) {
+          const int buf = int(tcount & 1u);
+          const uint32_t ph = (tcount >> 1) & 1u;
+          if (!mbar_wait(acc_empty(buf), ph ^ 1u, wc)) { ok = false; break; }
+          if (!mbar_wait(a_full(buf), ph, wc)) { ok = false; break; }
+          fence_after();
+          const uint32_t d_tmem = tmem_base + uint32_t(buf) * TCH;
+          for (int kk = 0; kk < rp / 8; ++kk) {
+            const uint32_t koff = uint32_t(kk) * 256u;  // 8 k = two core matrices
+            const uint64_t ah = sdesc(sbase + lay.a_hi[buf] + koff, 128u, sbo, kSwizzleNone);
+            const uint64_t al = sdesc(sbase + lay.a_lo[buf] + koff, 128u, sbo, kSwizzleNone);
+            const uint64_t bh = sdesc(sbase + lay.b_hi + koff, 128u, sbo, kSwizzleNone);
+            const uint64_t bl = sdesc(sbase + lay.b_lo + koff, 128u, sbo, kSwizzleNone);
+            mma_tf32(d_tmem, ah, bh, ID_TF32, kk > 0 ? 1u : 0u);
+            mma_tf32(d_tmem, ah, bl, ID_TF32, 1u);
+            mma_tf32(d_tmem, al, bh, ID_TF32, 1u);
+          }
+          issued = true;
+          mma_commit(a_empty(buf));
+          mma_commit(acc_full(buf));
+        }
+        if (!ok) break;
+        mma_commit(b_empty);
+      }
+      if (!ok && issued) {
+        mma_commit(drain_bar);
+        mbar_drain(drain_bar, 0, limit_ns);
+      }
+    }
+    __syncwarp();
+  } else {
+    // ---------------- epilogue: warps 4..7, TMEM lane quarter = warp % 4
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    uint32_t tcount = 0;
+    bool ok = true;
+    for (int64_t it = blockIdx.x; it < g.items && ok; it += gridDim.x) {
+      int l;
+      int64_t jt, ck;
+      decode(g, it, l, jt, ck);
+      const int64_t j0 = jt * TCH;
+      const int64_t nbeg = ck * CHUNK;
+      const int64_t nend = (nbeg + CHUNK < g.N) ? nbeg + CHUNK : g.N;
+      float sq = 0.f;
+      double sqd = 0.0;
+      for (int64_t n0 = nbeg; n0 < nend; n0 += TM, ++tcount) {
+        const int buf = int(tcount & 1u);
+        const uint32_t ph = (tcount >> 1) & 1u;
+        const bool w_ok = mbar_wait(acc_full(buf), ph, wc);
+        if (!__all_sync(0xffffffffu, w_ok)) { ok = false; break; }
+        fence_after();
+        const int64_t n = n0 + row;
+        const bool nv = n < nend;
+        const int64_t rbase = (int64_t(l) * g.N + n) * g.d;
+        const uint32_t stage = sbase + lay.stage + uint32_t(q) * STAGE_WARP;
+#pragma unroll 1
+        for (int c = 0; c < TCH / 32; ++c) {
+          float v[32];
+          tmem_ld32(tmem_base + (uint32_t(q * 32) << 16) + uint32_t(buf * TCH + c * 32), v);
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int64_t n = n0 + tg * 8 + i;
-        if (n >= nend) continue;
-        const int64_t row = (int64_t(l) * N + n) * d;
+          for (int u = 0; u < 32; ++u) sq = fmaf(v[u], v[u], sq);
+          if (kBF16 && use_tma) {
+            // one bulk group per 64-channel box (4 per tile): before the first write into box
+            // c/2, the group that last read it (4 groups back) must be done reading
+            if ((c & 1) == 0) {
+              if (lane == 0) bulk_wait_group_read3();
+              __syncwarp();
+            }
+            // row `lane` of box c/2 (64 channels, 128 bytes per row), 16-byte chunks (c%2)*4 + u,
+            // placed with the 128-byte swizzle: chunk index XOR (row % 8)
+            const uint32_t box = stage + uint32_t(c >> 1) * (32u * 128u) + uint32_t(lane) * 128u;
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int64_t jb = h ? jB : jA;
-          const bool full = h ? fullB : fullA;
-          const float* a = &acc[i][4 * h];
-          if (full) {
+            for (int u = 0; u < 4; ++u) {
+              const uint32_t chunk = uint32_t((c & 1) * 4 + u) ^ uint32_t(lane & 7);
+              const uint32_t a = box + chunk * 16u;
+              asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a),
+                           "r"(pack_bf16x2(v[8 * u], v[8 * u + 1])), "r"(pack_bf16x2(v[8 * u + 2], v[8 * u + 3])),
+                           "r"(pack_bf16x2(v[8 * u + 4], v[8 * u + 5])), "r"(pack_bf16x2(v[8 * u + 6], v[8 * u + 7]))
+                           : "memory");
+            }
+            if (c & 1) {
+              fence_proxy_async_smem();  // box rows visible to the TMA unit
+              __syncwarp();
+              if (lane == 0) {
+                const int h = c >> 1;
+                const int rows0 = int(n0) + q * 32;
+                if (rows0 < nend && j0 + 64 * h < g.d)
+                  tma_store_3d(&tmT, stage + uint32_t(h) * (32u * 128u), int(j0) + 64 * h, rows0, l);
+                bulk_commit_group();
+              }
+            }
+            continue;
+          }
+          const int64_t jb = j0 + c * 32;
+          if (!nv || jb >= g.d) continue;
+          const bool whole = (jb + 32 <= g.d) && (g.d % 8 == 0);
+          if (whole) {
             if (kBF16) {
-              uint2 v;
-              v.x = pack_bf16x2(a[0], a[1]);
-              v.y = pack_bf16x2(a[2], a[3]);
-              *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(Tout) + row + jb) = v;
+              uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(Tout) + rbase + jb);
+#pragma unroll
+              for (int u = 0; u < 4; ++u)
+                o[u] = make_uint4(pack_bf16x2(v[8 * u], v[8 * u + 1]), pack_bf16x2(v[8 * u + 2], v[8 * u + 3]),
+                                  pack_bf16x2(v[8 * u + 4], v[8 * u + 5]), pack_bf16x2(v[8 * u + 6], v[8 * u + 7]));
             } else {
-              *reinterpret_cast<float4*>(static_cast<float*>(Tout) + row + jb) = make_float4(a[0], a[1], a[2], a[3]);
+              float4* o = reinterpret_cast<float4*>(static_cast<float*>(Tout) + rbase + jb);
+#pragma unroll
+              for (int u = 0; u < 8; ++u) o[u] = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
             }
           } else {
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              if (jb + u >= d) break;
+            for (int u = 0; u < 32; ++u) {
+              if (jb + u >= g.d) break;
               if (kBF16)
-                static_cast<__nv_bfloat16*>(Tout)[row + jb + u] = __float2bfloat16_rn(a[u]);
+                static_cast<__nv_bfloat16*>(Tout)[rbase + jb + u] = __float2bfloat16_rn(v[u]);
               else
-                static_cast<float*>(Tout)[row + jb + u] = a[u];
+                static_cast<float*>(Tout)[rbase + jb + u] = v[u];
             }
           }
         }
+        fence_before();
+        mbar_arrive(acc_empty(buf));
+        sqd += double(sq);
+        sq = 0.f;
       }
-      __syncthreads();  // u_s and e_s are rewritten by the next tile
-    }
-    if (do_sq) {
-      double dsq = sq;
+      if (!ok) break;
+      if (partials != nullptr) {
+        // one partial per (item, epilogue warp): no synchronisation across warps
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) dsq += __shfl_xor_sync(0xffffffffu, dsq, off);
-      if ((t & 31) == 0) red[t >> 5] = dsq;
-      __syncthreads();
-      if (t == 0) {
-        double a = 0.0;
-        for (int i = 0; i < 8; ++i) a += red[i];
-        partials[int64_t(l) * nchunks + ck] = a;
+        for (int off = 16; off > 0; off >>= 1) sqd += __shfl_xor_sync(0xffffffffu, sqd, off);
+        if (lane == 0) partials[((int64_t(l) * g.nd + jt) * g.nchunks + ck) * 4 + q] = sqd;
       }
     }
   }
+
+  if (kBF16 && use_tma && warp >= 4 && warp < 8 && lane == 0) bulk_wait_group0();
+  fence_before();
+  __syncthreads();
+  fence_after();
+  if (warp == 8) tmem_dealloc(tmem_base, TMEM_COLS);
 }
 
 // out[l] = sum of partials[l * nparts : (l + 1) * nparts] in a fixed order.
 __global__ void __launch_bounds__(256) k_reduce_partials(const double* __restrict__ partials,
                                                          int64_t nparts, double* __restrict__ out) {
-  __shared__ double red[256];
+  __shared__ double sm[256];
   const int l = blockIdx.x;
   double a = 0.0;
   for (int64_t i = threadIdx.x; i < nparts; i += 256) a += partials[int64_t(l) * nparts + i];
-  red[threadIdx.x] = a;
+  sm[threadIdx.x] = a;
   __syncthreads();
   for (int w = 128; w > 0; w >>= 1) {
-    if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+    if (threadIdx.x < w) sm[threadIdx.x] += sm[threadIdx.x + w];
     __syncthreads();
   }
-  if (threadIdx.x == 0) out[l] = red[0];
+  if (threadIdx.x == 0) out[l] = sm[0];
 }
 
 }  // namespace
 
 int64_t targets_num_partials(int64_t N, int64_t d) {
-  (void)d;
-  return (N + CHUNK - 1) / CHUNK;
+  return ((d + TCH - 1) / TCH) * ((N + CHUNK - 1) / CHUNK) * 4;
 }
 
-size_t targets_workspace_bytes(int64_t N, int L, int r) {
-  return align256(sizeof(double) * size_t(L) * size_t(targets_num_partials(N, 0))) +
-         align256(sizeof(float) * size_t(L) * size_t(r) * size_t(r));
+size_t targets_workspace_bytes(int64_t N, int L, int64_t d) {
+  return align256(sizeof(double) * size_t(L) * size_t(targets_num_partials(N, d))) + 256;
 }
 
 int targets_max_C() { return kMaxC; }
+int targets_max_r() { return kMaxRP; }
 
 cudaError_t launch_targets(const float* E, int64_t N, int C, const float* P, const float* Q,
                            int L, int r, int64_t d, void* T, int t_dtype, double* tsq,
-                           void* workspace, cudaStream_t s) {
+                           void* workspace, int32_t* status, cudaStream_t s) {
   if (N == 0 || d == 0) {
     if (tsq) return cudaMemsetAsync(tsq, 0, sizeof(double) * L, s);
     return cudaSuccess;
   }
-  double* partials = nullptr;
-  float* M = nullptr;
-  cudaError_t e;
-  if (tsq) {
-    partials = static_cast<double*>(workspace);
-    M = reinterpret_cast<float*>(static_cast<char*>(workspace) +
-                                 align256(sizeof(double) * size_t(L) * size_t(targets_num_partials(N, d))));
-    k_qqt<<<L, 256, 0, s>>>(Q, r, d, M);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+  Geo g;
+  g.N = N;
+  g.d = d;
+  g.C = C;
+  g.r = r;
+  g.rp = (r + 7) / 8 * 8;
+  g.L = L;
+  g.nd = (d + TCH - 1) / TCH;
+  g.nchunks = (N + CHUNK - 1) / CHUNK;
+  g.items = int64_t(L) * g.nd * g.nchunks;
+  double* partials = tsq ? static_cast<double*>(workspace) : nullptr;
+  int32_t* abort_flag = reinterpret_cast<int32_t*>(
+      static_cast<char*>(workspace) + align256(sizeof(double) * size_t(L) * size_t(targets_num_partials(N, d))));
+  cudaError_t e = cudaMemsetAsync(abort_flag, 0, sizeof(int32_t), s);
+  if (e != cudaSuccess) return e;
+  int64_t grid = sm_count();
+  if (grid > g.items) grid = g.items;
+  // bf16 output with 16-byte rows: tiles leave through TMA stores (3-D map over channel, token,
+  // block; 64 x 32 boxes, 128-byte swizzle); otherwise plain stores
+  CUtensorMap tmT;
+  memset(&tmT, 0, sizeof(tmT));
+  int use_tma = 0;
+  if (t_dtype == LOCA_BF16 && d % 8 == 0 && N < (int64_t(1) << 31) && d < (int64_t(1) << 31)) {
+    auto fn = tensor_map_encoder();
+    if (fn != nullptr) {
+      cuuint64_t dims[3] = {cuuint64_t(d), cuuint64_t(N), cuuint64_t(L)};
+      cuuint64_t strides[2] = {cuuint64_t(d) * 2, cuuint64_t(N) * cuuint64_t(d) * 2};
+      cuuint32_t box[3] = {64, 32, 1};
+      cuuint32_t estr[3] = {1, 1, 1};
+      if (fn(&tmT, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, T, dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS)
+        use_tma = 1;
+    }
   }
-  const int64_t items = int64_t(L) * ((d + TD - 1) / TD) * ((N + CHUNK - 1) / CHUNK);
-  int64_t grid = int64_t(sm_count()) * 2;
-  if (grid > items) grid = items;
-  const size_t shm = sizeof(float) * size_t(r * TD + TN * r + TN * kMaxC + kMaxC * r + r * r);
+  const Layout lay = layout_for(g.rp);
+  const size_t shm = lay.total;
+  const unsigned long long limit = 4000000000ull;
   if (t_dtype == LOCA_BF16) {
-    e = cudaFuncSetAttribute(k_targets<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(shm));
+    e = cudaFuncSetAttribute(k_targets_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(shm));
     if (e != cudaSuccess) return e;
-    k_targets<true><<<unsigned(grid), 256, shm, s>>>(E, N, C, P, Q, M, r, d, L, T, partials);
+    k_targets_tc<true><<<unsigned(grid), NTHREADS, shm, s>>>(E, P, Q, g, T, tmT, use_tma, partials, status,
+                                                             abort_flag, limit);
   } else {
-    e = cudaFuncSetAttribute(k_targets<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(shm));
+    e = cudaFuncSetAttribute(k_targets_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(shm));
     if (e != cudaSuccess) return e;
-    k_targets<false><<<unsigned(grid), 256, shm, s>>>(E, N, C, P, Q, M, r, d, L, T, partials);
+    k_targets_tc<false><<<unsigned(grid), NTHREADS, shm, s>>>(E, P, Q, g, T, tmT, 0, partials, status,
+                                                              abort_flag, limit);
   }
   e = cudaGetLastError();
   if (e != cudaSuccess || tsq == nullptr) return e;

@@ -170,7 +170,7 @@ def targets_workspace_size(N, L, d) -> int:
 
 def loca_targets(E, P, Q, T, tsq=None, workspace=None, stream=None):
     """Feedback targets ``T_l = (E P_l) Q_l`` into ``T`` (L x N x d, bf16 or f32) and
-    ``tsq`` (L, float64, optional)."""
+    ``tsq`` (L, float64, optional).  A workspace is always used (allocated if not given)."""
     _dev(E, "E", torch.float32, 2)
     _dev(P, "P", torch.float32, 3)
     _dev(Q, "Q", torch.float32, 3)
@@ -181,11 +181,8 @@ def loca_targets(E, P, Q, T, tsq=None, workspace=None, stream=None):
     L2, r2, d = Q.shape
     if C2 != C or L2 != L or r2 != r or tuple(T.shape) != (L, N, d):
         raise ValueError("shape mismatch among E (N x C), P (L x C x r), Q (L x r x d), T (L x N x d)")
-    ws = None
-    nbytes = 0
-    if tsq is not None:
-        nbytes = targets_workspace_size(N, L, d)
-        ws = _workspace(nbytes, E.device, workspace)
+    nbytes = targets_workspace_size(N, L, d)
+    ws = _workspace(nbytes, E.device, workspace)
     rc = lib().loca_targets(_ptr(E), N, C, _ptr(P), _ptr(Q), L, r, d, _ptr(T), _code(T.dtype), _ptr(tsq),
                             _ptr(ws), nbytes, _stream(stream))
     _check(rc, "loca_targets")

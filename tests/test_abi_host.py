@@ -56,7 +56,7 @@ def _ws(fn, *args):
 
 def test_workspace_sizes(L):
     rc, n = _ws(L.loca_targets_workspace_size, 131072, 28, 3584)
-    assert rc == 0 and n >= 8 * 28 * (131072 // 1024) + 4 * 28 * 64 * 64 and n % 256 == 0
+    assert rc == 0 and n >= 8 * 28 * 14 * (131072 // 4096) * 4 + 4 and n % 256 == 0
     rc, n = _ws(L.loca_accumulate_workspace_size, 28, 131072, 3584, 1)
     assert rc == 0 and n > 0
     rc, n = _ws(L.loca_ridge_solve_workspace_size, 28, 3584, 16)
@@ -83,10 +83,10 @@ def test_validation_codes(L):
     msg = L.loca_last_error_string()
     assert msg == b""
     # r out of range
-    assert L.loca_targets(fake, 8, 4, fake, fake, 2, 65, 64, fake, 1, None, None, 0, None) == 2
+    assert L.loca_targets(fake, 8, 4, fake, fake, 2, 33, 64, fake, 1, None, fake, 1 << 20, None) == 2
     # misaligned T (T must be 16-byte aligned)
-    assert L.loca_targets(fake, 8, 4, fake, fake, 2, 4, 64, P(258), 1, None, None, 0, None) == 3
-    # tsq requested but no workspace
+    assert L.loca_targets(fake, 8, 4, fake, fake, 2, 4, 64, P(258), 1, None, fake, 1 << 20, None) == 3
+    # no workspace
     assert L.loca_targets(fake, 8, 4, fake, fake, 2, 4, 64, fake, 1, fake, None, 0, None) == 7
     # bf16 statistics need d % 8 == 0
     assert L.loca_accumulate(fake, fake, 1, 2, 64, 60, fake, ctypes.c_float(0.01), 1, fake, fake, fake,
