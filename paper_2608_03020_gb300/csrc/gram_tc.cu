@@ -2,27 +2,34 @@
 //   Gram_l  (+)= X_l^T X_l          Cross_l (+)= alpha_l T_l^T X_l        (d x d, fp32)
 // with X_l, T_l token-major bf16 (N x d) and the token axis as the reduction axis.
 //
-// Design (one persistent CTA per SM, 192 threads):
-//   warp 0       TMA producer: 3-D tensor maps over (channel, token, block) with 128-byte
-//                swizzle; boxes of 64 channels x 64 tokens land as the MN-major canonical
-//                layout the tensor core reads (channels contiguous, one 128-byte row per token).
-//   warp 1       owns 512 TMEM columns and issues tcgen05.mma (kind::f16, bf16 x bf16 -> fp32,
-//                M = 128, N = 256, K = 16, both operands MN-major) from one thread.
-//   warps 2-5    epilogue: tcgen05.ld of the two 128 x 256 fp32 accumulators, scale, store.
-// Work item = one 256-channel column tile nt of X (the B operand, loaded once per stage) and up
-// to two 128-row accumulators that share it: Gram tiles that touch the upper triangle and all
-// cross tiles of that column, paired in order.  Sharing B gives 128 flop per byte of operand
-// traffic.  Gram elements (i, j) with i <= j are stored directly and mirrored to (j, i), so each
-// output element is written by exactly one thread (deterministic, no atomics).
-// Pipeline: 3 stages of 64 tokens (64 KB each); stage release and accumulator hand-off through
-// tcgen05.commit -> mbarrier.  Every wait is bounded: on expiry the CTA records
-// LOCA_ERR_TIMEOUT in the status word, sets a launch-local abort flag that makes every other
-// wait give up, drains its own copies and MMAs, frees TMEM and returns.
+// Design: persistent CTA pairs (clusters of 2, one CTA per SM), 192 threads per CTA.
+//   The pair computes 256-row x 256-column accumulator tiles with tcgen05.mma.cta_group::2
+//   (kind::f16, bf16 x bf16 -> fp32, M = 256, N = 256, K = 16, both operands MN-major): each CTA
+//   loads its own 128 rows of A and its own 128 columns of B, and its TMEM holds its 128 rows of
+//   the result.  Per SM a pipeline stage is then 48 KB (two A tiles and half a B tile, 64 tokens)
+//   for the MMA work a single-CTA 128 x 256 tile pair needs 64 KB for, so four stages fit in
+//   shared memory; the extra stage covers the load latency of 152 SMs streaming the same rows.
+//   warp 0       TMA producer (both CTAs): one 4-D load per operand (64-channel blocks of a
+//                (64 channels, token, channel block, block) view, 128-byte swizzle) when
+//                d % 64 == 0, else one 3-D load per 64-channel block.  The loads of both CTAs
+//                count their bytes on the even CTA's full barrier (pair form of the TMA load);
+//                the even CTA arms it with the bytes of both.
+//   warp 1       owns 512 TMEM columns (two 128 x 256 fp32 accumulators per CTA); in the even
+//                CTA one thread issues the MMAs.  Its loop is kept short (descriptors built once,
+//                advanced by integer adds; bounded wait entered only if an inline try_wait fails)
+//                so that issue keeps pace with the tensor core.
+//   warps 2-5    epilogue (both CTAs): tcgen05.ld, scale, store.
+// Work item = one 256-column tile of X (B) and up to two 256-row accumulators sharing it (Gram
+// tiles that touch the upper triangle and all cross tiles of that column, paired in order).
+// Gram elements (i, j), i <= j, are stored directly and mirrored to (j, i): every output element
+// has one writer (deterministic, no atomics).  MMA commits multicast to both CTAs' barriers.
+// Every mbarrier wait is bounded: on expiry the status word gets LOCA_ERR_TIMEOUT, a launch-local
+// flag makes every other wait give up, the even CTA drains the loads and MMAs in flight, and
+// both CTAs meet at the final cluster barrier before TMEM is freed.
 #include <cuda.h>
-#include <cudaTypedefs.h>
 #include <cuda_bf16.h>
 
-#include <mutex>
+#include <cstring>
 
 #include "loca_internal.h"
 #include "tc_ptx.cuh"
@@ -30,27 +37,30 @@
 namespace loca {
 namespace {
 
-constexpr int BM = 128;                           // accumulator rows (channels of X or T)
-constexpr int BN = 256;                           // accumulator columns (channels of X)
-constexpr int BK = 64;                            // tokens per pipeline stage
-constexpr int STAGES = 3;
-constexpr int SUB_BYTES = 64 * BK * 2;            // one TMA box: 64 channels x 64 tokens (8 KB)
-constexpr int A_BYTES = BM * BK * 2;              // 16 KB
-constexpr int B_BYTES = BN * BK * 2;              // 32 KB
-constexpr int STAGE_BYTES = 2 * A_BYTES + B_BYTES;
+using namespace tc;
+
+constexpr int BMP = 256;                            // accumulator rows per CTA pair
+constexpr int BMC = 128;                            // accumulator rows per CTA (TMEM lanes)
+constexpr int BN = 256;                             // accumulator columns (channels of X)
+constexpr int BNC = 128;                            // B columns loaded per CTA
+constexpr int BK = 64;                              // tokens per pipeline stage
+constexpr int STAGES = 4;
+constexpr int SUB_BYTES = 64 * BK * 2;              // one 64-channel x 64-token swizzled tile (8 KB)
+constexpr int A_BYTES = BMC * BK * 2;               // 16 KB
+constexpr int B_BYTES = BNC * BK * 2;               // 16 KB
+constexpr int STAGE_BYTES = 2 * A_BYTES + B_BYTES;  // 48 KB
 constexpr int TMEM_COLS = 512;
 constexpr int NUM_THREADS = 192;
+constexpr int NUM_BARS = 2 * STAGES + 3;
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /* align slack */ + 256 /* barriers */;
 
-// Instruction descriptor (kind::f16): D fp32, A bf16, B bf16, A and B MN-major, N, M.
-constexpr uint32_t IDESC = tc::idesc(1, 1, 1, 1, BM, BN);
-
-using namespace tc;
+// Instruction descriptor (kind::f16): D fp32, A bf16, B bf16, A and B MN-major, M = 256, N = 256.
+constexpr uint32_t IDESC_PAIR = tc::idesc(1, 1, 1, 1, BMP, BN);
 
 // ------------------------------------------------------------------ work items
 struct Geo {
   int L, d, N;
-  int nM, nN;       // row tiles (128) and column tiles (256)
+  int nM, nN;       // 256-row tiles and 256-column tiles
   int per_block;    // work items per block l
 };
 
@@ -58,7 +68,7 @@ struct Geo {
 __device__ __host__ __forceinline__ int gram_rows(const Geo& g, int nt) {
   int last = nt * BN + BN - 1;
   if (last > g.d - 1) last = g.d - 1;
-  int c = last / BM + 1;
+  int c = last / BMP + 1;
   return c < g.nM ? c : g.nM;
 }
 __device__ __host__ __forceinline__ int items_of_col(const Geo& g, int nt) {
@@ -69,7 +79,7 @@ struct Item {
   int l, nt;
   int nslots;
   int kind[2];  // 0 = Gram (rows from X), 1 = cross (rows from T)
-  int mt[2];
+  int mt[2];    // 256-row tile index
 };
 
 __device__ __forceinline__ Item decode(const Geo& g, int it) {
@@ -95,17 +105,19 @@ __device__ __forceinline__ Item decode(const Geo& g, int it) {
 }
 
 // ------------------------------------------------------------------ kernel
-__global__ void __launch_bounds__(NUM_THREADS, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     k_gram_cross_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmT,
-                    Geo g, int total_items, const float* __restrict__ alpha, int zero_first,
-                    float* __restrict__ gram, float* __restrict__ cross, int32_t* status,
-                    int32_t* abort_flag, unsigned long long limit_ns) {
+                    const __grid_constant__ CUtensorMap tmXa, const __grid_constant__ CUtensorMap tmTa,
+                    const __grid_constant__ CUtensorMap tmXb, int blocked, Geo g, int total_items,
+                    const float* __restrict__ alpha, int zero_first, float* __restrict__ gram,
+                    float* __restrict__ cross, int32_t* status, int32_t* abort_flag,
+                    unsigned long long limit_ns) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
-  // bars[0..S-1] full, [S..2S-1] empty, [2S] acc_full, [2S+1] acc_empty, [2S+2] drain
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 4);
+  // full[S] (loads of both CTAs, used in the even CTA), empty[S], acc_full, acc_empty, drain
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + NUM_BARS + 1);
   const uint32_t smem_base = smem_u32(smem);
   const uint32_t bar_base = smem_u32(bars);
   auto full_bar = [&](int s) { return bar_base + 8u * s; };
@@ -116,6 +128,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int cid = int(cluster_id_x());
+  const int ncl = int(ncluster_x());
   const WaitCtl wc{status, abort_flag, limit_ns};
 
   if (threadIdx.x == 0) {
@@ -124,101 +140,123 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       mbar_init(empty_bar(s), 1);
     }
     mbar_init(acc_full, 1);
-    mbar_init(acc_empty, 128);
+    mbar_init(acc_empty, 8);  // lane 0 of the 4 epilogue warps of each CTA
     mbar_init(drain_bar, 1);
     mbar_init_fence();
-    prefetch_tensormap(&tmX);
-    prefetch_tensormap(&tmT);
+    if (blocked) {
+      prefetch_tensormap(&tmXa);
+      prefetch_tensormap(&tmTa);
+      prefetch_tensormap(&tmXb);
+    } else {
+      prefetch_tensormap(&tmX);
+      prefetch_tensormap(&tmT);
+    }
   }
-  if (warp == 1) tmem_alloc(smem_u32(tmem_slot), TMEM_COLS);
+  if (warp == 1) tmem_alloc_pair(smem_u32(tmem_slot), TMEM_COLS);
   fence_before();
-  __syncthreads();
+  cluster_sync();  // barriers of both CTAs initialised, TMEM allocated
   fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const int nkb = (g.N + BK - 1) / BK;
 
   if (warp == 0) {
     if (lane == 0) {
-      // ---------------- TMA producer
+      // ---------------- TMA producer (both CTAs): this CTA's rows of A and columns of B
       int stage = 0;
       uint32_t phase = 0;
-      uint32_t pending = 0, pending_par = 0;  // stages with loads in flight, their phase parity
+      uint32_t pending = 0, pending_par = 0;  // even CTA: armed stages and their phase parity
       bool ok = true;
-      for (int it = blockIdx.x; it < total_items && ok; it += gridDim.x) {
+      for (int it = cid; it < total_items && ok; it += ncl) {
         const Item w = decode(g, it);
-        const uint32_t bytes = uint32_t(w.nslots) * A_BYTES + B_BYTES;
+        const uint32_t bytes_both = 2u * (uint32_t(w.nslots) * A_BYTES + B_BYTES);
         for (int kb = 0; kb < nkb; ++kb) {
-          if (!mbar_wait(empty_bar(stage), phase ^ 1u, wc)) { ok = false; break; }
-          const uint32_t fb = full_bar(stage);
-          mbar_arrive_expect_tx(fb, bytes);
-          const uint32_t st = smem_base + uint32_t(stage) * STAGE_BYTES;
-          const int tok = kb * BK;
-          for (int s = 0; s < w.nslots; ++s) {
-            const CUtensorMap* map = w.kind[s] == 0 ? &tmX : &tmT;
-            const uint32_t dst = st + uint32_t(s) * A_BYTES;
-            tma_load_3d(dst, map, fb, w.mt[s] * BM, tok, w.l);
-            tma_load_3d(dst + SUB_BYTES, map, fb, w.mt[s] * BM + 64, tok, w.l);
+          if (!mbar_try_wait_cluster(empty_bar(stage), phase ^ 1u) &&
+              !mbar_wait_cluster(empty_bar(stage), phase ^ 1u, wc)) {
+            ok = false;
+            break;
           }
+          const uint32_t fb = mapa_shared(full_bar(stage), 0);
+          if (leader) {
+            mbar_arrive_expect_tx(full_bar(stage), bytes_both);
+            pending |= 1u << stage;
+            pending_par = (pending_par & ~(1u << stage)) | (phase << stage);
+          }
+          const uint32_t st = smem_base + uint32_t(stage) * STAGE_BYTES;
           const uint32_t bdst = st + 2u * A_BYTES;
-#pragma unroll
-          for (int h = 0; h < BN / 64; ++h)
-            tma_load_3d(bdst + uint32_t(h) * SUB_BYTES, &tmX, fb, w.nt * BN + h * 64, tok, w.l);
-          pending |= 1u << stage;
-          pending_par = (pending_par & ~(1u << stage)) | (phase << stage);
+          const int tok = kb * BK;
+          const int col0 = w.nt * BN + int(rank) * BNC;
+          if (blocked) {
+            for (int s = 0; s < w.nslots; ++s)
+              tma_load_4d_pair(st + uint32_t(s) * A_BYTES, w.kind[s] == 0 ? &tmXa : &tmTa, fb, 0, tok,
+                               (w.mt[s] * BMP + int(rank) * BMC) / 64, w.l);
+            tma_load_4d_pair(bdst, &tmXb, fb, 0, tok, col0 / 64, w.l);
+          } else {
+            for (int s = 0; s < w.nslots; ++s) {
+              const CUtensorMap* map = w.kind[s] == 0 ? &tmX : &tmT;
+              const uint32_t dst = st + uint32_t(s) * A_BYTES;
+              const int row0 = w.mt[s] * BMP + int(rank) * BMC;
+              tma_load_3d_pair(dst, map, fb, row0, tok, w.l);
+              tma_load_3d_pair(dst + SUB_BYTES, map, fb, row0 + 64, tok, w.l);
+            }
+            tma_load_3d_pair(bdst, &tmX, fb, col0, tok, w.l);
+            tma_load_3d_pair(bdst + SUB_BYTES, &tmX, fb, col0 + 64, tok, w.l);
+          }
           if (++stage == STAGES) { stage = 0; phase ^= 1u; }
         }
       }
-      if (!ok) {
-        // let the copies already issued land before the CTA can exit
-        const uint64_t t0 = globaltimer();
-        for (int s = 0; s < STAGES; ++s) {
-          if (!(pending & (1u << s))) continue;
-          while (!mbar_try_wait(full_bar(s), (pending_par >> s) & 1u)) {
-            if (globaltimer() - t0 > limit_ns) break;
-          }
-        }
+      if (!ok && leader) {
+        // the armed stages count the bytes of both CTAs: let them land before either CTA exits
+        for (int s = 0; s < STAGES; ++s)
+          if (pending & (1u << s)) mbar_drain(full_bar(s), (pending_par >> s) & 1u, limit_ns);
       }
     }
     __syncwarp();
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ---------------- MMA issuer
+    if (lane == 0 && leader) {
+      // ---------------- MMA issuer (even CTA)
       int stage = 0;
       uint32_t phase = 0, acc_phase = 0;
       bool ok = true;
       bool issued = false;
-      for (int it = blockIdx.x; it < total_items && ok; it += gridDim.x) {
+      const uint64_t a_desc0 = sdesc(smem_base, SUB_BYTES, 1024u, kSwizzle128B);
+      const uint64_t b_desc0 = sdesc(smem_base + 2u * A_BYTES, SUB_BYTES, 1024u, kSwizzle128B);
+      constexpr uint64_t kStageStep = STAGE_BYTES >> 4, kSlotStep = A_BYTES >> 4, kKStep = 2048 >> 4;
+      const uint32_t d0 = tmem_base, d1 = tmem_base + uint32_t(BN);
+      for (int it = cid; it < total_items && ok; it += ncl) {
         const Item w = decode(g, it);
-        if (!mbar_wait(acc_empty, acc_phase ^ 1u, wc)) { ok = false; break; }
+        const bool two = w.nslots == 2;
+        if (!mbar_try_wait_cluster(acc_empty, acc_phase ^ 1u) &&
+            !mbar_wait_cluster(acc_empty, acc_phase ^ 1u, wc)) {
+          ok = false;
+          break;
+        }
         fence_after();
         for (int kb = 0; kb < nkb; ++kb) {
-          if (!mbar_wait(full_bar(stage), phase, wc)) { ok = false; break; }
+          if (!mbar_try_wait_cluster(full_bar(stage), phase) &&
+              !mbar_wait_cluster(full_bar(stage), phase, wc)) {
+            ok = false;
+            break;
+          }
           fence_after();
-          const uint32_t st = smem_base + uint32_t(stage) * STAGE_BYTES;
-          const uint32_t bsm = st + 2u * A_BYTES;
+          const uint64_t so = uint64_t(stage) * kStageStep;
+          const uint64_t ad = a_desc0 + so, bd = b_desc0 + so;
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk) {
-            const uint64_t bd = sdesc(bsm + uint32_t(kk) * 2048u, SUB_BYTES, 1024u, kSwizzle128B);
-            for (int s = 0; s < w.nslots; ++s) {
-              const uint64_t ad = sdesc(st + uint32_t(s) * A_BYTES + uint32_t(kk) * 2048u,
-                                        SUB_BYTES, 1024u, kSwizzle128B);
-              mma_f16(tmem_base + uint32_t(s) * BN, ad, bd, IDESC, (kb | kk) != 0 ? 1u : 0u);
-            }
+            const uint32_t acc = (kb | kk) != 0 ? 1u : 0u;
+            mma_f16_pair(d0, ad + kk * kKStep, bd + kk * kKStep, IDESC_PAIR, acc);
+            if (two) mma_f16_pair(d1, ad + kSlotStep + kk * kKStep, bd + kk * kKStep, IDESC_PAIR, acc);
           }
           issued = true;
-          mma_commit(empty_bar(stage));  // frees the stage once these MMAs have read it
+          mma_commit_pair_mc(empty_bar(stage), 0x3);  // frees the stage in both CTAs
           if (++stage == STAGES) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
-        mma_commit(acc_full);  // accumulators complete
+        mma_commit_pair_mc(acc_full, 0x3);  // accumulators of both CTAs complete
         acc_phase ^= 1u;
       }
       if (!ok && issued) {
-        mma_commit(drain_bar);
-        const uint64_t t0 = globaltimer();
-        while (!mbar_try_wait(drain_bar, 0)) {
-          if (globaltimer() - t0 > limit_ns) break;
-        }
+        mma_commit_pair(drain_bar);
+        mbar_drain(drain_bar, 0, limit_ns);
       }
     }
     __syncwarp();
@@ -226,17 +264,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     // ---------------- epilogue: warps 2..5, TMEM lane quarter = warp % 4
     const int q = warp & 3;
     const int row_in_tile = q * 32 + lane;
+    const uint32_t acc_empty_leader = leader ? acc_empty : mapa_shared(acc_empty, 0);
     uint32_t acc_phase = 0;
-    for (int it = blockIdx.x; it < total_items; it += gridDim.x) {
+    for (int it = cid; it < total_items; it += ncl) {
       const Item w = decode(g, it);
-      const bool ok = mbar_wait(acc_full, acc_phase, wc);
+      const bool ok = mbar_wait_cluster(acc_full, acc_phase, wc);
       if (!__all_sync(0xffffffffu, ok)) break;  // warp-uniform decision, warp reconverged
       fence_after();
       const float al = alpha[w.l];
       for (int s = 0; s < w.nslots; ++s) {
         const bool is_gram = w.kind[s] == 0;
         float* out = (is_gram ? gram : cross) + int64_t(w.l) * g.d * g.d;
-        const int i = w.mt[s] * BM + row_in_tile;
+        const int i = w.mt[s] * BMP + int(rank) * BMC + row_in_tile;
         const float sc = is_gram ? 1.f : al;
 #pragma unroll 1
         for (int c = 0; c < BN / 32; ++c) {
@@ -283,18 +322,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
       }
       fence_before();
-      mbar_arrive(acc_empty);
+      __syncwarp();
+      if (lane == 0) {
+        if (leader) mbar_arrive(acc_empty);
+        else mbar_arrive_remote(acc_empty_leader);
+      }
       acc_phase ^= 1u;
     }
   }
 
   fence_before();
-  __syncthreads();
+  cluster_sync();  // no CTA leaves while its peer may still use its barriers, smem or TMEM
   fence_after();
-  if (warp == 1) tmem_dealloc(tmem_base, TMEM_COLS);
+  if (warp == 1) tmem_dealloc_pair(tmem_base, TMEM_COLS);
 }
 
 // ------------------------------------------------------------------ host side
+// 3-D view (channel, token, block) of X or T; boxes of 64 channels x BK tokens.
 bool make_map(CUtensorMap* m, const void* base, int L, int64_t N, int64_t d) {
   auto fn = tensor_map_encoder();
   if (!fn) return false;
@@ -302,11 +346,44 @@ bool make_map(CUtensorMap* m, const void* base, int L, int64_t N, int64_t d) {
   cuuint64_t strides[2] = {cuuint64_t(d) * 2, cuuint64_t(N) * cuuint64_t(d) * 2};
   cuuint32_t box[3] = {64, BK, 1};
   cuuint32_t estr[3] = {1, 1, 1};
-  const CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims,
-                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  return r == CUDA_SUCCESS;
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// 4-D view (64 channels, token, 64-channel block, block) of X or T, for d % 64 == 0: one box of
+// `nblk` channel blocks x BK tokens lands as nblk consecutive 64 x BK swizzled tiles.
+bool make_map_blocked(CUtensorMap* m, const void* base, int L, int64_t N, int64_t d, int nblk) {
+  auto fn = tensor_map_encoder();
+  if (!fn) return false;
+  cuuint64_t dims[4] = {64, cuuint64_t(N), cuuint64_t(d / 64), cuuint64_t(L)};
+  cuuint64_t strides[3] = {cuuint64_t(d) * 2, 128, cuuint64_t(N) * cuuint64_t(d) * 2};
+  cuuint32_t box[4] = {64, BK, cuuint32_t(nblk), 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Clusters of 2 that can be resident at once (every SM pairs on GB300: 76 clusters on 152 SMs).
+int resident_clusters() {
+  int clusters = sm_count() / 2;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(unsigned(2 * clusters));
+  cfg.blockDim = dim3(NUM_THREADS);
+  cfg.dynamicSmemBytes = SMEM_BYTES;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = 2;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, k_gram_cross_tc, &cfg) == cudaSuccess && n > 0 && n < clusters)
+    clusters = n;
+  cudaGetLastError();  // an unsupported query leaves the default
+  return clusters;
 }
 
 }  // namespace
@@ -314,26 +391,37 @@ bool make_map(CUtensorMap* m, const void* base, int L, int64_t N, int64_t d) {
 cudaError_t launch_gram_cross_tc(const void* X, const void* T, int L, int64_t N, int64_t d,
                                  const float* alpha, int zero_first, float* gram, float* cross,
                                  int32_t* status, int32_t* abort_flag, cudaStream_t s) {
-  CUtensorMap mx, mt;
+  CUtensorMap mx, mt, mxa, mta, mxb;
+  memset(&mxa, 0, sizeof(mxa));
+  memset(&mta, 0, sizeof(mta));
+  memset(&mxb, 0, sizeof(mxb));
   if (!make_map(&mx, X, L, N, d) || !make_map(&mt, T, L, N, d)) return cudaErrorInvalidValue;
+  int blocked = 0;
+  if (d % 64 == 0 && make_map_blocked(&mxa, X, L, N, d, BMC / 64) &&
+      make_map_blocked(&mta, T, L, N, d, BMC / 64) && make_map_blocked(&mxb, X, L, N, d, BNC / 64))
+    blocked = 1;
   Geo g;
   g.L = L;
   g.d = int(d);
   g.N = int(N);
-  g.nM = int((d + BM - 1) / BM);
+  g.nM = int((d + BMP - 1) / BMP);
   g.nN = int((d + BN - 1) / BN);
   g.per_block = 0;
   for (int nt = 0; nt < g.nN; ++nt) g.per_block += items_of_col(g, nt);
   const int total = g.per_block * L;
-  int grid = sm_count();
-  if (grid > total) grid = total;
-  cudaError_t e = cudaMemsetAsync(abort_flag, 0, sizeof(int32_t), s);
+  cudaError_t e = cudaFuncSetAttribute(k_gram_cross_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       SMEM_BYTES);
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(k_gram_cross_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  static int clusters_cached = 0;  // per process; the library drives one device type
+  if (clusters_cached == 0) clusters_cached = resident_clusters();
+  int clusters = clusters_cached;
+  if (clusters > total) clusters = total;
+  if (clusters < 1) clusters = 1;
+  e = cudaMemsetAsync(abort_flag, 0, sizeof(int32_t), s);
   if (e != cudaSuccess) return e;
-  k_gram_cross_tc<<<grid, NUM_THREADS, SMEM_BYTES, s>>>(mx, mt, g, total, alpha, zero_first, gram,
-                                                        cross, status, abort_flag,
-                                                        4000000000ull /* 4 s per wait */);
+  k_gram_cross_tc<<<2 * clusters, NUM_THREADS, SMEM_BYTES, s>>>(mx, mt, mxa, mta, mxb, blocked, g, total,
+                                                                alpha, zero_first, gram, cross, status,
+                                                                abort_flag, 4000000000ull /* 4 s per wait */);
   return cudaGetLastError();
 }
 
