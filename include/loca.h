@@ -155,8 +155,8 @@ int loca_accumulate(const void* X, const void* T, int dtype, int32_t L, int64_t 
  *   (0 if tsq[l] == 0), xsq_total[l] = (zero_first ? 0 : xsq_total[l]) + xsq_b[l].
  *   alpha: L float device output.  Workspace: loca_batch_step_workspace_size.
  * loca_gram_cross (Eq. 9; S7): gram_l (+)= X_l^T X_l, cross_l (+)= alpha[l] T_l^T X_l with the
- *   alpha of loca_batch_step.  Workspace: loca_gram_cross_workspace_size (256 bytes; holds a
- *   launch-local flag).  Arguments, layouts, dtypes and determinism as loca_accumulate.
+ *   alpha of loca_batch_step.  Workspace: loca_gram_cross_workspace_size (256 bytes; holds
+ *   launch-local flags).  Arguments, layouts, dtypes and determinism as loca_accumulate.
  */
 int loca_batch_step_workspace_size(int32_t L, size_t* bytes /* host */);
 int loca_batch_step(const void* X, int dtype, int32_t L, int64_t N, int64_t d, const double* tsq,

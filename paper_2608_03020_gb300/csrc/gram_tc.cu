@@ -23,6 +23,13 @@
 // tiles that touch the upper triangle and all cross tiles of that column, paired in order).
 // Gram elements (i, j), i <= j, are stored directly and mirrored to (j, i): every output element
 // has one writer (deterministic, no atomics).  MMA commits multicast to both CTAs' barriers.
+// Lockstep: all clusters stream the same token window of X_l and T_l at the same time, so each
+// operand line is read from HBM once and then served from L2 to the ~25 tiles that need it.  The
+// clusters start every round of work items together: the even CTA's producer counts the items whose
+// loads it has issued on a launch-local counter and, before the next item, waits (bounded, as a hint
+// only) until every cluster has done the same.  Without it the clusters drift apart over a few
+// items (items differ in length and epilogue cost), the L2 no longer holds what the others read,
+// and the load latency, not the tensor core, sets the pace (about 1.25x slower at 7B size).
 // Every mbarrier wait is bounded: on expiry the status word gets LOCA_ERR_TIMEOUT, a launch-local
 // flag makes every other wait give up, the even CTA drains the loads and MMAs in flight, and
 // both CTAs meet at the final cluster barrier before TMEM is freed.
@@ -111,7 +118,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
                     const __grid_constant__ CUtensorMap tmXb, int blocked, Geo g, int total_items,
                     const float* __restrict__ alpha, int zero_first, float* __restrict__ gram,
                     float* __restrict__ cross, int32_t* status, int32_t* abort_flag,
-                    unsigned long long limit_ns) {
+                    uint32_t* round_ctr, unsigned long long limit_ns, unsigned long long sync_ns) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -166,7 +173,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       uint32_t phase = 0;
       uint32_t pending = 0, pending_par = 0;  // even CTA: armed stages and their phase parity
       bool ok = true;
-      for (int it = cid; it < total_items && ok; it += ncl) {
+      bool sync = leader;  // dropped for the rest of the launch if a round wait runs out
+      uint32_t round = 0;
+      for (int it = cid; it < total_items && ok; it += ncl, ++round) {
+        if (sync && round > 0) {
+          // every cluster has issued the loads of its previous item (hint: bounded, no error)
+          const uint32_t target = uint32_t(ncl) * round;
+          const uint64_t t0 = globaltimer();
+          while (*reinterpret_cast<volatile uint32_t*>(round_ctr) < target) {
+            if (globaltimer() - t0 > sync_ns) {
+              sync = false;
+              break;
+            }
+          }
+        }
         const Item w = decode(g, it);
         const uint32_t bytes_both = 2u * (uint32_t(w.nslots) * A_BYTES + B_BYTES);
         for (int kb = 0; kb < nkb; ++kb) {
@@ -203,6 +223,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
           }
           if (++stage == STAGES) { stage = 0; phase ^= 1u; }
         }
+        if (ok && leader) atomicAdd(round_ctr, 1u);
       }
       if (!ok && leader) {
         // the armed stages count the bytes of both CTAs: let them land before either CTA exits
@@ -417,11 +438,15 @@ cudaError_t launch_gram_cross_tc(const void* X, const void* T, int L, int64_t N,
   int clusters = clusters_cached;
   if (clusters > total) clusters = total;
   if (clusters < 1) clusters = 1;
-  e = cudaMemsetAsync(abort_flag, 0, sizeof(int32_t), s);
+  // abort flag and round counter (two int32 of the launch-local flag area)
+  e = cudaMemsetAsync(abort_flag, 0, 2 * sizeof(int32_t), s);
   if (e != cudaSuccess) return e;
-  k_gram_cross_tc<<<2 * clusters, NUM_THREADS, SMEM_BYTES, s>>>(mx, mt, mxa, mta, mxb, blocked, g, total,
-                                                                alpha, zero_first, gram, cross, status,
-                                                                abort_flag, 4000000000ull /* 4 s per wait */);
+  // a round takes about nkb x 1024 tensor-core cycles; wait for the slowest cluster up to ~3x that
+  const int64_t nkb = (N + BK - 1) / BK;
+  const unsigned long long sync_ns = 50000ull + 2000ull * (unsigned long long)nkb;
+  k_gram_cross_tc<<<2 * clusters, NUM_THREADS, SMEM_BYTES, s>>>(
+      mx, mt, mxa, mta, mxb, blocked, g, total, alpha, zero_first, gram, cross, status, abort_flag,
+      reinterpret_cast<uint32_t*>(abort_flag + 1), 4000000000ull /* 4 s per wait */, sync_ns);
   return cudaGetLastError();
 }
 

@@ -56,7 +56,8 @@ cudaError_t launch_sumsq_and_step(const void* X, int dtype, int L, int64_t N, in
 cudaError_t launch_gram_cross_f32(const float* X, const float* T, int L, int64_t N, int64_t d,
                                   const float* alpha, int zero_first, float* gram, float* cross,
                                   cudaStream_t s);
-// bf16-input Gram / cross on tcgen05 tensor cores.
+// bf16-input Gram / cross on tcgen05 tensor cores.  abort_flag points to two int32 of launch-local
+// device memory (abort flag, round counter), both reset by the launcher on stream s.
 cudaError_t launch_gram_cross_tc(const void* X, const void* T, int L, int64_t N, int64_t d,
                                  const float* alpha, int zero_first, float* gram, float* cross,
                                  int32_t* status, int32_t* abort_flag, cudaStream_t s);
