@@ -14,8 +14,10 @@
 //   warp 8      owns 512 TMEM columns (two 128 x 256 fp32 accumulators) and issues the MMAs.
 //   warps 4-7   epilogue: tcgen05.ld, sum of squares of the fp32 values (||T_l||^2), rounding
 //               to the output type; in bf16 each warp stages its 32 token rows in shared
-//               memory (128-byte swizzled boxes) and writes them with TMA bulk tensor stores,
-//               so HBM sees whole lines; fp32 output uses plain stores (one row per thread).
+//               memory (128-byte swizzled boxes) and writes them with TMA bulk tensor stores
+//               (two 128-channel boxes per tile when d % 64 == 0), so HBM sees whole lines;
+//               fp32 output uses plain stores (one row per thread).  TMEM is read 64 columns
+//               per wait.
 // Work item = (block l, 256-channel tile, 4096-token chunk); ||T_l||^2 partials are written
 // per item and epilogue warp and summed in a fixed order by k_reduce_partials
 // (deterministic).  All waits are bounded (see tc_ptx.cuh) and no warp waits on another
@@ -99,7 +101,7 @@ __device__ __forceinline__ void decode(const Geo& g, int64_t it, int& l, int64_t
 template <bool kBF16>
 __global__ void __launch_bounds__(NTHREADS, 1)
     k_targets_tc(const float* __restrict__ E, const float* __restrict__ P, const float* __restrict__ Q,
-                 Geo g, void* __restrict__ Tout, const __grid_constant__ CUtensorMap tmT, int use_tma,
+                 Geo g, void* __restrict__ Tout, const __grid_constant__ CUtensorMap tmT, int store_mode,
                  double* __restrict__ partials, int32_t* status, int32_t* abort_flag,
                  unsigned long long limit_ns) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -279,66 +281,77 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         const int64_t rbase = (int64_t(l) * g.N + n) * g.d;
         const uint32_t stage = sbase + lay.stage + uint32_t(q) * STAGE_WARP;
 #pragma unroll 1
-        for (int c = 0; c < TCH / 32; ++c) {
-          float v[32];
-          tmem_ld32(tmem_base + (uint32_t(q * 32) << 16) + uint32_t(buf * TCH + c * 32), v);
+        for (int cp = 0; cp < TCH / 64; ++cp) {
+          // 64 channels (one 128-byte swizzled box) per step; two TMEM loads, one wait
+          float v[64];
+          tmem_ld32x2(tmem_base + (uint32_t(q * 32) << 16) + uint32_t(buf * TCH + cp * 64), v);
 #pragma unroll
-          for (int u = 0; u < 32; ++u) sq = fmaf(v[u], v[u], sq);
-          if (kBF16 && use_tma) {
-            // one bulk group per 64-channel box (4 per tile): before the first write into box
-            // c/2, the group that last read it (4 groups back) must be done reading
-            if ((c & 1) == 0) {
-              if (lane == 0) bulk_wait_group_read3();
+          for (int u = 0; u < 64; ++u) sq = fmaf(v[u], v[u], sq);
+          if (kBF16 && store_mode != 0) {
+            // before the first write into a staging region, the bulk group that last read it (one
+            // tile earlier) must be done reading: 4 groups per tile (3-D boxes) or 2 (4-D boxes)
+            if (store_mode == 1 || (cp & 1) == 0) {
+              if (lane == 0) {
+                if (store_mode == 1) bulk_wait_group_read3();
+                else bulk_wait_group_read1();
+              }
               __syncwarp();
             }
-            // row `lane` of box c/2 (64 channels, 128 bytes per row), 16-byte chunks (c%2)*4 + u,
-            // placed with the 128-byte swizzle: chunk index XOR (row % 8)
-            const uint32_t box = stage + uint32_t(c >> 1) * (32u * 128u) + uint32_t(lane) * 128u;
+            // row `lane` of box cp (64 channels, 128 bytes), 16-byte chunk u placed with the
+            // 128-byte swizzle: chunk index XOR (row % 8)
+            const uint32_t box = stage + uint32_t(cp) * (32u * 128u) + uint32_t(lane) * 128u;
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              const uint32_t chunk = uint32_t((c & 1) * 4 + u) ^ uint32_t(lane & 7);
-              const uint32_t a = box + chunk * 16u;
+            for (int u = 0; u < 8; ++u) {
+              const uint32_t a = box + ((uint32_t(u) ^ uint32_t(lane & 7)) * 16u);
               asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a),
                            "r"(pack_bf16x2(v[8 * u], v[8 * u + 1])), "r"(pack_bf16x2(v[8 * u + 2], v[8 * u + 3])),
                            "r"(pack_bf16x2(v[8 * u + 4], v[8 * u + 5])), "r"(pack_bf16x2(v[8 * u + 6], v[8 * u + 7]))
                            : "memory");
             }
-            if (c & 1) {
-              fence_proxy_async_smem();  // box rows visible to the TMA unit
-              __syncwarp();
-              if (lane == 0) {
-                const int h = c >> 1;
-                const int rows0 = int(n0) + q * 32;
-                if (rows0 < nend && j0 + 64 * h < g.d)
-                  tma_store_3d(&tmT, stage + uint32_t(h) * (32u * 128u), int(j0) + 64 * h, rows0, l);
+            fence_proxy_async_smem();  // box rows visible to the TMA unit
+            __syncwarp();
+            if (lane == 0) {
+              const int rows0 = int(n0) + q * 32;
+              if (store_mode == 1) {
+                if (rows0 < nend && j0 + 64 * cp < g.d)
+                  tma_store_3d(&tmT, stage + uint32_t(cp) * (32u * 128u), int(j0) + 64 * cp, rows0, l);
+                bulk_commit_group();
+              } else if (cp & 1) {
+                const int h = cp >> 1;  // boxes 2h, 2h+1 leave as one 4-D box of two channel blocks
+                if (rows0 < nend && j0 + 128 * h < g.d)
+                  tma_store_4d(&tmT, stage + uint32_t(h) * (64u * 128u), 0, rows0, int(j0 / 64) + 2 * h, l);
                 bulk_commit_group();
               }
             }
             continue;
           }
-          const int64_t jb = j0 + c * 32;
-          if (!nv || jb >= g.d) continue;
-          const bool whole = (jb + 32 <= g.d) && (g.d % 8 == 0);
-          if (whole) {
-            if (kBF16) {
-              uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(Tout) + rbase + jb);
 #pragma unroll
-              for (int u = 0; u < 4; ++u)
-                o[u] = make_uint4(pack_bf16x2(v[8 * u], v[8 * u + 1]), pack_bf16x2(v[8 * u + 2], v[8 * u + 3]),
-                                  pack_bf16x2(v[8 * u + 4], v[8 * u + 5]), pack_bf16x2(v[8 * u + 6], v[8 * u + 7]));
+          for (int hh = 0; hh < 2; ++hh) {
+            const float* vv = v + 32 * hh;
+            const int64_t jb = j0 + cp * 64 + hh * 32;
+            if (!nv || jb >= g.d) continue;
+            const bool whole = (jb + 32 <= g.d) && (g.d % 8 == 0);
+            if (whole) {
+              if (kBF16) {
+                uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(Tout) + rbase + jb);
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                  o[u] = make_uint4(pack_bf16x2(vv[8 * u], vv[8 * u + 1]), pack_bf16x2(vv[8 * u + 2], vv[8 * u + 3]),
+                                    pack_bf16x2(vv[8 * u + 4], vv[8 * u + 5]), pack_bf16x2(vv[8 * u + 6], vv[8 * u + 7]));
+              } else {
+                float4* o = reinterpret_cast<float4*>(static_cast<float*>(Tout) + rbase + jb);
+#pragma unroll
+                for (int u = 0; u < 8; ++u) o[u] = make_float4(vv[4 * u], vv[4 * u + 1], vv[4 * u + 2], vv[4 * u + 3]);
+              }
             } else {
-              float4* o = reinterpret_cast<float4*>(static_cast<float*>(Tout) + rbase + jb);
 #pragma unroll
-              for (int u = 0; u < 8; ++u) o[u] = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
-            }
-          } else {
-#pragma unroll
-            for (int u = 0; u < 32; ++u) {
-              if (jb + u >= g.d) break;
-              if (kBF16)
-                static_cast<__nv_bfloat16*>(Tout)[rbase + jb + u] = __float2bfloat16_rn(v[u]);
-              else
-                static_cast<float*>(Tout)[rbase + jb + u] = v[u];
+              for (int u = 0; u < 32; ++u) {
+                if (jb + u >= g.d) break;
+                if (kBF16)
+                  static_cast<__nv_bfloat16*>(Tout)[rbase + jb + u] = __float2bfloat16_rn(vv[u]);
+                else
+                  static_cast<float*>(Tout)[rbase + jb + u] = vv[u];
+              }
             }
           }
         }
@@ -357,7 +370,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     }
   }
 
-  if (kBF16 && use_tma && warp >= 4 && warp < 8 && lane == 0) bulk_wait_group0();
+  if (kBF16 && store_mode != 0 && warp >= 4 && warp < 8 && lane == 0) bulk_wait_group0();
   fence_before();
   __syncthreads();
   fence_after();
@@ -417,14 +430,26 @@ cudaError_t launch_targets(const float* E, int64_t N, int C, const float* P, con
   if (e != cudaSuccess) return e;
   int64_t grid = sm_count();
   if (grid > g.items) grid = g.items;
-  // bf16 output with 16-byte rows: tiles leave through TMA stores (3-D map over channel, token,
-  // block; 64 x 32 boxes, 128-byte swizzle); otherwise plain stores
+  // bf16 output with 16-byte rows: tiles leave through TMA stores, 128-byte swizzled boxes of 64
+  // channels x 32 tokens.  d % 64 == 0: a 4-D view (64 channels, token, channel block, block) and
+  // boxes of two channel blocks (store_mode 2); else a 3-D view (channel, token, block), one box per
+  // 64 channels (store_mode 1).  Otherwise plain stores (store_mode 0).
   CUtensorMap tmT;
   memset(&tmT, 0, sizeof(tmT));
-  int use_tma = 0;
+  int store_mode = 0;
   if (t_dtype == LOCA_BF16 && d % 8 == 0 && N < (int64_t(1) << 31) && d < (int64_t(1) << 31)) {
     auto fn = tensor_map_encoder();
-    if (fn != nullptr) {
+    if (fn != nullptr && d % 64 == 0) {
+      cuuint64_t dims[4] = {64, cuuint64_t(N), cuuint64_t(d / 64), cuuint64_t(L)};
+      cuuint64_t strides[3] = {cuuint64_t(d) * 2, 128, cuuint64_t(N) * cuuint64_t(d) * 2};
+      cuuint32_t box[4] = {64, 32, 2, 1};
+      cuuint32_t estr[4] = {1, 1, 1, 1};
+      if (fn(&tmT, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, T, dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS)
+        store_mode = 2;
+    }
+    if (fn != nullptr && store_mode == 0) {
       cuuint64_t dims[3] = {cuuint64_t(d), cuuint64_t(N), cuuint64_t(L)};
       cuuint64_t strides[2] = {cuuint64_t(d) * 2, cuuint64_t(N) * cuuint64_t(d) * 2};
       cuuint32_t box[3] = {64, 32, 1};
@@ -432,7 +457,7 @@ cudaError_t launch_targets(const float* E, int64_t N, int C, const float* P, con
       if (fn(&tmT, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, T, dims, strides, box, estr,
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS)
-        use_tma = 1;
+        store_mode = 1;
     }
   }
   const Layout lay = layout_for(g.rp);
@@ -441,7 +466,7 @@ cudaError_t launch_targets(const float* E, int64_t N, int C, const float* P, con
   if (t_dtype == LOCA_BF16) {
     e = cudaFuncSetAttribute(k_targets_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(shm));
     if (e != cudaSuccess) return e;
-    k_targets_tc<true><<<unsigned(grid), NTHREADS, shm, s>>>(E, P, Q, g, T, tmT, use_tma, partials, status,
+    k_targets_tc<true><<<unsigned(grid), NTHREADS, shm, s>>>(E, P, Q, g, T, tmT, store_mode, partials, status,
                                                              abort_flag, limit);
   } else {
     e = cudaFuncSetAttribute(k_targets_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(shm));

@@ -112,6 +112,7 @@ def test_error_parity(lc, case):
     ("bf16", 2, 300, 512, 4, 32),
     ("f32", 1, 5000, 264, 5, 12),
     ("bf16", 1, 4100, 120, 3, 3),
+    ("bf16", 2, 3000, 960, 2, 8),
 ])
 def test_targets_parity(lc, tdt, L, N, d, C, r):
     """S3 / S11.  Each output is an fp32 dot product of length r after an fp32 product of length C:
