@@ -41,10 +41,12 @@ METRIC = "LoCA fit tokens/s/block at Qwen2.5-7B shape, 1 GB300; % bf16 tensor-co
 UNIT = "tokens/s/block"
 FALLBACK_SUSTAINED_TFLOPS = 1700.0  # profiling recipe's sustained figure, used if no measured file
 
-# dram bytes per launch of k_gram_cross_tc from an ncu capture (see profiles/), valid only for
-# the kernel source whose sha256 prefix is given; otherwise traffic is reported as null
-GRAM_TC_TRAFFIC = {"sha256": "4c359b83e81645d7", "read_per_token_block": 39725.0,
-                   "write_per_block": 91.047e6, "source": "profiles/gram_cross_tc_qwen2.5-7b.md"}
+# dram bytes (read + write) per launch of k_gram_cross_tc from a one-pass ncu capture of this
+# workload (profiles/gram_cross_tc_qwen2.5-7b.md), valid only for the kernel source whose sha256
+# prefix is given and for the captured (L, N, d); otherwise traffic is reported as null
+GRAM_TC_TRAFFIC = {"sha256": "8cdf0222cc14cd98", "L": 28, "N": 131072, "d": 3584,
+                   "read": 213542255104, "write": 3000712960,
+                   "source": "profiles/gram_cross_tc_qwen2.5-7b.md"}
 
 
 def parse():
@@ -325,9 +327,8 @@ def main():
     src = open(os.path.join(ROOT, "paper_2608_03020_gb300", "csrc", "gram_tc.cu"), "rb").read()
     sha = hashlib.sha256(src).hexdigest()[:16]
     traffic = None
-    if GRAM_TC_TRAFFIC["sha256"] == sha:
-        # dram bytes per launch, scaled from a smaller ncu capture of the same kernel source
-        traffic = GRAM_TC_TRAFFIC["read_per_token_block"] * L * N + GRAM_TC_TRAFFIC["write_per_block"] * L
+    if GRAM_TC_TRAFFIC["sha256"] == sha and (GRAM_TC_TRAFFIC["L"], GRAM_TC_TRAFFIC["N"], GRAM_TC_TRAFFIC["d"]) == (L, N, d):
+        traffic = float(GRAM_TC_TRAFFIC["read"] + GRAM_TC_TRAFFIC["write"])
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "traffic": traffic, "kernel": "k_gram_cross_tc",
                 "peak_kind": f"bf16 dense sustained, {peak_kind}", "flops_per_launch": flops}
