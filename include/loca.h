@@ -148,6 +148,34 @@ int loca_accumulate(const void* X, const void* T, int dtype, int32_t L, int64_t 
                     double* xsq_total, void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * loca_accumulate_streamed — loca_accumulate with X read from host memory (Eqs. 6, 9, 10; S7,
+ * S8: the same statistics, the same results).  For activations kept in host memory (a
+ * calibration set larger than device memory, or a producer on the CPU side): X_host is copied
+ * to the device group by group of `group` blocks and the statistics of group g run while group
+ * g + 1 is being copied, so the copy time and the kernel time overlap instead of adding up.
+ *
+ * X_host   L x N x d host array of `dtype` (page-locked memory gives the full copy rate;
+ *          pageable memory works, but the driver stages each copy and the call then waits for
+ *          it on the host).
+ * staging  device array of at least 2 x group x N x d elements of `dtype`, 16-byte aligned: two
+ *          copy slots used alternately; on return it holds the last one or two groups.
+ * group    blocks per copy (1 <= group; values above L are clamped to L).
+ * T, tsq, eta, zero_first, gram, cross, xsq_total, dtype, workspace: as loca_accumulate
+ *          (workspace size: loca_accumulate_workspace_size).
+ *
+ * Ordering: the kernels run on `stream`, each after the copy of its group.  The copies run
+ * on a copy stream that the library creates on the first call on each device (with four
+ * events; no device memory is allocated).  A copy into a slot waits for the kernels that last
+ * read that slot (in this or an earlier call), but not for any other work on `stream`: the
+ * caller must not let other queued work read or write `staging`.  X_host must stay valid and
+ * unchanged until the copies have run (synchronise `stream` before reusing it).
+ */
+int loca_accumulate_streamed(const void* X_host, void* staging, const void* T, int dtype, int32_t L,
+                             int64_t N, int64_t d, int32_t group, const double* tsq, float eta,
+                             int zero_first, float* gram, float* cross, double* xsq_total,
+                             void* workspace, size_t workspace_bytes, void* stream);
+
+/*
  * loca_batch_step and loca_gram_cross — the two halves of loca_accumulate, for callers that
  * schedule them separately (for example to time the tensor-core kernel on its own).
  *

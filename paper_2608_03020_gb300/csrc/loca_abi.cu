@@ -135,6 +135,43 @@ int check_ws(void* ws, size_t have, size_t need) {
 
 char* ws_at(void* ws, size_t off) { return static_cast<char*>(ws) + off; }
 
+// Per-device copy stream and events of loca_accumulate_streamed: copied[s] marks the end of the
+// latest copy into staging slot s, consumed[s] the end of the kernels that last read slot s.
+struct CopyLane {
+  cudaStream_t copy = nullptr;
+  cudaEvent_t copied[2] = {nullptr, nullptr};
+  cudaEvent_t consumed[2] = {nullptr, nullptr};
+  std::mutex mu;  // one call enqueues its copy / wait / record sequence at a time
+};
+
+CopyLane* copy_lane() {
+  static CopyLane* lanes[kMaxDevices] = {};
+  static std::mutex mu;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lock(mu);
+  if (lanes[dev] == nullptr) {
+    CopyLane* c = new CopyLane();
+    cudaError_t e = cudaStreamCreateWithFlags(&c->copy, cudaStreamNonBlocking);
+    for (int i = 0; i < 2 && e == cudaSuccess; ++i) {
+      e = cudaEventCreateWithFlags(&c->copied[i], cudaEventDisableTiming);
+      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->consumed[i], cudaEventDisableTiming);
+    }
+    if (e != cudaSuccess) {
+      for (int i = 0; i < 2; ++i) {
+        if (c->copied[i]) cudaEventDestroy(c->copied[i]);
+        if (c->consumed[i]) cudaEventDestroy(c->consumed[i]);
+      }
+      if (c->copy) cudaStreamDestroy(c->copy);
+      delete c;
+      fail(LOCA_ERR_CUDA, "cannot create the copy stream and events: %s", cudaGetErrorString(e));
+      return nullptr;
+    }
+    lanes[dev] = c;
+  }
+  return lanes[dev];
+}
+
 }  // namespace
 
 extern "C" {
@@ -342,6 +379,60 @@ int loca_accumulate(const void* X, const void* T, int dtype, int32_t L, int64_t 
   if (rc != LOCA_OK) return rc;
   return run_gram_cross(X, T, dtype, L, N, d, alpha, zero_first, gram, cross,
                         reinterpret_cast<int32_t*>(ws_at(workspace, lay.abort_flag)), s);
+}
+
+int loca_accumulate_streamed(const void* X_host, void* staging, const void* T, int dtype, int32_t L,
+                             int64_t N, int64_t d, int32_t group, const double* tsq, float eta,
+                             int zero_first, float* gram, float* cross, double* xsq_total,
+                             void* workspace, size_t workspace_bytes, void* stream) {
+  g_msg[0] = 0;
+  int rc = validate_stats_inputs(staging, T, dtype, L, N, d, true);
+  if (rc != LOCA_OK) return rc;
+  if (N > 0 && !X_host) return fail(LOCA_ERR_INVALID_ARG, "X_host is required");
+  if (group < 1) return fail(LOCA_ERR_SHAPE, "need group >= 1, got %d", group);
+  if (group > L) group = L;
+  if (!(eta >= 0.f)) return fail(LOCA_ERR_INVALID_ARG, "eta must be >= 0");
+  if (!tsq || !gram || !cross || !xsq_total)
+    return fail(LOCA_ERR_INVALID_ARG, "tsq, gram, cross and xsq_total are required");
+  if (!aligned(gram, 16) || !aligned(cross, 16) || !aligned(tsq, 8) || !aligned(xsq_total, 8))
+    return fail(LOCA_ERR_ALIGNMENT, "gram and cross need 16-byte, tsq and xsq_total 8-byte alignment");
+  const AccumWs lay = accum_ws(L);
+  rc = check_ws(workspace, workspace_bytes, lay.total);
+  if (rc != LOCA_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  float* alpha = reinterpret_cast<float*>(ws_at(workspace, lay.alpha));
+  double* partials = reinterpret_cast<double*>(ws_at(workspace, lay.partials));
+  int32_t* flags = reinterpret_cast<int32_t*>(ws_at(workspace, lay.abort_flag));
+  if (N == 0)  // nothing to copy: the statistics of an empty batch
+    return loca_accumulate(staging, T, dtype, L, N, d, tsq, eta, zero_first, gram, cross, xsq_total,
+                           workspace, workspace_bytes, stream);
+  CopyLane* lane = copy_lane();
+  if (!lane) return LOCA_ERR_CUDA;  // message set by copy_lane
+  std::lock_guard<std::mutex> lock(lane->mu);
+  const size_t es = dtype == LOCA_BF16 ? 2 : 4;
+  const size_t block_bytes = size_t(N) * size_t(d) * es;
+  const size_t dd = size_t(d) * size_t(d);
+  for (int32_t l0 = 0, g = 0; l0 < L; l0 += group, ++g) {
+    const int32_t nb = (L - l0 < group) ? L - l0 : group;
+    const int slot = g & 1;
+    char* dst = static_cast<char*>(staging) + size_t(slot) * size_t(group) * block_bytes;
+    const char* src = static_cast<const char*>(X_host) + size_t(l0) * block_bytes;
+    cudaError_t e = cudaStreamWaitEvent(lane->copy, lane->consumed[slot], 0);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(dst, src, size_t(nb) * block_bytes, cudaMemcpyHostToDevice, lane->copy);
+    if (e == cudaSuccess) e = cudaEventRecord(lane->copied[slot], lane->copy);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, lane->copied[slot], 0);
+    if (e != cudaSuccess) return cuda_fail(e, "streamed accumulate: copy");
+    const char* Tg = static_cast<const char*>(T) + size_t(l0) * block_bytes;
+    rc = run_batch_step(dst, dtype, nb, N, d, tsq + l0, eta, zero_first, xsq_total + l0, alpha + l0,
+                        partials + size_t(l0) * size_t(sumsq_num_partials()), s);
+    if (rc != LOCA_OK) return rc;
+    rc = run_gram_cross(dst, Tg, dtype, nb, N, d, alpha + l0, zero_first, gram + size_t(l0) * dd,
+                        cross + size_t(l0) * dd, flags, s);
+    if (rc != LOCA_OK) return rc;
+    e = cudaEventRecord(lane->consumed[slot], s);
+    if (e != cudaSuccess) return cuda_fail(e, "streamed accumulate: event");
+  }
+  return LOCA_OK;
 }
 
 int loca_ridge_solve_workspace_size(int32_t L, int64_t d, int32_t k, size_t* bytes) {

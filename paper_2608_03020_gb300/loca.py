@@ -44,6 +44,8 @@ SIGNATURES = [
      [_P, _P, ctypes.c_int, _I32, _I64, _I64, _P, _F, ctypes.c_int, _P, _P, _P, _P, _SZ, _P]),
     ("loca_accumulate_noalloc", ctypes.c_int,
      [_P, _P, ctypes.c_int, _I32, _I64, _I64, _P, _F, ctypes.c_int, _P, _P, _P, _P]),
+    ("loca_accumulate_streamed", ctypes.c_int,
+     [_P, _P, _P, ctypes.c_int, _I32, _I64, _I64, _I32, _P, _F, ctypes.c_int, _P, _P, _P, _P, _SZ, _P]),
     ("loca_batch_step_workspace_size", ctypes.c_int, [_I32, ctypes.POINTER(_SZ)]),
     ("loca_batch_step", ctypes.c_int, [_P, ctypes.c_int, _I32, _I64, _I64, _P, _F, ctypes.c_int, _P, _P, _P, _SZ, _P]),
     ("loca_gram_cross_workspace_size", ctypes.c_int, [ctypes.POINTER(_SZ)]),
@@ -230,6 +232,35 @@ def loca_accumulate_noalloc(X, T, tsq, eta, gram, cross, xsq_total, zero_first, 
                                        int(bool(zero_first)), _ptr(gram), _ptr(cross), _ptr(xsq_total),
                                        _stream(stream))
     _check(rc, "loca_accumulate_noalloc")
+
+
+def loca_accumulate_streamed(X_host, staging, T, tsq, eta, gram, cross, xsq_total, zero_first, group=2,
+                             workspace=None, stream=None):
+    """loca_accumulate with X in host memory: X_host (L x N x d, CPU tensor, ideally pinned) is
+    copied to the device `group` blocks at a time into `staging` (a device tensor with room for
+    2 x group x N x d elements, used as two alternating slots) while the statistics of the
+    previous group run on the stream."""
+    if not isinstance(X_host, torch.Tensor) or X_host.is_cuda or X_host.dim() != 3 or not X_host.is_contiguous():
+        raise TypeError("X_host must be a contiguous 3-D CPU tensor")
+    _dev(staging, "staging", X_host.dtype)
+    _dev(T, "T", X_host.dtype, 3)
+    _dev(tsq, "tsq", torch.float64, 1)
+    _dev(gram, "gram", torch.float32, 3)
+    _dev(cross, "cross", torch.float32, 3)
+    _dev(xsq_total, "xsq_total", torch.float64, 1)
+    L, N, d = X_host.shape
+    group = max(1, min(int(group), L))
+    if tuple(T.shape) != (L, N, d) or tuple(gram.shape) != (L, d, d) or tuple(cross.shape) != (L, d, d):
+        raise ValueError("shape mismatch among X_host, T (L x N x d) and gram, cross (L x d x d)")
+    if staging.numel() < 2 * group * N * d:
+        raise ValueError(f"staging has {staging.numel()} elements, need 2 x group x N x d = {2 * group * N * d}")
+    nbytes = accumulate_workspace_size(L, N, d, X_host.dtype)
+    ws = _workspace(nbytes, T.device, workspace)
+    rc = lib().loca_accumulate_streamed(ctypes.c_void_p(X_host.data_ptr()), _ptr(staging), _ptr(T),
+                                        _code(X_host.dtype), L, N, d, group, _ptr(tsq), float(eta),
+                                        int(bool(zero_first)), _ptr(gram), _ptr(cross), _ptr(xsq_total),
+                                        _ptr(ws), nbytes, _stream(stream))
+    _check(rc, "loca_accumulate_streamed")
 
 
 def batch_step_workspace_size(L) -> int:

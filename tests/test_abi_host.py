@@ -106,6 +106,11 @@ def test_validation_codes(L):
     lam = (ctypes.c_float * 1)(1e-3)
     assert L.loca_ridge_solve(fake, fake, None, fake, None, lam, 1, 2, 64, 33, fake, fake, None, None,
                               fake, 1 << 24, None) == 2
+    # streamed accumulate: group < 1, missing host X
+    assert L.loca_accumulate_streamed(fake, fake, fake, 1, 2, 64, 64, 0, fake, ctypes.c_float(0.01), 1, fake,
+                                      fake, fake, fake, 1 << 20, None) == 2
+    assert L.loca_accumulate_streamed(None, fake, fake, 1, 2, 64, 64, 1, fake, ctypes.c_float(0.01), 1, fake,
+                                      fake, fake, fake, 1 << 20, None) == 1
     # calibration: r > m
     assert L.loca_calib_fit(fake, fake, 16, 4, 64, 2, ctypes.c_float(0.1), 5, fake, fake, None, fake,
                             1 << 20, None) == 2

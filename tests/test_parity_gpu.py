@@ -235,6 +235,56 @@ def test_zero_targets_give_zero_cross(lc):
     assert torch.count_nonzero(cross) == 0
 
 
+@pytest.mark.parametrize("dtype,L,N,d,group,pinned", [
+    ("bf16", 5, 1000, 328, 2, True),
+    ("bf16", 3, 2048, 512, 1, False),
+    ("bf16", 4, 700, 896, 4, True),
+    ("f32", 3, 300, 72, 2, True),
+])
+def test_accumulate_streamed_matches_device_path(lc, dtype, L, N, d, group, pinned):
+    """Eqs. 6, 9, 10; S7.  X streamed from host memory in groups of blocks gives the statistics of
+    the device-resident call: Gram and cross bit for bit where each block's step is the same
+    (the kernels of one block do not depend on the other blocks), xsq / alpha to the rounding of
+    a differently split fp64 sum.  Two calls in a row (overwrite, then accumulate) also exercise
+    the reuse of the two staging slots across calls; checked against the oracle as well."""
+    tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    eta = 0.02
+    Xs, Ts, ref, got, hosts = [], [], [], [], []
+    staging = torch.empty((2 * group, N, d), dtype=tdt, device="cuda")
+    for rep in range(2):
+        X, T = _synthetic_stats_inputs(L, N, d, dtype, seed=77 + rep + d)
+        Xs.append(X)
+        Ts.append(T)
+        Xd, Td = _dev(X, tdt), _dev(T, tdt)
+        tsq = _dev(np.array([np.sum(T[l] ** 2) for l in range(L)]), torch.float64)
+        Xh = Xd.cpu()
+        if pinned:
+            Xh = Xh.pin_memory()
+        hosts.append(Xh)  # host memory must outlive the copies the call queues
+        # device-resident reference call and streamed call, each continuing its own accumulators
+        if rep == 0:
+            dg = torch.empty((L, d, d), device="cuda"); dc = torch.empty_like(dg)
+            dx = torch.empty((L,), dtype=torch.float64, device="cuda")
+            sg = torch.empty_like(dg); sc = torch.empty_like(dg); sx = torch.empty_like(dx)
+            ref.append((dg, dc, dx))
+            got.append((sg, sc, sx))
+        dg, dc, dx = ref[0]
+        sg, sc, sx = got[0]
+        lc.loca_accumulate(Xd, Td, tsq, eta, dg, dc, dx, zero_first=(rep == 0))
+        lc.loca_accumulate_streamed(Xh, staging, Td, tsq, eta, sg, sc, sx, zero_first=(rep == 0), group=group)
+    torch.cuda.synchronize()
+    assert lc.loca_device_status() == 0
+    dg, dc, dx = ref[0]
+    sg, sc, sx = got[0]
+    assert torch.equal(sg, dg)
+    tol = 1e-6
+    assert _rel(_np(sc), _np(dc)) <= tol
+    assert np.allclose(_np(sx), _np(dx), rtol=1e-12, atol=0)
+    g_ref, c_ref, x_ref = O.accumulate_stats(Xs, Ts, eta)
+    t = 1e-5 if dtype == "f32" else 2e-3
+    assert _rel(_np(sg), g_ref) <= t and _rel(_np(sc), c_ref) <= t
+
+
 # ------------------------------------------------------------------------- ridge solve
 
 @pytest.mark.parametrize("k,d,L,with_prev,relative", [
