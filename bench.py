@@ -393,9 +393,14 @@ def main():
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        tokens = 8192
+        # bounded sample: one block, a token prefix sized from a 2048-token pilot run to take about
+        # 15 s of CPU time (capped at the full N)
+        pilot = min(2048, N)
+        host = host_sample(w, tokens=pilot)
+        oracle_sample(w, min(512, pilot), host)
+        per_token = oracle_sample(w, pilot, host) / pilot
+        tokens = int(min(N, max(pilot, (15.0 / max(per_token, 1e-9)) // 1024 * 1024)))
         host = host_sample(w, tokens=tokens)
-        oracle_sample(w, 512, host)
         sec = oracle_sample(w, tokens, host)
         cpu = {"value": tokens / sec, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
                "sample": f"one block (of {L}), first {tokens} of {N} tokens, full d={d}, C={C}, r={r}, k={k}; "
