@@ -176,6 +176,19 @@ int loca_accumulate_streamed(const void* X_host, void* staging, const void* T, i
                              void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * loca_host_alloc / loca_host_free — host memory for inputs streamed to the GPU (for example
+ * X_host of loca_accumulate_streamed).  The paper has no counterpart: this concerns only the
+ * speed of host-to-device copies.  Page-locked memory with 4 KiB pages copies at a rate that
+ * varies widely once buffers reach tens of GB; this memory is backed by 2 MiB pages (anonymous
+ * mapping, transparent huge pages advised, touched once in parallel) and registered with CUDA,
+ * and copies at the full link rate.  Contents start at zero.  The size is rounded up to a
+ * multiple of 2 MiB.  Free with loca_host_free (it unregisters and unmaps); a pointer not
+ * returned by loca_host_alloc is rejected with LOCA_ERR_INVALID_ARG.  Needs a CUDA device.
+ */
+int loca_host_alloc(size_t bytes, void** ptr /* host, out */);
+int loca_host_free(void* ptr);
+
+/*
  * loca_batch_step and loca_gram_cross — the two halves of loca_accumulate, for callers that
  * schedule them separately (for example to time the tensor-core kernel on its own).
  *

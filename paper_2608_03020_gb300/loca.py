@@ -46,6 +46,8 @@ SIGNATURES = [
      [_P, _P, ctypes.c_int, _I32, _I64, _I64, _P, _F, ctypes.c_int, _P, _P, _P, _P]),
     ("loca_accumulate_streamed", ctypes.c_int,
      [_P, _P, _P, ctypes.c_int, _I32, _I64, _I64, _I32, _P, _F, ctypes.c_int, _P, _P, _P, _P, _SZ, _P]),
+    ("loca_host_alloc", ctypes.c_int, [_SZ, ctypes.POINTER(ctypes.c_void_p)]),
+    ("loca_host_free", ctypes.c_int, [_P]),
     ("loca_batch_step_workspace_size", ctypes.c_int, [_I32, ctypes.POINTER(_SZ)]),
     ("loca_batch_step", ctypes.c_int, [_P, ctypes.c_int, _I32, _I64, _I64, _P, _F, ctypes.c_int, _P, _P, _P, _SZ, _P]),
     ("loca_gram_cross_workspace_size", ctypes.c_int, [ctypes.POINTER(_SZ)]),
@@ -232,6 +234,36 @@ def loca_accumulate_noalloc(X, T, tsq, eta, gram, cross, xsq_total, zero_first, 
                                        int(bool(zero_first)), _ptr(gram), _ptr(cross), _ptr(xsq_total),
                                        _stream(stream))
     _check(rc, "loca_accumulate_noalloc")
+
+
+class _HostBlock:
+    """Owns one loca_host_alloc buffer; freed when the last tensor viewing it is gone."""
+
+    def __init__(self, nbytes):
+        p = ctypes.c_void_p(0)
+        _check(lib().loca_host_alloc(nbytes, ctypes.byref(p)), "loca_host_alloc")
+        self.ptr = p.value
+
+    def __del__(self):
+        if getattr(self, "ptr", None):
+            lib().loca_host_free(ctypes.c_void_p(self.ptr))
+            self.ptr = None
+
+
+def host_empty(shape, dtype):
+    """A CPU tensor in loca_host_alloc memory (page-locked, 2 MiB pages, zero-filled): host
+    inputs in it copy to the GPU at the full link rate."""
+    shape = tuple(int(s) for s in shape)
+    n = 1
+    for s in shape:
+        n *= s
+    nbytes = n * torch.empty((), dtype=dtype).element_size()
+    if nbytes == 0:
+        return torch.empty(shape, dtype=dtype)
+    owner = _HostBlock(nbytes)
+    buf = (ctypes.c_uint8 * nbytes).from_address(owner.ptr)
+    buf.owner = owner  # the tensor keeps `buf` alive, `buf` keeps the allocation
+    return torch.frombuffer(buf, dtype=dtype).view(shape)
 
 
 def loca_accumulate_streamed(X_host, staging, T, tsq, eta, gram, cross, xsq_total, zero_first, group=2,

@@ -111,6 +111,9 @@ def test_validation_codes(L):
                                       fake, fake, fake, 1 << 20, None) == 2
     assert L.loca_accumulate_streamed(None, fake, fake, 1, 2, 64, 64, 1, fake, ctypes.c_float(0.01), 1, fake,
                                       fake, fake, fake, 1 << 20, None) == 1
+    # host memory: freeing NULL is a no-op; a pointer the library did not hand out is rejected
+    assert L.loca_host_free(None) == 0
+    assert L.loca_host_free(fake) == 1
     # calibration: r > m
     assert L.loca_calib_fit(fake, fake, 16, 4, 64, 2, ctypes.c_float(0.1), 5, fake, fake, None, fake,
                             1 << 20, None) == 2

@@ -235,13 +235,13 @@ def test_zero_targets_give_zero_cross(lc):
     assert torch.count_nonzero(cross) == 0
 
 
-@pytest.mark.parametrize("dtype,L,N,d,group,pinned", [
-    ("bf16", 5, 1000, 328, 2, True),
-    ("bf16", 3, 2048, 512, 1, False),
-    ("bf16", 4, 700, 896, 4, True),
-    ("f32", 3, 300, 72, 2, True),
+@pytest.mark.parametrize("dtype,L,N,d,group,host", [
+    ("bf16", 5, 1000, 328, 2, "loca"),
+    ("bf16", 3, 2048, 512, 1, "pageable"),
+    ("bf16", 4, 700, 896, 4, "torch"),
+    ("f32", 3, 300, 72, 2, "loca"),
 ])
-def test_accumulate_streamed_matches_device_path(lc, dtype, L, N, d, group, pinned):
+def test_accumulate_streamed_matches_device_path(lc, dtype, L, N, d, group, host):
     """Eqs. 6, 9, 10; S7.  X streamed from host memory in groups of blocks gives the statistics of
     the device-resident call: Gram and cross bit for bit where each block's step is the same
     (the kernels of one block do not depend on the other blocks), xsq / alpha to the rounding of
@@ -258,8 +258,10 @@ def test_accumulate_streamed_matches_device_path(lc, dtype, L, N, d, group, pinn
         Xd, Td = _dev(X, tdt), _dev(T, tdt)
         tsq = _dev(np.array([np.sum(T[l] ** 2) for l in range(L)]), torch.float64)
         Xh = Xd.cpu()
-        if pinned:
+        if host == "torch":
             Xh = Xh.pin_memory()
+        elif host == "loca":
+            Xh = lc.host_empty(Xh.shape, Xh.dtype).copy_(Xh)
         hosts.append(Xh)  # host memory must outlive the copies the call queues
         # device-resident reference call and streamed call, each continuing its own accumulators
         if rep == 0:
@@ -283,6 +285,27 @@ def test_accumulate_streamed_matches_device_path(lc, dtype, L, N, d, group, pinn
     g_ref, c_ref, x_ref = O.accumulate_stats(Xs, Ts, eta)
     t = 1e-5 if dtype == "f32" else 2e-3
     assert _rel(_np(sg), g_ref) <= t and _rel(_np(sc), c_ref) <= t
+
+
+def test_host_empty_is_pinned_zeroed_and_freed(lc):
+    """loca_host_alloc memory: page-locked (device-visible), zero-filled, rounded to 2 MiB, and
+    released when the last tensor viewing it goes away (allocating again reuses the space)."""
+    import gc
+
+    for _ in range(3):
+        h = lc.host_empty((3, 1000, 333), torch.bfloat16)
+        assert h.is_pinned() and h.shape == (3, 1000, 333)
+        assert torch.count_nonzero(h) == 0
+        v = h[1]
+        del h
+        gc.collect()
+        v.fill_(2.0)  # the view keeps the allocation alive
+        d = v.to("cuda", non_blocking=True)
+        torch.cuda.synchronize()
+        assert float(d.float().sum()) == 2.0 * 1000 * 333
+        del v, d
+        gc.collect()
+    assert lc.host_empty((0, 5), torch.float32).numel() == 0
 
 
 # ------------------------------------------------------------------------- ridge solve
