@@ -176,6 +176,48 @@ int loca_accumulate_streamed(const void* X_host, void* staging, const void* T, i
                              void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * loca_kspace_accumulate / loca_kspace_solve — the paper's own statistics in adapter space
+ * (Eqs. 6, 8, 9; S7, S8) instead of the d x d Gram and cross product: the same solved system
+ * (Theorem S6), O(L (k^2 + C k)) state, and one HBM read of X per block and mini-batch.
+ *
+ * loca_kspace_accumulate, for every block l, with p_n = A_l^T x_n (Eq. 9's features) and the
+ * targets q_n = (e_n P_l) Q_l applied through the factors (S3, S11; T is never formed):
+ *   xsq_b[l]  = ||X_l||_F^2;   tsq_b[l] = sum_n ||q_n||^2 = sum_n u_n^T (Q_l Q_l^T) u_n, u_n = e_n P_l
+ *   alpha[l]  = -eta sqrt(xsq_b[l] / tsq_b[l])  (0 if tsq_b[l] == 0; = -eta_bar, Eq. 10, S8)
+ *   G_l      (+)= sum_n p_n p_n^T                       (k x k)
+ *   SC_l     (+)= alpha[l] sum_n e_n p_n^T              (C x k)
+ *   xsq_total[l] (+)= xsq_b[l]
+ * so that C_l = B_prev,l G_l + Q_l^T (P_l^T SC_l) = sum_n rho_n p_n^T with
+ * rho_n = B_prev p_n - eta_bar q_n (Eq. 6).  zero_first != 0 overwrites instead of adding.
+ *   X  L x N x d bf16 (LOCA_BF16 only), 16-byte aligned, d % 8 == 0;  A  L x d x k float (k <= 32);
+ *   E  N x C float (C <= 16);  P  L x C x r float, Q  L x r x d float (r <= 32);
+ *   G  L x k x k float;  SC  L x C x k float;  xsq_total  L double;  alpha  L float or NULL.
+ *   Workspace: loca_kspace_workspace_size (holds X A_l, N x kp floats per block, kp = 16 or 32,
+ *   and per-tile partial sums).
+ *   Arithmetic: X A_l on the tensor cores with A_l split into two bf16 parts (A_l to 2^-16) and
+ *   fp32 accumulation; the token sums in fp32 over 128 tokens, fp64 across; fixed-order
+ *   reductions (deterministic).
+ *
+ * loca_kspace_solve (Eq. 8; Theorem S6; S7): for every candidate j and block l,
+ *   lambda_{j,l} = lambda_rel[j] * xsq_total[l] / d  (absolute lambda_rel if xsq_total == NULL),
+ *   B[j, l] = C_l (G_l + lambda I)^-1 by Cholesky (no inverse), C_l as above.
+ *   lambda_rel: nl host floats (nl <= 16, each > 0); B: nl x L x d x k float; info: nl x L int32
+ *   (0, or the order of the first non-positive leading minor; then B[j, l] is zero);
+ *   B_prev: L x d x k or NULL (= 0); C_out: L x d x k or NULL.
+ */
+int loca_kspace_workspace_size(int32_t L, int64_t N, int64_t d, int32_t k, int32_t C, int32_t r,
+                               size_t* bytes /* host */);
+int loca_kspace_accumulate(const void* X, int dtype, int32_t L, int64_t N, int64_t d, const float* A,
+                           int32_t k, const float* E, int32_t C, const float* P, const float* Q,
+                           int32_t r, float eta, int zero_first, float* G, float* SC,
+                           double* xsq_total, float* alpha, void* workspace, size_t workspace_bytes,
+                           void* stream);
+int loca_kspace_solve(const float* G, const float* SC, const double* xsq_total, const float* P,
+                      const float* Q, const float* B_prev, const float* lambda_rel /* host */,
+                      int32_t nl, int32_t L, int64_t d, int32_t k, int32_t C, int32_t r, float* B,
+                      int32_t* info, float* C_out, void* stream);
+
+/*
  * loca_host_alloc / loca_host_free — host memory for inputs streamed to the GPU (for example
  * X_host of loca_accumulate_streamed).  The paper has no counterpart: this concerns only the
  * speed of host-to-device copies.  Page-locked memory with 4 KiB pages copies at a rate that

@@ -435,6 +435,80 @@ int loca_accumulate_streamed(const void* X_host, void* staging, const void* T, i
   return LOCA_OK;
 }
 
+int loca_kspace_workspace_size(int32_t L, int64_t N, int64_t d, int32_t k, int32_t C, int32_t r, size_t* bytes) {
+  if (!bytes) return fail(LOCA_ERR_INVALID_ARG, "bytes is NULL");
+  if (L < 1 || N < 0 || d < 1 || k < 1 || k > 32 || C < 1 || C > kspace_max_C() || r < 1 || r > kspace_max_r())
+    return fail(LOCA_ERR_SHAPE, "need L >= 1, N >= 0, d >= 1, 1 <= k <= 32, 1 <= C <= %d, 1 <= r <= %d",
+                kspace_max_C(), kspace_max_r());
+  *bytes = kspace_ws(L, N, d, k, C, r).total;
+  return LOCA_OK;
+}
+
+int loca_kspace_accumulate(const void* X, int dtype, int32_t L, int64_t N, int64_t d, const float* A, int32_t k,
+                           const float* E, int32_t C, const float* P, const float* Q, int32_t r, float eta,
+                           int zero_first, float* G, float* SC, double* xsq_total, float* alpha,
+                           void* workspace, size_t workspace_bytes, void* stream) {
+  g_msg[0] = 0;
+  if (dtype != LOCA_BF16) return fail(LOCA_ERR_UNSUPPORTED_DTYPE, "the k-space path takes bf16 X (dtype LOCA_BF16)");
+  if (L < 1 || L > 65535 || N < 0 || N > 2147483647LL || d < 1 || d > 65536)
+    return fail(LOCA_ERR_SHAPE, "need 1 <= L <= 65535, 0 <= N < 2^31, 1 <= d <= 65536");
+  if (d % 8 != 0) return fail(LOCA_ERR_SHAPE, "need d %% 8 == 0 (16-byte rows), got d=%lld", (long long)d);
+  if (k < 1 || k > 32 || k > d) return fail(LOCA_ERR_SHAPE, "need 1 <= k <= min(d, 32), got k=%d", k);
+  if (C < 1 || C > kspace_max_C()) return fail(LOCA_ERR_SHAPE, "need 1 <= C <= %d, got C=%d", kspace_max_C(), C);
+  if (r < 1 || r > kspace_max_r()) return fail(LOCA_ERR_SHAPE, "need 1 <= r <= %d, got r=%d", kspace_max_r(), r);
+  if (!(eta >= 0.f)) return fail(LOCA_ERR_INVALID_ARG, "eta must be >= 0");
+  if ((N > 0 && (!X || !E)) || !A || !P || !Q || !G || !SC || !xsq_total)
+    return fail(LOCA_ERR_INVALID_ARG, "X, A, E, P, Q, G, SC and xsq_total are required");
+  if ((X && !aligned(X, 16)) || !aligned(A, 4) || (E && !aligned(E, 4)) || !aligned(P, 4) || !aligned(Q, 4) ||
+      !aligned(G, 4) || !aligned(SC, 4) || !aligned(xsq_total, 8) || (alpha && !aligned(alpha, 4)))
+    return fail(LOCA_ERR_ALIGNMENT, "X needs 16-byte, xsq_total 8-byte, the other arrays 4-byte alignment");
+  const KspaceWs lay = kspace_ws(L, N, d, k, C, r);
+  int rc = check_ws(workspace, workspace_bytes, lay.total);
+  if (rc != LOCA_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (N == 0) {
+    if (zero_first) {
+      cudaError_t e = cudaMemsetAsync(G, 0, sizeof(float) * size_t(L) * k * k, s);
+      if (e == cudaSuccess) e = cudaMemsetAsync(SC, 0, sizeof(float) * size_t(L) * C * k, s);
+      if (e == cudaSuccess) e = cudaMemsetAsync(xsq_total, 0, sizeof(double) * size_t(L), s);
+      if (e != cudaSuccess) return cuda_fail(e, "k-space accumulate: zeroing");
+    }
+    if (alpha) {
+      cudaError_t e = cudaMemsetAsync(alpha, 0, sizeof(float) * size_t(L), s);
+      if (e != cudaSuccess) return cuda_fail(e, "k-space accumulate: zeroing");
+    }
+    return LOCA_OK;
+  }
+  int32_t* status = device_status_word();
+  if (!status) return fail(LOCA_ERR_CUDA, "cannot resolve the device status word");
+  cudaError_t e = launch_kspace_accumulate(X, L, N, d, A, k, E, C, P, Q, r, eta, zero_first, G, SC, xsq_total,
+                                           alpha, workspace, status, s);
+  if (e != cudaSuccess) return cuda_fail(e, "k-space accumulate launch");
+  return LOCA_OK;
+}
+
+int loca_kspace_solve(const float* G, const float* SC, const double* xsq_total, const float* P, const float* Q,
+                      const float* B_prev, const float* lambda_rel, int32_t nl, int32_t L, int64_t d, int32_t k,
+                      int32_t C, int32_t r, float* B, int32_t* info, float* C_out, void* stream) {
+  g_msg[0] = 0;
+  if (L < 1 || L > 65535 || d < 1) return fail(LOCA_ERR_SHAPE, "need 1 <= L <= 65535, d >= 1");
+  if (k < 1 || k > 32 || k > d) return fail(LOCA_ERR_SHAPE, "need 1 <= k <= min(d, 32), got k=%d", k);
+  if (C < 1 || C > kspace_max_C()) return fail(LOCA_ERR_SHAPE, "need 1 <= C <= %d, got C=%d", kspace_max_C(), C);
+  if (r < 1 || r > kspace_max_r()) return fail(LOCA_ERR_SHAPE, "need 1 <= r <= %d, got r=%d", kspace_max_r(), r);
+  if (nl < 1 || nl > 16) return fail(LOCA_ERR_SHAPE, "need 1 <= nl <= 16, got nl=%d", nl);
+  if (!G || !SC || !P || !Q || !lambda_rel || !B || !info)
+    return fail(LOCA_ERR_INVALID_ARG, "G, SC, P, Q, lambda_rel, B and info are required");
+  for (int j = 0; j < nl; ++j)
+    if (!(lambda_rel[j] > 0.f)) return fail(LOCA_ERR_INVALID_ARG, "lambda_rel[%d] must be > 0", j);
+  if (!aligned(G, 4) || !aligned(SC, 4) || !aligned(P, 4) || !aligned(Q, 4) || !aligned(B, 4) || !aligned(info, 4) ||
+      (B_prev && !aligned(B_prev, 4)) || (xsq_total && !aligned(xsq_total, 8)) || (C_out && !aligned(C_out, 4)))
+    return fail(LOCA_ERR_ALIGNMENT, "pointers must be aligned to their element size");
+  cudaError_t e = launch_kspace_solve(G, SC, xsq_total, P, Q, B_prev, lambda_rel, nl, L, d, k, C, r, B, info, C_out,
+                                      static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "k-space solve launch");
+  return LOCA_OK;
+}
+
 int loca_ridge_solve_workspace_size(int32_t L, int64_t d, int32_t k, size_t* bytes) {
   if (!bytes) return fail(LOCA_ERR_INVALID_ARG, "bytes is NULL");
   if (L < 1 || d < 1 || k < 1) return fail(LOCA_ERR_SHAPE, "need L, d, k >= 1");

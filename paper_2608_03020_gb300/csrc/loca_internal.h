@@ -62,6 +62,22 @@ cudaError_t launch_gram_cross_tc(const void* X, const void* T, int L, int64_t N,
                                  const float* alpha, int zero_first, float* gram, float* cross,
                                  int32_t* status, int32_t* abort_flag, cudaStream_t s);
 
+// ---- k-space statistics and solve (kspace.cu)
+struct KspaceWs {
+  size_t W, M, Xp, xsq_part, part, flags, total;
+};
+KspaceWs kspace_ws(int L, int64_t N, int64_t d, int k, int C, int r);
+int kspace_max_C();
+int kspace_max_r();
+cudaError_t launch_kspace_accumulate(const void* X, int L, int64_t N, int64_t d, const float* A, int k,
+                                     const float* E, int C, const float* P, const float* Q, int r, float eta,
+                                     int zero_first, float* G, float* SC, double* xsq_total, float* alpha_out,
+                                     void* workspace, int32_t* status, cudaStream_t s);
+cudaError_t launch_kspace_solve(const float* G, const float* SC, const double* xsq_total, const float* P,
+                                const float* Q, const float* B_prev, const float* lambda_rel, int nl, int L,
+                                int64_t d, int k, int C, int r, float* B, int32_t* info, float* C_out,
+                                cudaStream_t s);
+
 // ---- ridge solve (solve.cu)
 cudaError_t launch_project_rows(const float* gram, const float* cross, const float* A, int L,
                                 int64_t d, int k, float* GA, float* CA, cudaStream_t s);

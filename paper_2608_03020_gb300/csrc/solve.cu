@@ -10,6 +10,7 @@
 //                 by a forward and a back substitution:  B[j, l, i] = C_l[i] (G_l + lambda I)^-1.
 //                 k is padded to a compile-time size with an identity block (its solution
 //                 columns are zero), so each row's solve stays in registers.
+#include "chol.cuh"
 #include "loca_internal.h"
 
 namespace loca {
@@ -146,39 +147,8 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
       G_out[(int64_t(l) * k + a) * k + b] = float(0.5 * (double(Gf[a][b]) + double(Gf[b][a])));
     }
   }
-  // Cholesky, lower factor, column by column (warp 0; lanes over rows)
-  if (threadIdx.x < 32) {
-    const int lane = threadIdx.x;
-    int inf = 0;
-    for (int c = 0; c < KM; ++c) {
-      double diag = Md[c][c];
-      for (int t = 0; t < c; ++t) diag -= Md[c][t] * Md[c][t];
-      if (!(diag > 0.0)) {
-        inf = c + 1;
-        break;
-      }
-      const double lcc = sqrt(diag);
-      __syncwarp();
-      for (int r = c + 1 + lane; r < KM; r += 32) {
-        double v = Md[r][c];
-        for (int t = 0; t < c; ++t) v -= Md[r][t] * Md[c][t];
-        Md[r][c] = v / lcc;
-      }
-      __syncwarp();
-      if (lane == 0) Md[c][c] = lcc;
-      __syncwarp();
-    }
-    if (lane == 0) s_info = inf;
-  }
-  __syncthreads();
-  const int inf = s_info;
+  const int inf = chol_factor<KM>(Md, Lf, Linv, &s_info);
   if (threadIdx.x == 0) info[int64_t(j) * L + l] = inf;
-  for (int e = threadIdx.x; e < KM * KM; e += CS_THREADS) {
-    const int a = e / KM, b = e % KM;
-    Lf[a][b] = (b <= a) ? float(Md[a][b]) : 0.f;
-  }
-  for (int a = threadIdx.x; a < KM; a += CS_THREADS) Linv[a] = float(1.0 / Md[a][a]);
-  __syncthreads();
 
   float* Bj = B + (int64_t(j) * L + l) * d * k;
   const float* Bp = B_prev ? B_prev + int64_t(l) * d * k : nullptr;
@@ -209,22 +179,7 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
         if (s < k) Bj[i * k + s] = 0.f;
       continue;
     }
-    // forward: Lf y = c
-#pragma unroll
-    for (int s = 0; s < KM; ++s) {
-      float a = c[s];
-#pragma unroll
-      for (int t = 0; t < s; ++t) a = fmaf(-Lf[s][t], c[t], a);
-      c[s] = a * Linv[s];
-    }
-    // back: Lf^T x = y
-#pragma unroll
-    for (int s = KM - 1; s >= 0; --s) {
-      float a = c[s];
-#pragma unroll
-      for (int t = s + 1; t < KM; ++t) a = fmaf(-Lf[t][s], c[t], a);
-      c[s] = a * Linv[s];
-    }
+    chol_solve_row<KM>(Lf, Linv, c);
 #pragma unroll
     for (int s = 0; s < KM; ++s)
       if (s < k) Bj[i * k + s] = c[s];

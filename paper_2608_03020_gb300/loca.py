@@ -46,6 +46,12 @@ SIGNATURES = [
      [_P, _P, ctypes.c_int, _I32, _I64, _I64, _P, _F, ctypes.c_int, _P, _P, _P, _P]),
     ("loca_accumulate_streamed", ctypes.c_int,
      [_P, _P, _P, ctypes.c_int, _I32, _I64, _I64, _I32, _P, _F, ctypes.c_int, _P, _P, _P, _P, _SZ, _P]),
+    ("loca_kspace_workspace_size", ctypes.c_int, [_I32, _I64, _I64, _I32, _I32, _I32, ctypes.POINTER(_SZ)]),
+    ("loca_kspace_accumulate", ctypes.c_int,
+     [_P, ctypes.c_int, _I32, _I64, _I64, _P, _I32, _P, _I32, _P, _P, _I32, _F, ctypes.c_int, _P, _P, _P, _P, _P,
+      _SZ, _P]),
+    ("loca_kspace_solve", ctypes.c_int,
+     [_P, _P, _P, _P, _P, _P, ctypes.POINTER(_F), _I32, _I32, _I64, _I32, _I32, _I32, _P, _P, _P, _P]),
     ("loca_host_alloc", ctypes.c_int, [_SZ, ctypes.POINTER(ctypes.c_void_p)]),
     ("loca_host_free", ctypes.c_int, [_P]),
     ("loca_batch_step_workspace_size", ctypes.c_int, [_I32, ctypes.POINTER(_SZ)]),
@@ -293,6 +299,65 @@ def loca_accumulate_streamed(X_host, staging, T, tsq, eta, gram, cross, xsq_tota
                                         int(bool(zero_first)), _ptr(gram), _ptr(cross), _ptr(xsq_total),
                                         _ptr(ws), nbytes, _stream(stream))
     _check(rc, "loca_accumulate_streamed")
+
+
+def kspace_workspace_size(L, N, d, k, C, r) -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib().loca_kspace_workspace_size(L, N, d, k, C, r, ctypes.byref(out)), "loca_kspace_workspace_size")
+    return out.value
+
+
+def loca_kspace_accumulate(X, A, E, P, Q, eta, G, SC, xsq_total, zero_first, alpha=None, workspace=None,
+                           stream=None):
+    """The paper's k-space statistics of one mini-batch: G_l (+)= (X_l A_l)^T (X_l A_l),
+    SC_l (+)= alpha_l E^T (X_l A_l), xsq_total (+)= ||X_l||^2, with alpha_l = -eta RMS(X_l)/RMS(T_l)
+    and T_l = E P_l Q_l never formed."""
+    _dev(X, "X", torch.bfloat16, 3)
+    _dev(A, "A", torch.float32, 3)
+    _dev(E, "E", torch.float32, 2)
+    _dev(P, "P", torch.float32, 3)
+    _dev(Q, "Q", torch.float32, 3)
+    _dev(G, "G", torch.float32, 3)
+    _dev(SC, "SC", torch.float32, 3)
+    _dev(xsq_total, "xsq_total", torch.float64, 1)
+    _dev(alpha, "alpha", torch.float32, 1)
+    L, N, d = X.shape
+    k = A.shape[2]
+    C, r = P.shape[1], P.shape[2]
+    if (tuple(A.shape) != (L, d, k) or tuple(E.shape) != (N, C) or tuple(Q.shape) != (L, r, d)
+            or tuple(G.shape) != (L, k, k) or tuple(SC.shape) != (L, C, k) or P.shape[0] != L):
+        raise ValueError("shape mismatch among X, A, E, P, Q, G, SC")
+    nbytes = kspace_workspace_size(L, N, d, k, C, r)
+    ws = _workspace(nbytes, X.device, workspace)
+    rc = lib().loca_kspace_accumulate(_ptr(X), LOCA_BF16, L, N, d, _ptr(A), k, _ptr(E), C, _ptr(P), _ptr(Q), r,
+                                      float(eta), int(bool(zero_first)), _ptr(G), _ptr(SC), _ptr(xsq_total),
+                                      _ptr(alpha), _ptr(ws), nbytes, _stream(stream))
+    _check(rc, "loca_kspace_accumulate")
+
+
+def loca_kspace_solve(G, SC, P, Q, lambda_rel, B, info, xsq_total=None, B_prev=None, C_out=None, stream=None):
+    """Ridge solves from the k-space statistics: B[j, l] (G_l + lambda_j I) = C_l with
+    C_l = B_prev,l G_l + Q_l^T (P_l^T SC_l); lambda_j = lambda_rel[j] xsq_total[l] / d."""
+    _dev(G, "G", torch.float32, 3)
+    _dev(SC, "SC", torch.float32, 3)
+    _dev(P, "P", torch.float32, 3)
+    _dev(Q, "Q", torch.float32, 3)
+    _dev(B, "B", torch.float32, 4)
+    _dev(info, "info", torch.int32, 2)
+    _dev(xsq_total, "xsq_total", torch.float64, 1)
+    _dev(B_prev, "B_prev", torch.float32, 3)
+    _dev(C_out, "C_out", torch.float32, 3)
+    L, k, _ = G.shape
+    C, r = P.shape[1], P.shape[2]
+    d = Q.shape[2]
+    lam = [float(v) for v in lambda_rel]
+    nl = len(lam)
+    if tuple(B.shape) != (nl, L, d, k) or tuple(info.shape) != (nl, L) or tuple(SC.shape) != (L, C, k):
+        raise ValueError("shape mismatch among G, SC, Q, B, info")
+    arr = (ctypes.c_float * nl)(*lam)
+    rc = lib().loca_kspace_solve(_ptr(G), _ptr(SC), _ptr(xsq_total), _ptr(P), _ptr(Q), _ptr(B_prev), arr, nl, L, d,
+                                 k, C, r, _ptr(B), _ptr(info), _ptr(C_out), _stream(stream))
+    _check(rc, "loca_kspace_solve")
 
 
 def batch_step_workspace_size(L) -> int:

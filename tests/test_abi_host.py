@@ -111,6 +111,18 @@ def test_validation_codes(L):
                                       fake, fake, fake, 1 << 20, None) == 2
     assert L.loca_accumulate_streamed(None, fake, fake, 1, 2, 64, 64, 1, fake, ctypes.c_float(0.01), 1, fake,
                                       fake, fake, fake, 1 << 20, None) == 1
+    # k-space path: bf16 only, C and r limits, d % 8
+    assert L.loca_kspace_accumulate(fake, 0, 2, 64, 64, fake, 4, fake, 2, fake, fake, 4, ctypes.c_float(0.01), 1,
+                                    fake, fake, fake, None, fake, 1 << 20, None) == 4
+    assert L.loca_kspace_accumulate(fake, 1, 2, 64, 64, fake, 4, fake, 17, fake, fake, 4, ctypes.c_float(0.01), 1,
+                                    fake, fake, fake, None, fake, 1 << 20, None) == 2
+    assert L.loca_kspace_accumulate(fake, 1, 2, 64, 60, fake, 4, fake, 2, fake, fake, 4, ctypes.c_float(0.01), 1,
+                                    fake, fake, fake, None, fake, 1 << 20, None) == 2
+    lam = (ctypes.c_float * 1)(1e-3)
+    assert L.loca_kspace_solve(fake, fake, None, fake, fake, None, lam, 1, 2, 64, 4, 2, 33, fake, fake, None,
+                               None) == 2
+    rc, n = _ws(L.loca_kspace_workspace_size, 28, 131072, 3584, 16, 4, 16)
+    assert rc == 0 and n >= 28 * 131072 * 16 * 4  # X A_l for every block
     # host memory: freeing NULL is a no-op; a pointer the library did not hand out is rejected
     assert L.loca_host_free(None) == 0
     assert L.loca_host_free(fake) == 1
