@@ -60,6 +60,7 @@ def parse():
     ap.add_argument("--L", type=int, default=None, help="override the workload's block count")
     ap.add_argument("--N", type=int, default=None, help="override the workload's token count")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-kspace", action="store_true", help="skip the k-space statistics measurement")
     ap.add_argument("--e2e-group", type=int, default=2, help="blocks per host-to-device copy in the e2e leg")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -72,6 +73,14 @@ def peaks():
             mp = json.load(f)
         return float(mp["bf16_tflops_sustained"]), "measured"
     return FALLBACK_SUSTAINED_TFLOPS, "fallback"
+
+
+def hbm_peak():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return float(json.load(f)["hbm_gbs"])
+    return 6800.0  # the profiling recipe's fallback copy rate
 
 
 class ClockSampler:
@@ -335,6 +344,58 @@ def main():
                 "frac": achieved / peak, "traffic": traffic, "kernel": "k_gram_cross_tc",
                 "peak_kind": f"bf16 dense sustained, {peak_kind}", "flops_per_launch": flops}
 
+    # the paper's own k-space statistics on the same inputs (no T, no d x d statistics):
+    # error -> k-space accumulate (X A_l on the tensor cores, one HBM read of X) -> k-space solve
+    kspace = None
+    if not args.no_kspace:
+        G_k = torch.empty((L, k, k), **f32)
+        SC_k = torch.empty((L, C, k), **f32)
+        xsq_k = torch.empty((L,), dtype=torch.float64, device=dev)
+        B_k = torch.empty((nl, L, d, k), **f32)
+        info_k = torch.empty((nl, L), dtype=torch.int32, device=dev)
+        ws_k = torch.empty(lc.kspace_workspace_size(L, N, d, k, C, r), dtype=torch.uint8, device=dev)
+
+        def kstep(ev=None):
+            if ev is not None:
+                ev[0].record(stream)
+            lc.loca_error(z, cols, y, E, ce=ce, stream=stream)
+            if ev is not None:
+                ev[1].record(stream)
+            lc.loca_kspace_accumulate(X, A, E, P, Q, w.eta, G_k, SC_k, xsq_k, zero_first=True, workspace=ws_k,
+                                      stream=stream)
+            if ev is not None:
+                ev[2].record(stream)
+            lc.loca_kspace_solve(G_k, SC_k, P, Q, w.lambda_rel, B_k, info_k, xsq_total=xsq_k, stream=stream)
+            if ev is not None:
+                ev[3].record(stream)
+
+        for _ in range(args.warmup):
+            kstep()
+        torch.cuda.synchronize()
+        kev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+        barrier(world)
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for i in range(args.steps):
+            kstep(kev[i])
+        b.record(stream)
+        torch.cuda.synchronize()
+        ms_k = max_over_ranks(world, a.elapsed_time(b)) / args.steps
+        if lc.loca_device_status() != 0 or int(info_k.abs().sum().item()) != 0:
+            raise SystemExit("the k-space steps reported a device error or a non-PD system")
+        kst = {n: statistics.mean(e[i].elapsed_time(e[i + 1]) for e in kev)
+               for i, n in enumerate(["error", "accumulate", "solve"])}
+        xbytes = float(X.numel() * X.element_size())
+        kspace = {"value": world * N * L / (ms_k / 1e3), "unit": UNIT, "ms_per_step": ms_k, "stages_ms": kst,
+                  "launches_per_step": 1 + 4 + 1,
+                  "roofline": {"bound": "hbm", "achieved": xbytes / (kst["accumulate"] / 1e3) / 1e9,
+                               "peak": hbm_peak(), "unit": "GB/s",
+                               "frac": xbytes / (kst["accumulate"] / 1e3) / 1e9 / hbm_peak(),
+                               "traffic": None, "kernel": "loca_kspace_accumulate (prep, X A on tcgen05, stats, final)",
+                               "bytes_per_launch": xbytes}}
+
     # end to end through the public API: host inputs copied in, adapters copied out, per step
     e2e = None
     if not args.no_e2e:
@@ -420,6 +481,7 @@ def main():
             "roofline": roofline,
             "gpu_launches": launches_per_step * args.steps,
             "e2e": e2e,
+            "kspace": kspace,
             "cpu_baseline": cpu,
             "clocks": clk.summary(),
         }

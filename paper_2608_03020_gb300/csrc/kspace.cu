@@ -12,7 +12,7 @@
 //
 // Kernels:
 //   k_kspace_prep   per block: W_l = A_l^T split into bf16 hi / lo rows (2 kp x d, kp = 16 or
-//                   32; A_l ~= hi + lo to 2^-16), and M_l = Q_l Q_l^T (r x r).
+//                   32; A_l ~= hi + lo to 2^-16), and M_l = Q_l Q_l^T (r x r), 8 CTAs per block.
 //   k_kspace_xa     Xp = X_l W_l^T on tcgen05 (kind::f16, M = 128 tokens, N = 2 kp, K = 16, both
 //                   operands K-major with the 128-byte swizzle): a persistent CTA per SM streams
 //                   128-token x 64-channel tiles of X (16 KB) and the matching W tile through an
@@ -41,14 +41,18 @@ using namespace tc;
 
 // ------------------------------------------------------------------ prep
 constexpr int PREP_THREADS = 256;
+constexpr int PREP_SPLIT = 8;  // CTAs per block
 
+// grid (L, PREP_SPLIT): each CTA splits a slice of A_l^T and forms a slice of the r x r entries
+// of Q_l Q_l^T, one warp per entry (lanes over channels; fp32 lane sums, fp64 across lanes).
 __global__ void __launch_bounds__(PREP_THREADS) k_kspace_prep(const float* __restrict__ A, const float* __restrict__ Q,
                                                              int64_t d, int k, int kp, int r,
                                                              __nv_bfloat16* __restrict__ W, float* __restrict__ M) {
-  const int l = blockIdx.x;
+  const int l = blockIdx.x, part = blockIdx.y;
   const float* Al = A + int64_t(l) * d * k;
   __nv_bfloat16* Wl = W + int64_t(l) * 2 * kp * d;
-  for (int64_t e = threadIdx.x; e < int64_t(kp) * d; e += PREP_THREADS) {
+  const int64_t tot = int64_t(kp) * d;
+  for (int64_t e = int64_t(part) * PREP_THREADS + threadIdx.x; e < tot; e += int64_t(PREP_SPLIT) * PREP_THREADS) {
     const int s = int(e / d);
     const int64_t j = e - int64_t(s) * d;
     const float a = (s < k) ? Al[j * k + s] : 0.f;
@@ -57,18 +61,17 @@ __global__ void __launch_bounds__(PREP_THREADS) k_kspace_prep(const float* __res
     Wl[int64_t(s) * d + j] = hi;
     Wl[int64_t(kp + s) * d + j] = lo;
   }
-  // M_l = Q_l Q_l^T: fp32 sums of 64 terms, accumulated in fp64
   const float* Ql = Q + int64_t(l) * r * d;
-  for (int e = threadIdx.x; e < r * r; e += PREP_THREADS) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  constexpr int kWarps = PREP_THREADS / 32;
+  for (int e = part * kWarps + warp; e < r * r; e += PREP_SPLIT * kWarps) {
     const int a = e / r, b = e % r;
-    double acc = 0.0;
-    for (int64_t j0 = 0; j0 < d; j0 += 64) {
-      float part = 0.f;
-      const int64_t j1 = (j0 + 64 < d) ? j0 + 64 : d;
-      for (int64_t j = j0; j < j1; ++j) part = fmaf(Ql[int64_t(a) * d + j], Ql[int64_t(b) * d + j], part);
-      acc += double(part);
-    }
-    M[(int64_t(l) * r + a) * r + b] = float(acc);
+    float acc = 0.f;
+    for (int64_t j = lane; j < d; j += 32) acc = fmaf(Ql[int64_t(a) * d + j], Ql[int64_t(b) * d + j], acc);
+    double v = double(acc);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    if (lane == 0) M[(int64_t(l) * r + a) * r + b] = float(v);
   }
 }
 
@@ -207,14 +210,15 @@ __global__ void __launch_bounds__(XA_THREADS, 1)
         const bool w_ok = mbar_wait(full_bar(stage), phase, wc);
         if (!__all_sync(0xffffffffu, w_ok)) { ok = false; break; }
         // squares of this token's 64 channels: row `row` of the swizzled tile (chunk order is
-        // irrelevant for a sum); zero-filled out-of-range tokens and channels add nothing
+        // irrelevant for a sum, so lane i starts at chunk i % 8 and the 32 lanes' 16-byte reads
+        // spread over all banks); zero-filled out-of-range tokens and channels add nothing
         const uint32_t ra = sbase + uint32_t(stage) * XA_STAGE + uint32_t(row >> 3) * 1024u + uint32_t(row & 7) * 128u;
         float part = 0.f;
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
           uint32_t w0, w1, w2, w3;
           asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(w0), "=r"(w1), "=r"(w2), "=r"(w3)
-                       : "r"(ra + uint32_t(c) * 16u));
+                       : "r"(ra + uint32_t((c + row) & 7) * 16u));
           const uint32_t wv[4] = {w0, w1, w2, w3};
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
@@ -278,7 +282,7 @@ __global__ void __launch_bounds__(ST_THREADS) k_kspace_stats(const float* __rest
                                                            int64_t N, int C, int r, int nch,
                                                            double* __restrict__ part) {
   __shared__ float xs[ST_SUB][KP + 1];
-  __shared__ float es[ST_SUB][kMaxCk];
+  __shared__ float es[ST_SUB][kMaxCk + 1];
   __shared__ float Ms[kMaxRk][kMaxRk + 1];
   __shared__ float Ps[kMaxCk][kMaxRk];
   __shared__ double red[ST_THREADS];
@@ -569,7 +573,7 @@ cudaError_t launch_kspace_accumulate(const void* X, int L, int64_t N, int64_t d,
   const int nch = int((N + ST_CHUNK - 1) / ST_CHUNK);
   cudaError_t e = cudaMemsetAsync(abort_flag, 0, sizeof(int32_t), s);
   if (e != cudaSuccess) return e;
-  k_kspace_prep<<<L, PREP_THREADS, 0, s>>>(A, Q, d, k, kp, r, W, M);
+  k_kspace_prep<<<dim3(unsigned(L), PREP_SPLIT), PREP_THREADS, 0, s>>>(A, Q, d, k, kp, r, W, M);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   CUtensorMap tmX, tmW;
