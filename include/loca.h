@@ -192,8 +192,8 @@ int loca_accumulate_streamed(const void* X_host, void* staging, const void* T, i
  *   X  L x N x d bf16 (LOCA_BF16 only), 16-byte aligned, d % 8 == 0;  A  L x d x k float (k <= 32);
  *   E  N x C float (C <= 16);  P  L x C x r float, Q  L x r x d float (r <= 32);
  *   G  L x k x k float;  SC  L x C x k float;  xsq_total  L double;  alpha  L float or NULL.
- *   Workspace: loca_kspace_workspace_size (holds X A_l, N x kp floats per block, kp = 16 or 32,
- *   and per-tile partial sums).
+ *   Workspace: loca_kspace_workspace_size (the split A_l, Q_l Q_l^T, per-CTA partial sums and
+ *   E^T E partials; 2 KB per 1024 tokens beyond a fixed part).
  *   Arithmetic: X A_l on the tensor cores with A_l split into two bf16 parts (A_l to 2^-16) and
  *   fp32 accumulation; the token sums in fp32 over 128 tokens, fp64 across; fixed-order
  *   reductions (deterministic).

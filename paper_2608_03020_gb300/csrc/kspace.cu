@@ -13,15 +13,21 @@
 // Kernels:
 //   k_kspace_prep   per block: W_l = A_l^T split into bf16 hi / lo rows (2 kp x d, kp = 16 or
 //                   32; A_l ~= hi + lo to 2^-16), and M_l = Q_l Q_l^T (r x r), 8 CTAs per block.
-//   k_kspace_xa     Xp = X_l W_l^T on tcgen05 (kind::f16, M = 128 tokens, N = 2 kp, K = 16, both
+//   k_kspace_xa     p = W_l x_n on tcgen05 (kind::f16, M = 128 tokens, N = 2 kp, K = 16, both
 //                   operands K-major with the 128-byte swizzle): a persistent CTA per SM streams
 //                   128-token x 64-channel tiles of X (16 KB) and the matching W tile through an
-//                   8-stage TMA ring; the epilogue warps also sum the squares of every X tile
-//                   from shared memory, and write p = hi-part + lo-part (fp32) per token.
-//   k_kspace_stats  token-parallel partials of Xp^T Xp, E^T Xp and sum u^T M u (fp32 over 128
-//                   tokens, fp64 across).
-//   k_kspace_final  fixed-order reduction of all partials per block (deterministic), alpha_l,
-//                   and the update of G, S, xsq_total.
+//                   8-stage TMA ring.  Per tile, four epilogue warps take p = hi part + lo part
+//                   from TMEM (one token per thread) and add the tile's sums over their 32 tokens
+//                   (p p^T upper triangle, e p^T; fp32) to per-lane registers; each CTA's run of
+//                   tiles of a block ends in
+//                   one write of its (block, CTA, warp) fp64 partial slot.  Two further warps sum
+//                   the squares of every X tile and, with the MMA commit, release the stages, so
+//                   the statistics never hold up the ring.  Nothing but X is read from HBM in
+//                   bulk, and no warp waits for another outside the mbarrier pipeline.
+//   k_kspace_ete    E^T E of the batch (C x C), shared by every block: ||T_l||^2 =
+//                   <P_l (Q_l Q_l^T) P_l^T, E^T E>, so no per-token work is needed for it.
+//   k_kspace_final  fixed-order reduction of the partial slots per block (deterministic),
+//                   ||T_l||^2, alpha_l, and the update of G, S, xsq_total.
 //   k_kspace_solve  lambda from the trace, Cholesky of G_l + lambda I, C_l rows from Q_l^T (P_l^T
 //                   S_l) (+ B_prev,l G_l), forward and back substitution per row.
 // Every mbarrier wait is bounded (see tc_ptx.cuh).
@@ -76,20 +82,28 @@ __global__ void __launch_bounds__(PREP_THREADS) k_kspace_prep(const float* __res
 }
 
 // ------------------------------------------------------------------ X A on the tensor cores
-constexpr int XA_THREADS = 192;
+constexpr int XA_THREADS = 256;  // producer, MMA, 4 TMEM / statistics warps, 2 sum-of-squares warps
 constexpr int XA_TM = 128;          // tokens per tile (TMEM lanes)
 constexpr int XA_BK = 64;           // channels per stage (one 128-byte swizzle row)
 constexpr int XA_STAGES = 8;
 constexpr int XA_XBYTES = XA_TM * XA_BK * 2;  // 16 KB
 constexpr int XA_STAGE = 24 * 1024;           // X tile + up to 64 W rows (8 KB)
-constexpr int XA_SMEM = XA_STAGES * XA_STAGE + 1024 + 256;
 constexpr uint32_t XA_TMEM_COLS = 128;
+constexpr int XA_MAX_GRID = 256;   // partial slots per block are sized for at most this many CTAs
+constexpr int kMaxCk = 16;         // C limit of the k-space path
+constexpr int kMaxRk = 32;         // r limit
+constexpr int XA_EPI_SMEM = 4 * 32 * ((32 + 1) + (kMaxCk + 1)) * 4;  // per-warp p and e staging
+
+// partial slot: upper triangle of p p^T (kp (kp + 1) / 2), e p^T (C x kp), ||x||^2
+__host__ __device__ constexpr int ntri(int kp) { return kp * (kp + 1) / 2; }
+__host__ __device__ constexpr int part_stride(int kp, int C) { return ntri(kp) + C * kp + 1; }
+constexpr int XA_SMEM = XA_STAGES * XA_STAGE + 1024 + 256 + XA_EPI_SMEM;
 
 template <int KP>
 __global__ void __launch_bounds__(XA_THREADS, 1)
     k_kspace_xa(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW, int L,
-                int64_t N, int64_t d, int ntiles, float* __restrict__ Xp, double* __restrict__ xsq_part,
-                int32_t* status, int32_t* abort_flag, unsigned long long limit_ns) {
+                int64_t N, int64_t d, int ntiles, const float* __restrict__ E, int C,
+                double* __restrict__ part, int32_t* status, int32_t* abort_flag, unsigned long long limit_ns) {
   constexpr int NCOL = 2 * KP;
   constexpr uint32_t WBYTES = uint32_t(NCOL) * 128u;
   constexpr uint32_t ID = tc::idesc(1, 1, 0, 0, XA_TM, NCOL);
@@ -97,6 +111,7 @@ __global__ void __launch_bounds__(XA_THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + XA_STAGES * XA_STAGE);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * XA_STAGES + 6);
+  float* epi = reinterpret_cast<float*>(smem + XA_STAGES * XA_STAGE + 256);
   const uint32_t sbase = smem_u32(smem);
   const uint32_t bar0 = smem_u32(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
@@ -110,7 +125,7 @@ __global__ void __launch_bounds__(XA_THREADS, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < XA_STAGES; ++s) {
       mbar_init(full_bar(s), 1);
-      mbar_init(empty_bar(s), 5);  // the MMA commit and lane 0 of the four epilogue warps
+      mbar_init(empty_bar(s), 3);  // the MMA commit and lane 0 of the two sum-of-squares warps
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(acc_full(b), 1);
@@ -194,45 +209,115 @@ __global__ void __launch_bounds__(XA_THREADS, 1)
       }
     }
     __syncwarp();
-  } else {
-    // epilogue warps 2..5: TMEM lane quarter q; token row = q * 32 + lane of each tile
-    const int q = warp & 3;
-    const int row = q * 32 + lane;
+  } else if (warp >= 6) {
+    // sum-of-squares warps 6, 7: tokens (warp - 6) * 64 + lane and + 32 of every stage; they alone
+    // (with the MMA commit) release the stages, so the statistics below never hold up the ring
+    const int w2 = warp - 6;
+    const int PS = part_stride(KP, C);
+    const int64_t nslot = int64_t(gridDim.x) * 4;
+    const int xe = ntri(KP) + C * KP;  // the ||x||^2 entry of slots (CTA, w2)
+    double xs = 0.0;
+    int cur_l = -1;
+    auto flush = [&](int lf) {
+      double a = xs;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) a += __shfl_xor_sync(0xffffffffu, a, off);
+      if (lane == 0) part[(int64_t(lf) * PS + xe) * nslot + int64_t(blockIdx.x) * 4 + w2] = a;
+    };
     int stage = 0;
-    uint32_t phase = 0, tcount = 0;
-    for (int it = blockIdx.x; it < total; it += gridDim.x, ++tcount) {
+    uint32_t phase = 0;
+    for (int it = blockIdx.x; it < total; it += gridDim.x) {
       const int l = it / ntiles;
-      const int tile = it - l * ntiles;
-      const int t0 = tile * XA_TM;
-      double xs = 0.0;
+      if (l != cur_l) {
+        if (cur_l >= 0) flush(cur_l);
+        cur_l = l;
+        xs = 0.0;
+      }
       bool ok = true;
       for (int kc = 0; kc < nkc; ++kc) {
         const bool w_ok = mbar_wait(full_bar(stage), phase, wc);
         if (!__all_sync(0xffffffffu, w_ok)) { ok = false; break; }
-        // squares of this token's 64 channels: row `row` of the swizzled tile (chunk order is
-        // irrelevant for a sum, so lane i starts at chunk i % 8 and the 32 lanes' 16-byte reads
-        // spread over all banks); zero-filled out-of-range tokens and channels add nothing
-        const uint32_t ra = sbase + uint32_t(stage) * XA_STAGE + uint32_t(row >> 3) * 1024u + uint32_t(row & 7) * 128u;
-        float part = 0.f;
+        // squares of the tokens' 64 channels: rows of the swizzled tile (chunk order is irrelevant
+        // for a sum, so lane i starts at chunk i % 8 and the 32 lanes' 16-byte reads spread over
+        // all banks); zero-filled out-of-range tokens and channels add nothing
+        float pa[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // independent chains
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          uint32_t w0, w1, w2, w3;
-          asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(w0), "=r"(w1), "=r"(w2), "=r"(w3)
-                       : "r"(ra + uint32_t((c + row) & 7) * 16u));
-          const uint32_t wv[4] = {w0, w1, w2, w3};
+        for (int h = 0; h < 2; ++h) {
+          const int row = w2 * 64 + h * 32 + lane;
+          const uint32_t ra = sbase + uint32_t(stage) * XA_STAGE + uint32_t(row) * 128u;
 #pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const float lo = __uint_as_float(wv[u] << 16), hi = __uint_as_float(wv[u] & 0xffff0000u);
-            part = fmaf(lo, lo, part);
-            part = fmaf(hi, hi, part);
+          for (int c = 0; c < 8; ++c) {
+            uint32_t w0, w1, w3, w4;
+            asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(w0), "=r"(w1), "=r"(w3), "=r"(w4)
+                         : "r"(ra + uint32_t((c + row) & 7) * 16u));
+            const uint32_t wv[4] = {w0, w1, w3, w4};
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const float lo = __uint_as_float(wv[u] << 16), hi = __uint_as_float(wv[u] & 0xffff0000u);
+              pa[2 * u] = fmaf(lo, lo, pa[2 * u]);
+              pa[2 * u + 1] = fmaf(hi, hi, pa[2 * u + 1]);
+            }
           }
         }
-        xs += double(part);
+        xs += double(((pa[0] + pa[1]) + (pa[2] + pa[3])) + ((pa[4] + pa[5]) + (pa[6] + pa[7])));
         __syncwarp();
         if (lane == 0) mbar_arrive(empty_bar(stage));
         if (++stage == XA_STAGES) { stage = 0; phase ^= 1u; }
       }
       if (!ok) break;
+    }
+    if (cur_l >= 0) flush(cur_l);  // warp-uniform
+  } else {
+    // epilogue warps 2..5: TMEM lane quarter q; token row = q * 32 + lane of each tile
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    constexpr int PSTR = KP + 1, ESTR = kMaxCk + 1;
+    constexpr int NTRI = ntri(KP);
+    constexpr int NG = (NTRI + 31) / 32;
+    const int PS = part_stride(KP, C);
+    float* ps = epi + (warp - 2) * 32 * (33 + ESTR);
+    float* es = ps + 32 * 33;
+    // upper-triangle entries owned by this lane: eidx = lane + 32 i -> (a, b), a <= b
+    int pair[NG];
+#pragma unroll
+    for (int i2 = 0; i2 < NG; ++i2) {
+      int rem = lane + 32 * i2, a = 0;
+      while (a < KP && rem >= KP - a) {
+        rem -= KP - a;
+        ++a;
+      }
+      pair[i2] = (a << 8) | (a + rem);
+    }
+    constexpr int NSM = (kMaxCk * KP + 31) / 32;
+    const int NS = C * KP;
+    // this lane's sums for the current block (fp32 within one CTA's run of tiles of a block; the
+    // runs are written once, as fp64, when the block changes, and reduced in a fixed order later)
+    float accg[NG], accs[NSM];
+    int cur_l = -1;
+    const int64_t nslot = int64_t(gridDim.x) * 4;
+    auto flush = [&](int lf) {
+      // entry-major: entry e of block lf at part[(lf * PS + e) * nslot + this slot]
+      double* slot = part + int64_t(lf) * PS * nslot + int64_t(blockIdx.x) * 4 + q;
+#pragma unroll
+      for (int i2 = 0; i2 < NG; ++i2)
+        if (lane + 32 * i2 < NTRI) slot[int64_t(lane + 32 * i2) * nslot] = double(accg[i2]);
+#pragma unroll
+      for (int i2 = 0; i2 < NSM; ++i2)
+        if (lane + 32 * i2 < NS) slot[int64_t(NTRI + lane + 32 * i2) * nslot] = double(accs[i2]);
+    };
+    uint32_t tcount = 0;
+    for (int it = blockIdx.x; it < total; it += gridDim.x, ++tcount) {
+      const int l = it / ntiles;
+      const int tile = it - l * ntiles;
+      const int t0 = tile * XA_TM;
+      if (l != cur_l) {
+        if (cur_l >= 0) flush(cur_l);
+        cur_l = l;
+#pragma unroll
+        for (int i2 = 0; i2 < NG; ++i2) accg[i2] = 0.f;
+#pragma unroll
+        for (int i2 = 0; i2 < NSM; ++i2) accs[i2] = 0.f;
+      }
       const int buf = int(tcount & 1u);
       const bool a_ok = mbar_wait(acc_full(buf), (tcount >> 1) & 1u, wc);
       if (!__all_sync(0xffffffffu, a_ok)) break;
@@ -247,18 +332,40 @@ __global__ void __launch_bounds__(XA_THREADS, 1)
       fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(acc_empty(buf));
+      // stage this warp's 32 tokens: p (kp) and e (C); tokens beyond N contribute zeros
       const int64_t n = int64_t(t0) + row;
-      if (n < N) {
-        float4* o = reinterpret_cast<float4*>(Xp + (int64_t(l) * N + n) * KP);
+      const bool nv = n < N;
 #pragma unroll
-        for (int u = 0; u < KP / 4; ++u)
-          o[u] = make_float4(v[4 * u] + v[KP + 4 * u], v[4 * u + 1] + v[KP + 4 * u + 1],
-                             v[4 * u + 2] + v[KP + 4 * u + 2], v[4 * u + 3] + v[KP + 4 * u + 3]);
+      for (int s2 = 0; s2 < KP; ++s2) ps[lane * PSTR + s2] = v[s2] + v[KP + s2];
+#pragma unroll
+      for (int c = 0; c < kMaxCk; ++c)
+        if (c < C) es[lane * ESTR + c] = nv ? E[n * C + c] : 0.f;
+      __syncwarp();
+      // the tile's sums over this warp's 32 tokens, for the entries this lane owns
+#pragma unroll
+      for (int i2 = 0; i2 < NG; ++i2) {
+        if (lane + 32 * i2 < NTRI) {
+          const int a = pair[i2] >> 8, b = pair[i2] & 0xff;
+          float acc = 0.f;
+#pragma unroll 8
+          for (int t = 0; t < 32; ++t) acc = fmaf(ps[t * PSTR + a], ps[t * PSTR + b], acc);
+          accg[i2] += acc;
+        }
       }
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) xs += __shfl_xor_sync(0xffffffffu, xs, off);
-      if (lane == 0) xsq_part[(int64_t(l) * ntiles + tile) * 4 + q] = xs;
+      for (int i2 = 0; i2 < NSM; ++i2) {
+        const int eidx = lane + 32 * i2;
+        if (eidx < NS) {
+          const int c = eidx / KP, s2 = eidx - c * KP;
+          float acc = 0.f;
+#pragma unroll 8
+          for (int t = 0; t < 32; ++t) acc = fmaf(es[t * ESTR + c], ps[t * PSTR + s2], acc);
+          accs[i2] += acc;
+        }
+      }
+      __syncwarp();  // the staging rows are rewritten by the next tile
     }
+    if (cur_l >= 0) flush(cur_l);  // warp-uniform: every lane reaches here together
   }
 
   fence_before();
@@ -267,161 +374,135 @@ __global__ void __launch_bounds__(XA_THREADS, 1)
   if (warp == 1) tmem_dealloc(tmem_base, XA_TMEM_COLS);
 }
 
-// ------------------------------------------------------------------ token-parallel partials
-constexpr int ST_THREADS = 256;
-constexpr int ST_SUB = 128;    // tokens staged in shared memory at a time
-constexpr int ST_CHUNK = 4096; // tokens per CTA
-constexpr int kMaxCk = 16;     // C limit of the k-space path
-constexpr int kMaxRk = 32;     // r limit
+// ------------------------------------------------------------------ E^T E
+// ||T_l||^2 = sum_n u_n^T (Q_l Q_l^T) u_n = <P_l (Q_l Q_l^T) P_l^T, E^T E>: the C x C matrix E^T E
+// of the batch serves every block.  Partials per chunk of tokens (fp32 over 256 tokens, fp64
+// across), reduced in a fixed order by k_kspace_final.
+constexpr int ETE_THREADS = 256;
+constexpr int ETE_SUB = 256;
+constexpr int ETE_CHUNK = 1024;
 
-__host__ __device__ constexpr int part_stride(int kp, int C) { return kp * kp + C * kp + 1; }
-
-template <int KP>
-__global__ void __launch_bounds__(ST_THREADS) k_kspace_stats(const float* __restrict__ Xp, const float* __restrict__ E,
-                                                           const float* __restrict__ P, const float* __restrict__ M,
-                                                           int64_t N, int C, int r, int nch,
-                                                           double* __restrict__ part) {
-  __shared__ float xs[ST_SUB][KP + 1];
-  __shared__ float es[ST_SUB][kMaxCk + 1];
-  __shared__ float Ms[kMaxRk][kMaxRk + 1];
-  __shared__ float Ps[kMaxCk][kMaxRk];
-  __shared__ double red[ST_THREADS];
-  const int ch = blockIdx.x, l = blockIdx.y;
-  const int tid = threadIdx.x;
-  for (int e = tid; e < r * r; e += ST_THREADS) Ms[e / r][e % r] = M[int64_t(l) * r * r + e];
-  for (int e = tid; e < C * r; e += ST_THREADS) Ps[e / r][e % r] = P[int64_t(l) * C * r + e];
-  constexpr int GPT = (KP * KP + ST_THREADS - 1) / ST_THREADS;
-  const int SPT = (C * KP + ST_THREADS - 1) / ST_THREADS;  // <= 2 (C <= 16, KP <= 32)
-  double g[GPT], sacc[2];
-#pragma unroll
-  for (int i = 0; i < GPT; ++i) g[i] = 0.0;
-  sacc[0] = sacc[1] = 0.0;
-  double tq = 0.0;
-  const int64_t n_beg = int64_t(ch) * ST_CHUNK;
-  const int64_t n_end = (n_beg + ST_CHUNK < N) ? n_beg + ST_CHUNK : N;
-  const float* Xl = Xp + int64_t(l) * N * KP;
-  for (int64_t s0 = n_beg; s0 < n_end; s0 += ST_SUB) {
+__global__ void __launch_bounds__(ETE_THREADS) k_kspace_ete(const float* __restrict__ E, int64_t N, int C,
+                                                          double* __restrict__ ete_part) {
+  __shared__ float es[ETE_SUB][kMaxCk + 1];
+  const int ch = blockIdx.x, tid = threadIdx.x;
+  const int a = tid / kMaxCk, b = tid % kMaxCk;
+  const int64_t n0 = int64_t(ch) * ETE_CHUNK;
+  const int64_t n1 = (n0 + ETE_CHUNK < N) ? n0 + ETE_CHUNK : N;
+  double acc = 0.0;
+  for (int64_t s0 = n0; s0 < n1; s0 += ETE_SUB) {
     __syncthreads();
-    for (int e = tid; e < ST_SUB * KP; e += ST_THREADS) {
-      const int t = e / KP, s = e % KP;
-      xs[t][s] = (s0 + t < n_end) ? Xl[(s0 + t) * KP + s] : 0.f;
-    }
-    for (int e = tid; e < ST_SUB * C; e += ST_THREADS) {
+    for (int e = tid; e < ETE_SUB * C; e += ETE_THREADS) {
       const int t = e / C, c = e % C;
-      es[t][c] = (s0 + t < n_end) ? E[(s0 + t) * C + c] : 0.f;
+      es[t][c] = (s0 + t < n1) ? E[(s0 + t) * C + c] : 0.f;
     }
     __syncthreads();
-#pragma unroll
-    for (int i = 0; i < GPT; ++i) {
-      const int e = tid + i * ST_THREADS;
-      if (e < KP * KP) {
-        const int a = e / KP, b = e % KP;
-        float acc = 0.f;
+    if (a < C && b < C) {
+      float part = 0.f;
 #pragma unroll 8
-        for (int t = 0; t < ST_SUB; ++t) acc = fmaf(xs[t][a], xs[t][b], acc);
-        g[i] += double(acc);
-      }
-    }
-    for (int i = 0; i < SPT; ++i) {
-      const int e = tid + i * ST_THREADS;
-      if (e < C * KP) {
-        const int c = e / KP, s = e % KP;
-        float acc = 0.f;
-#pragma unroll 8
-        for (int t = 0; t < ST_SUB; ++t) acc = fmaf(es[t][c], xs[t][s], acc);
-        sacc[i] += double(acc);
-      }
-    }
-    if (tid < ST_SUB) {
-      // ||t_n||^2 = u^T (Q Q^T) u with u = e_n P_l
-      float u[kMaxRk];
-#pragma unroll
-      for (int a = 0; a < kMaxRk; ++a) {
-        float acc = 0.f;
-        if (a < r)
-          for (int c = 0; c < C; ++c) acc = fmaf(es[tid][c], Ps[c][a], acc);
-        u[a] = acc;
-      }
-      float qq = 0.f;
-#pragma unroll
-      for (int a = 0; a < kMaxRk; ++a) {
-        if (a >= r) break;
-        float mu = 0.f;
-#pragma unroll
-        for (int b = 0; b < kMaxRk; ++b)
-          if (b < r) mu = fmaf(Ms[a][b], u[b], mu);
-        qq = fmaf(u[a], mu, qq);
-      }
-      tq += double(qq);
+      for (int t = 0; t < ETE_SUB; ++t) part = fmaf(es[t][a], es[t][b], part);
+      acc += double(part);
     }
   }
-  const int ps = part_stride(KP, C);
-  double* out = part + (int64_t(l) * nch + ch) * ps;
-#pragma unroll
-  for (int i = 0; i < GPT; ++i) {
-    const int e = tid + i * ST_THREADS;
-    if (e < KP * KP) out[e] = g[i];
-  }
-  for (int i = 0; i < SPT; ++i) {
-    const int e = tid + i * ST_THREADS;
-    if (e < C * KP) out[KP * KP + e] = sacc[i];
-  }
-  red[tid] = tq;
-  __syncthreads();
-  for (int w = ST_THREADS / 2; w > 0; w >>= 1) {
-    if (tid < w) red[tid] += red[tid + w];
-    __syncthreads();
-  }
-  if (tid == 0) out[ps - 1] = red[0];
+  if (a < C && b < C) ete_part[int64_t(ch) * kMaxCk * kMaxCk + a * kMaxCk + b] = acc;
 }
 
 // ------------------------------------------------------------------ per-block final reduction
 constexpr int FI_THREADS = 256;
+constexpr int FI_SPLIT = 4;  // CTAs per block (entries e with e % FI_SPLIT == part)
 
+// Sums the (CTA, warp) partial slots of block l in a fixed order (a CTA without tiles of block l,
+// possible only when blocks have fewer tiles than there are CTAs, never wrote its slot), forms
+// ||T_l||^2 = <P_l M_l P_l^T, E^T E>, the step alpha_l, and updates G, SC, xsq_total.
 __global__ void __launch_bounds__(FI_THREADS) k_kspace_final(const double* __restrict__ part,
-                                                           const double* __restrict__ xsq_part, int nch,
-                                                           int ntiles, int kp, int k, int C, float eta,
-                                                           int zero_first, float* __restrict__ G,
+                                                           const double* __restrict__ ete_part, int nch_e,
+                                                           const float* __restrict__ P, const float* __restrict__ M,
+                                                           int grid, int ntiles, int kp, int k, int C, int r,
+                                                           float eta, int zero_first, float* __restrict__ G,
                                                            float* __restrict__ SC, double* __restrict__ xsq_total,
                                                            float* __restrict__ alpha_out) {
+  __shared__ unsigned char has[XA_MAX_GRID];
+  __shared__ double ete[kMaxCk][kMaxCk];
+  __shared__ double pm[kMaxCk][kMaxRk];  // P_l M_l
   __shared__ double red[FI_THREADS];
-  __shared__ double s_xsq, s_tsq;
-  const int l = blockIdx.x, tid = threadIdx.x;
+  __shared__ double s_xsq;
+  const int l = blockIdx.x, prt = blockIdx.y, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int ps = part_stride(kp, C);
-  const double* pl = part + int64_t(l) * nch * ps;
-  // xsq of this batch: per-thread strided sums in a fixed order, then a fixed tree
-  double a = 0.0;
-  for (int64_t i = tid; i < int64_t(ntiles) * 4; i += FI_THREADS) a += xsq_part[int64_t(l) * ntiles * 4 + i];
-  red[tid] = a;
+  const int64_t lo = int64_t(l) * ntiles, hi = lo + ntiles;
+  for (int c = tid; c < grid; c += FI_THREADS) has[c] = (lo + ((int64_t(c) - lo) % grid + grid) % grid) < hi;
+  for (int e = tid; e < C * C; e += FI_THREADS) {
+    const int a = e / C, b = e % C;
+    double v = 0.0;
+    for (int ch = 0; ch < nch_e; ++ch) v += ete_part[int64_t(ch) * kMaxCk * kMaxCk + a * kMaxCk + b];
+    ete[a][b] = v;
+  }
+  const float* Pl = P + int64_t(l) * C * r;
+  const float* Ml = M + int64_t(l) * r * r;
+  for (int e = tid; e < C * r; e += FI_THREADS) {
+    const int c = e / r, b = e % r;
+    double v = 0.0;
+    for (int a = 0; a < r; ++a) v += double(Pl[c * r + a]) * double(Ml[a * r + b]);
+    pm[c][b] = v;
+  }
+  __syncthreads();
+  const int nslot = grid * 4;
+  // one warp; lanes over slots in order, then a fixed butterfly.  The ||x||^2 entry is written
+  // by the two sum-of-squares warps only (slots 0 and 1 of each CTA).
+  auto sum_entry = [&](int e, int nq) {
+    const double* pe = part + (int64_t(l) * ps + e) * nslot;
+    double v = 0.0;
+    for (int sidx = lane; sidx < nslot; sidx += 32)
+      if (has[sidx >> 2] && (sidx & 3) < nq) v += pe[sidx];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    return v;
+  };
+  const int nt = ntri(kp);
+  if (warp == 0) {
+    const double v = sum_entry(nt + C * kp, 2);
+    if (lane == 0) s_xsq = v;
+  }
+  // ||T_l||^2 = sum_{c, c'} (P M P^T)[c][c'] (E^T E)[c][c']
+  double t = 0.0;
+  for (int e = tid; e < C * C; e += FI_THREADS) {
+    const int a = e / C, b = e % C;
+    double kab = 0.0;
+    for (int j = 0; j < r; ++j) kab += pm[a][j] * double(Pl[b * r + j]);
+    t += kab * ete[a][b];
+  }
+  red[tid] = t;
   __syncthreads();
   for (int w = FI_THREADS / 2; w > 0; w >>= 1) {
     if (tid < w) red[tid] += red[tid + w];
     __syncthreads();
   }
-  if (tid == 0) {
-    s_xsq = red[0];
-    double t = 0.0;
-    for (int c = 0; c < nch; ++c) t += pl[int64_t(c) * ps + ps - 1];
-    s_tsq = t;
-  }
-  __syncthreads();
-  const double xsq_b = s_xsq, tsq_b = s_tsq;
+  const double xsq_b = s_xsq, tsq_b = red[0];
   const double al = tsq_b > 0.0 ? -double(eta) * sqrt(xsq_b / tsq_b) : 0.0;
-  for (int e = tid; e < k * k; e += FI_THREADS) {
-    const int r0 = e / k, c0 = e % k;
-    double v = 0.0;
-    for (int c = 0; c < nch; ++c) v += pl[int64_t(c) * ps + r0 * kp + c0];
-    float* o = G + int64_t(l) * k * k + e;
-    *o = zero_first ? float(v) : float(double(*o) + v);
+  // G entries (symmetric, from the upper triangle) and SC entries of this CTA's share
+  for (int e = prt * (FI_THREADS / 32) + warp; e < k * k + C * k; e += FI_SPLIT * (FI_THREADS / 32)) {
+    if (e < k * k) {
+      int a = e / k, b = e % k;
+      if (a > b) {
+        const int tmp = a;
+        a = b;
+        b = tmp;
+      }
+      const double v = sum_entry(a * kp - a * (a - 1) / 2 + (b - a), 4);  // row a of the upper triangle
+      if (lane == 0) {
+        float* o = G + int64_t(l) * k * k + e;
+        *o = zero_first ? float(v) : float(double(*o) + v);
+      }
+    } else {
+      const int e2 = e - k * k;
+      const int cc = e2 / k, s2 = e2 % k;
+      const double v = sum_entry(nt + cc * kp + s2, 4);
+      if (lane == 0) {
+        float* o = SC + int64_t(l) * C * k + e2;
+        *o = zero_first ? float(al * v) : float(double(*o) + al * v);
+      }
+    }
   }
-  for (int e = tid; e < C * k; e += FI_THREADS) {
-    const int cc = e / k, s = e % k;
-    double v = 0.0;
-    for (int c = 0; c < nch; ++c) v += pl[int64_t(c) * ps + kp * kp + cc * kp + s];
-    float* o = SC + int64_t(l) * C * k + e;
-    *o = zero_first ? float(al * v) : float(double(*o) + al * v);
-  }
-  if (tid == 0) {
+  if (prt == 0 && tid == 0) {
     xsq_total[l] = zero_first ? xsq_b : xsq_total[l] + xsq_b;
     if (alpha_out) alpha_out[l] = float(al);
   }
@@ -534,19 +615,15 @@ int kp_for(int k) { return k <= 16 ? 16 : 32; }
 KspaceWs kspace_ws(int L, int64_t N, int64_t d, int k, int C, int r) {
   KspaceWs w{};
   const int kp = kp_for(k);
-  const int64_t ntiles = (N + XA_TM - 1) / XA_TM;
-  const int64_t nch = (N + ST_CHUNK - 1) / ST_CHUNK;
   size_t off = 0;
   w.W = off;
   off += align256(sizeof(__nv_bfloat16) * size_t(L) * 2 * kp * size_t(d));
   w.M = off;
   off += align256(sizeof(float) * size_t(L) * r * r);
-  w.Xp = off;
-  off += align256(sizeof(float) * size_t(L) * size_t(N) * kp);
-  w.xsq_part = off;
-  off += align256(sizeof(double) * size_t(L) * size_t(ntiles) * 4);
   w.part = off;
-  off += align256(sizeof(double) * size_t(L) * size_t(nch) * part_stride(kp, C));
+  off += align256(sizeof(double) * size_t(L) * XA_MAX_GRID * 4 * part_stride(kp, C));
+  w.ete = off;
+  off += align256(sizeof(double) * size_t((N + ETE_CHUNK - 1) / ETE_CHUNK) * kMaxCk * kMaxCk);
   w.flags = off;
   off += 256;
   w.total = off;
@@ -564,13 +641,11 @@ cudaError_t launch_kspace_accumulate(const void* X, int L, int64_t N, int64_t d,
   char* ws = static_cast<char*>(workspace);
   __nv_bfloat16* W = reinterpret_cast<__nv_bfloat16*>(ws + lay.W);
   float* M = reinterpret_cast<float*>(ws + lay.M);
-  float* Xp = reinterpret_cast<float*>(ws + lay.Xp);
-  double* xsq_part = reinterpret_cast<double*>(ws + lay.xsq_part);
   double* part = reinterpret_cast<double*>(ws + lay.part);
+  double* ete = reinterpret_cast<double*>(ws + lay.ete);
   int32_t* abort_flag = reinterpret_cast<int32_t*>(ws + lay.flags);
   const int kp = kp_for(k);
   const int ntiles = int((N + XA_TM - 1) / XA_TM);
-  const int nch = int((N + ST_CHUNK - 1) / ST_CHUNK);
   cudaError_t e = cudaMemsetAsync(abort_flag, 0, sizeof(int32_t), s);
   if (e != cudaSuccess) return e;
   k_kspace_prep<<<dim3(unsigned(L), PREP_SPLIT), PREP_THREADS, 0, s>>>(A, Q, d, k, kp, r, W, M);
@@ -581,27 +656,28 @@ cudaError_t launch_kspace_accumulate(const void* X, int L, int64_t N, int64_t d,
       !make_map3(&tmW, W, uint64_t(d), uint64_t(2 * kp), uint64_t(L), uint32_t(2 * kp)))
     return cudaErrorInvalidValue;
   int grid = sm_count();
+  if (grid > XA_MAX_GRID) grid = XA_MAX_GRID;
   if (grid > L * ntiles) grid = L * ntiles;
   const unsigned long long limit = 4000000000ull;
   if (kp == 16) {
     e = cudaFuncSetAttribute(k_kspace_xa<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, XA_SMEM);
     if (e != cudaSuccess) return e;
-    k_kspace_xa<16><<<grid, XA_THREADS, XA_SMEM, s>>>(tmX, tmW, L, N, d, ntiles, Xp, xsq_part, status, abort_flag, limit);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    k_kspace_stats<16><<<dim3(unsigned(nch), unsigned(L)), ST_THREADS, 0, s>>>(Xp, E, P, M, N, C, r, nch, part);
+    k_kspace_xa<16><<<grid, XA_THREADS, XA_SMEM, s>>>(tmX, tmW, L, N, d, ntiles, E, C, part, status, abort_flag,
+                                                      limit);
   } else {
     e = cudaFuncSetAttribute(k_kspace_xa<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, XA_SMEM);
     if (e != cudaSuccess) return e;
-    k_kspace_xa<32><<<grid, XA_THREADS, XA_SMEM, s>>>(tmX, tmW, L, N, d, ntiles, Xp, xsq_part, status, abort_flag, limit);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    k_kspace_stats<32><<<dim3(unsigned(nch), unsigned(L)), ST_THREADS, 0, s>>>(Xp, E, P, M, N, C, r, nch, part);
+    k_kspace_xa<32><<<grid, XA_THREADS, XA_SMEM, s>>>(tmX, tmW, L, N, d, ntiles, E, C, part, status, abort_flag,
+                                                      limit);
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  k_kspace_final<<<L, FI_THREADS, 0, s>>>(part, xsq_part, nch, ntiles, kp, k, C, eta, zero_first, G, SC, xsq_total,
-                                          alpha_out);
+  const int nch_e = int((N + ETE_CHUNK - 1) / ETE_CHUNK);
+  k_kspace_ete<<<nch_e, ETE_THREADS, 0, s>>>(E, N, C, ete);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_kspace_final<<<dim3(unsigned(L), FI_SPLIT), FI_THREADS, 0, s>>>(part, ete, nch_e, P, M, grid, ntiles, kp, k, C,
+                                                                     r, eta, zero_first, G, SC, xsq_total, alpha_out);
   return cudaGetLastError();
 }
 

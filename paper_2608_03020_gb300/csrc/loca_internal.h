@@ -64,7 +64,7 @@ cudaError_t launch_gram_cross_tc(const void* X, const void* T, int L, int64_t N,
 
 // ---- k-space statistics and solve (kspace.cu)
 struct KspaceWs {
-  size_t W, M, Xp, xsq_part, part, flags, total;
+  size_t W, M, part, ete, flags, total;
 };
 KspaceWs kspace_ws(int L, int64_t N, int64_t d, int k, int C, int r);
 int kspace_max_C();
