@@ -61,6 +61,7 @@ def parse():
     ap.add_argument("--N", type=int, default=None, help="override the workload's token count")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-kspace", action="store_true", help="skip the k-space statistics measurement")
+    ap.add_argument("--no-vocab", action="store_true", help="skip the wide-vocabulary head-error measurement")
     ap.add_argument("--e2e-group", type=int, default=2, help="blocks per host-to-device copy in the e2e leg")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -396,6 +397,44 @@ def main():
                                "traffic": None, "kernel": "loca_kspace_accumulate (prep, X A on tcgen05, stats, final)",
                                "bytes_per_launch": xbytes}}
 
+    # the head error where it is HBM-bound: the Qwen2.5-14B row of the workloads (N = 131072 tokens,
+    # V = 151936 bf16 logits, C = 4 label columns; 39.8 GB of logits, drawn as in synth)
+    vocab = None
+    if not args.no_vocab and world == 1:
+        wv = S.WORKLOADS["qwen2.5-14b"]
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(1234)
+        zv = torch.empty((wv.N, wv.V), dtype=torch.bfloat16, device=dev)
+        fv = S.host_factors(wv, 0)
+        cols_v = torch.from_numpy(fv["label_cols"].astype(np.int32)).to(dev)
+        y_v = torch.from_numpy(fv["y"].astype(np.int32)).to(dev)
+        off = float(np.log(wv.V / wv.C))
+        for n0 in range(0, wv.N, 8192):
+            g = torch.randn((min(8192, wv.N - n0), wv.V), generator=gen, device=dev)
+            g[:, cols_v.long()] += off
+            zv[n0:n0 + g.shape[0]] = g.to(torch.bfloat16)
+            del g
+        Ev = torch.empty((wv.N, wv.C), **f32)
+        cev = torch.empty((wv.N,), **f32)
+        for _ in range(args.warmup):
+            lc.loca_error(zv, cols_v, y_v, Ev, ce=cev, stream=stream)
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(args.steps):
+            lc.loca_error(zv, cols_v, y_v, Ev, ce=cev, stream=stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        ms_v = a.elapsed_time(b) / args.steps
+        zb = float(zv.numel() * zv.element_size())
+        vocab = {"workload": "qwen2.5-14b head error", "N": wv.N, "V": wv.V, "C": wv.C, "ms": ms_v,
+                 "roofline": {"bound": "hbm", "achieved": zb / (ms_v / 1e3) / 1e9, "peak": hbm_peak(), "unit": "GB/s",
+                              "frac": zb / (ms_v / 1e3) / 1e9 / hbm_peak(), "kernel": "k_head_error<bf16>",
+                              "bytes_per_launch": zb}}
+        del zv, Ev, cev
+        torch.cuda.empty_cache()
+
     # end to end through the public API: host inputs copied in, adapters copied out, per step
     e2e = None
     if not args.no_e2e:
@@ -482,6 +521,7 @@ def main():
             "gpu_launches": launches_per_step * args.steps,
             "e2e": e2e,
             "kspace": kspace,
+            "head_error_vocab": vocab,
             "cpu_baseline": cpu,
             "clocks": clk.summary(),
         }

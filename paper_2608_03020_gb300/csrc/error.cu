@@ -5,6 +5,8 @@
 // so the row is read from HBM exactly once; the 32 partial (max, sum) pairs are merged with
 // warp shuffles.  The C label columns are then gathered to form
 //   E[n, c] = w_n (exp(z[n, col_c] - lse_n) - [y_n == c]),   ce[n] = w_n (lse_n - z[n, col_{y_n}]).
+// The running maximum and sum are kept in base-2 units (t = z log2 e), so each logit costs one
+// FMA and one exp2f; lse = (m + log2 s) ln 2.
 // Bound: HBM read of the logits (N * V * elsize bytes); for V == C the kernel is launch-bound.
 #include <cuda_bf16.h>
 #include <math.h>
@@ -17,22 +19,30 @@ namespace {
 __device__ __forceinline__ float to_f(float v) { return v; }
 __device__ __forceinline__ float to_f(__nv_bfloat16 v) { return __bfloat162float(v); }
 
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+
+// running maximum m and sum s of 2^(t - m) over t = z log2 e seen so far
 struct RunMax {
   float m = -INFINITY;
   float s = 0.f;
   __device__ __forceinline__ void rescale_to(float mn) {
     if (mn > m) {
-      s = (m == -INFINITY) ? 0.f : s * expf(m - mn);
+      s = (m == -INFINITY) ? 0.f : s * exp2f(m - mn);
       m = mn;
     }
+  }
+  __device__ __forceinline__ void add(float z) {  // one logit (natural units)
+    rescale_to(z * kLog2e);
+    if (m != -INFINITY) s += exp2f(fmaf(z, kLog2e, -m));
   }
 };
 
 __device__ __forceinline__ void merge(RunMax& a, float m2, float s2) {
   const float mn = fmaxf(a.m, m2);
   if (mn == -INFINITY) return;
-  const float sa = (a.m == -INFINITY) ? 0.f : a.s * expf(a.m - mn);
-  const float sb = (m2 == -INFINITY) ? 0.f : s2 * expf(m2 - mn);
+  const float sa = (a.m == -INFINITY) ? 0.f : a.s * exp2f(a.m - mn);
+  const float sb = (m2 == -INFINITY) ? 0.f : s2 * exp2f(m2 - mn);
   a.m = mn;
   a.s = sa + sb;
 }
@@ -68,11 +78,11 @@ __device__ __forceinline__ void accumulate_vec(RunMax& a, const float* v) {
   float vm = v[0];
 #pragma unroll
   for (int i = 1; i < n; ++i) vm = fmaxf(vm, v[i]);
-  a.rescale_to(vm);
+  a.rescale_to(vm * kLog2e);
   if (a.m == -INFINITY) return;
   float t = 0.f;
 #pragma unroll
-  for (int i = 0; i < n; ++i) t += expf(v[i] - a.m);
+  for (int i = 0; i < n; ++i) t += exp2f(fmaf(v[i], kLog2e, -a.m));
   a.s += t;
 }
 
@@ -110,17 +120,9 @@ __global__ void __launch_bounds__(256) k_head_error(const Tz* __restrict__ z, in
         }
         j0 = nvec * VN;
       }
-      for (int64_t j = j0 + lane; j < V; j += 32) {
-        const float v = to_f(row[j]);
-        a1.rescale_to(v);
-        if (a1.m != -INFINITY) a1.s += expf(v - a1.m);
-      }
+      for (int64_t j = j0 + lane; j < V; j += 32) a1.add(to_f(row[j]));
     } else {
-      for (int c = lane; c < C; c += 32) {
-        const float v = to_f(row[cols[c]]);
-        a0.rescale_to(v);
-        if (a0.m != -INFINITY) a0.s += expf(v - a0.m);
-      }
+      for (int c = lane; c < C; c += 32) a0.add(to_f(row[cols[c]]));
     }
     merge(a0, a1.m, a1.s);
 #pragma unroll
@@ -129,7 +131,7 @@ __global__ void __launch_bounds__(256) k_head_error(const Tz* __restrict__ z, in
       const float s2 = __shfl_xor_sync(0xffffffffu, a0.s, off);
       merge(a0, m2, s2);
     }
-    const float lse = a0.m + logf(a0.s);
+    const float lse = (a0.m + log2f(a0.s)) * kLn2;
     const int yn = y[n];
     const float wn = (yn < 0) ? 0.f : (w ? w[n] : 1.f);
     for (int c = lane; c < C; c += 32) {
