@@ -405,9 +405,9 @@ def main():
         gen = torch.Generator(device=dev)
         gen.manual_seed(1234)
         zv = torch.empty((wv.N, wv.V), dtype=torch.bfloat16, device=dev)
-        fv = S.host_factors(wv, 0)
-        cols_v = torch.from_numpy(fv["label_cols"].astype(np.int32)).to(dev)
-        y_v = torch.from_numpy(fv["y"].astype(np.int32)).to(dev)
+        rng = np.random.default_rng(1234)
+        cols_v = torch.from_numpy(np.sort(rng.choice(wv.V, size=wv.C, replace=False)).astype(np.int32)).to(dev)
+        y_v = torch.from_numpy(rng.integers(0, wv.C, wv.N).astype(np.int32)).to(dev)
         off = float(np.log(wv.V / wv.C))
         for n0 in range(0, wv.N, 8192):
             g = torch.randn((min(8192, wv.N - n0), wv.V), generator=gen, device=dev)
