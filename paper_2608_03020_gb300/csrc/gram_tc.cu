@@ -23,13 +23,15 @@
 // tiles that touch the upper triangle and all cross tiles of that column, paired in order).
 // Gram elements (i, j), i <= j, are stored directly and mirrored to (j, i): every output element
 // has one writer (deterministic, no atomics).  MMA commits multicast to both CTAs' barriers.
-// Lockstep: all clusters stream the same token window of X_l and T_l at the same time, so each
-// operand line is read from HBM once and then served from L2 to the ~25 tiles that need it.  The
-// clusters start every round of work items together: the even CTA's producer counts the items whose
-// loads it has issued on a launch-local counter and, before the next item, waits (bounded, as a hint
-// only) until every cluster has done the same.  Without it the clusters drift apart over a few
-// items (items differ in length and epilogue cost), the L2 no longer holds what the others read,
-// and the load latency, not the tensor core, sets the pace (about 1.25x slower at 7B size).
+// Lockstep: all clusters stream the same token window of X_l and T_l at the same time, so an
+// operand line read from HBM is then served from L2 to the other tiles that need it.  The even
+// CTA's producer passes a sync point at the start of every work item and every kSyncEvery
+// k-blocks within it: it counts the point on a launch-local counter and waits (bounded, as a hint
+// only) until every cluster with an item in this round has counted it too.  Without the item-level
+// points the clusters drift apart over a few items (items differ in length and epilogue cost), the
+// L2 no longer holds what the others read, and the load latency, not the tensor core, sets the
+// pace (about 1.25x slower at 7B size); the points within items keep the clusters' token windows
+// within ~L2 of each other (HBM re-reads 4.0x -> 2.6x of X and T, 3-4% faster under the power cap).
 // Every mbarrier wait is bounded: on expiry the status word gets LOCA_ERR_TIMEOUT, a launch-local
 // flag makes every other wait give up, the even CTA drains the loads and MMAs in flight, and
 // both CTAs meet at the final cluster barrier before TMEM is freed.
@@ -52,6 +54,7 @@ constexpr int BN = 256;                             // accumulator columns (chan
 constexpr int BNC = 128;                            // B columns loaded per CTA
 constexpr int BK = 64;                              // tokens per pipeline stage
 constexpr int STAGES = 4;
+constexpr int kSyncEvery = 128;                     // k-blocks between lockstep sync points
 constexpr int SUB_BYTES = 64 * BK * 2;              // one 64-channel x 64-token swizzled tile (8 KB)
 constexpr int A_BYTES = BMC * BK * 2;               // 16 KB
 constexpr int B_BYTES = BNC * BK * 2;               // 16 KB
@@ -173,23 +176,32 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       uint32_t phase = 0;
       uint32_t pending = 0, pending_par = 0;  // even CTA: armed stages and their phase parity
       bool ok = true;
-      bool sync = leader;  // dropped for the rest of the launch if a round wait runs out
-      uint32_t round = 0;
-      for (int it = cid; it < total_items && ok; it += ncl, ++round) {
-        if (sync && round > 0) {
-          // every cluster has issued the loads of its previous item (hint: bounded, no error)
-          const uint32_t target = uint32_t(ncl) * round;
-          const uint64_t t0 = globaltimer();
-          while (*reinterpret_cast<volatile uint32_t*>(round_ctr) < target) {
-            if (globaltimer() - t0 > sync_ns) {
-              sync = false;
-              break;
-            }
+      bool sync = leader;  // dropped for the rest of the launch if a wait runs out
+      // sync points: each item counts one every kSyncEvery k-blocks and one at its end (P per item)
+      const int P = (nkb + kSyncEvery - 1) / kSyncEvery;
+      uint32_t before = 0;  // counts expected from all earlier rounds
+      auto wait_for = [&](uint32_t target) {  // a hint: bounded, no error
+        const uint64_t t0 = globaltimer();
+        while (*reinterpret_cast<volatile uint32_t*>(round_ctr) < target) {
+          if (globaltimer() - t0 > sync_ns) {
+            sync = false;
+            break;
           }
         }
+      };
+      uint32_t round = 0;
+      for (int it = cid; it < total_items && ok; it += ncl, ++round) {
+        // clusters with an item in this round (the last round may be partial)
+        const int left = total_items - int(round) * ncl;
+        const uint32_t active = uint32_t(left < ncl ? left : ncl);
+        if (sync && round > 0) wait_for(before);  // every cluster finished issuing its last item
         const Item w = decode(g, it);
         const uint32_t bytes_both = 2u * (uint32_t(w.nslots) * A_BYTES + B_BYTES);
         for (int kb = 0; kb < nkb; ++kb) {
+          if (leader && kb > 0 && kb % kSyncEvery == 0) {
+            atomicAdd(round_ctr, 1u);
+            if (sync) wait_for(before + active * uint32_t(kb / kSyncEvery));
+          }
           if (!mbar_try_wait_cluster(empty_bar(stage), phase ^ 1u) &&
               !mbar_wait_cluster(empty_bar(stage), phase ^ 1u, wc)) {
             ok = false;
@@ -224,6 +236,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
           if (++stage == STAGES) { stage = 0; phase ^= 1u; }
         }
         if (ok && leader) atomicAdd(round_ctr, 1u);
+        before += active * uint32_t(P);
       }
       if (!ok && leader) {
         // the armed stages count the bytes of both CTAs: let them land before either CTA exits
