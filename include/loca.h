@@ -69,6 +69,18 @@ enum { LOCA_F32 = 0, LOCA_BF16 = 1 };
 /* Library ABI version (major * 10000 + minor * 100 + patch). */
 int loca_version(void);
 
+/*
+ * loca_set_wait_limit — test hook for the failure path (the paper has no counterpart).  Every
+ * wait of the tensor-core kernels on an mbarrier (a copy landing, an MMA completing) is bounded;
+ * when one runs out the kernel records LOCA_ERR_TIMEOUT in the device status word, makes the
+ * other waits of its launch give up, lets the copies and MMAs already in flight land, frees its
+ * tensor memory and returns, so the context stays usable.  This sets, for the whole process,
+ * how long such a wait may take in the single-CTA kernels (loca_targets, loca_kspace_accumulate)
+ * before it gives up: ns = 0 restores the default of 4 s; a tiny value makes a call time out on
+ * purpose, to test that path.  (The CTA-pair Gram / cross kernel always uses 4 s.)
+ */
+int loca_set_wait_limit(uint64_t ns);
+
 /* Message for the last non-OK status returned to the calling thread ("" if none). */
 const char* loca_last_error_string(void);
 

@@ -169,7 +169,7 @@ __global__ void __launch_bounds__(XA_THREADS, 1)
       }
       if (!ok) {
         for (int s = 0; s < XA_STAGES; ++s)
-          if (pending & (1u << s)) mbar_drain(full_bar(s), (pending_par >> s) & 1u, limit_ns);
+          if (pending & (1u << s)) mbar_drain(full_bar(s), (pending_par >> s) & 1u, kDrainLimitNs);
       }
     }
     __syncwarp();
@@ -205,7 +205,7 @@ __global__ void __launch_bounds__(XA_THREADS, 1)
       }
       if (!ok && issued) {
         mma_commit(drain_bar);
-        mbar_drain(drain_bar, 0, limit_ns);
+        mbar_drain(drain_bar, 0, kDrainLimitNs);
       }
     }
     __syncwarp();
@@ -658,7 +658,7 @@ cudaError_t launch_kspace_accumulate(const void* X, int L, int64_t N, int64_t d,
   int grid = sm_count();
   if (grid > XA_MAX_GRID) grid = XA_MAX_GRID;
   if (grid > L * ntiles) grid = L * ntiles;
-  const unsigned long long limit = 4000000000ull;
+  const unsigned long long limit = wait_limit_ns();
   if (kp == 16) {
     e = cudaFuncSetAttribute(k_kspace_xa<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, XA_SMEM);
     if (e != cudaSuccess) return e;

@@ -5,6 +5,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 
 #include "loca_internal.h"
@@ -67,6 +68,15 @@ int sm_count() {
     cache[dev] = v;
   }
   return cache[dev];
+}
+
+namespace {
+std::atomic<unsigned long long> g_wait_limit_ns{0};
+}
+
+unsigned long long wait_limit_ns() {
+  const unsigned long long v = g_wait_limit_ns.load(std::memory_order_relaxed);
+  return v == 0 ? 4000000000ull : v;
 }
 
 int32_t* device_status_word() {
@@ -179,6 +189,11 @@ extern "C" {
 int loca_version(void) { return 100; }
 
 const char* loca_last_error_string(void) { return g_msg; }
+
+int loca_set_wait_limit(uint64_t ns) {
+  g_wait_limit_ns.store(ns, std::memory_order_relaxed);
+  return LOCA_OK;
+}
 
 int loca_device_status(int32_t* host_status, void* stream) {
   if (host_status == nullptr) return fail(LOCA_ERR_INVALID_ARG, "host_status is NULL");

@@ -251,7 +251,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       }
       if (!ok && issued) {
         mma_commit(drain_bar);
-        mbar_drain(drain_bar, 0, limit_ns);
+        mbar_drain(drain_bar, 0, kDrainLimitNs);
       }
     }
     __syncwarp();
@@ -462,7 +462,7 @@ cudaError_t launch_targets(const float* E, int64_t N, int C, const float* P, con
   }
   const Layout lay = layout_for(g.rp);
   const size_t shm = lay.total;
-  const unsigned long long limit = 4000000000ull;
+  const unsigned long long limit = wait_limit_ns();
   if (t_dtype == LOCA_BF16) {
     e = cudaFuncSetAttribute(k_targets_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(shm));
     if (e != cudaSuccess) return e;

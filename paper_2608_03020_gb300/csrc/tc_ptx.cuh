@@ -52,13 +52,14 @@ struct WaitCtl {
 };
 
 // Bounded wait for the phase of parity `parity` of barrier `bar`.  Returns false when the wait
-// gave up (time limit reached, or another waiter of this launch gave up).
+// gave up (time limit reached, or another waiter of this launch gave up).  A try_wait that fails
+// may itself have suspended the thread for a while, so the limit is checked every 8 of them.
 static __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const WaitCtl& w) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 255u) == 0) {
+    if ((it & 7u) == 0) {
       if (*w.abort_flag != 0) return false;
       if (globaltimer() - t0 > w.limit_ns) {
         atomicExch(w.status, int32_t(LOCA_ERR_TIMEOUT));
@@ -69,6 +70,10 @@ static __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, con
     }
   }
 }
+
+// Limit of the drain waits below: independent of the (possibly tiny, for testing) limit of the
+// ordinary waits, so that copies and MMAs in flight always land before a CTA exits.
+constexpr uint64_t kDrainLimitNs = 2000000000ull;
 
 // Wait (up to limit_ns) for a phase without touching the abort flag: used to drain copies or
 // MMAs already in flight before a CTA that gave up exits.

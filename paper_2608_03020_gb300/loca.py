@@ -36,6 +36,7 @@ SIGNATURES = [
     ("loca_version", ctypes.c_int, []),
     ("loca_last_error_string", ctypes.c_char_p, []),
     ("loca_device_status", ctypes.c_int, [ctypes.POINTER(_I32), _P]),
+    ("loca_set_wait_limit", ctypes.c_int, [ctypes.c_uint64]),
     ("loca_error", ctypes.c_int, [_P, ctypes.c_int, _I64, _I64, _I64, _P, _I32, _P, _P, ctypes.c_int, _P, _P, _P]),
     ("loca_targets_workspace_size", ctypes.c_int, [_I64, _I32, _I64, ctypes.POINTER(_SZ)]),
     ("loca_targets", ctypes.c_int, [_P, _I64, _I32, _P, _P, _I32, _I32, _I64, _P, ctypes.c_int, _P, _P, _SZ, _P]),
@@ -148,6 +149,12 @@ def loca_device_status(stream=None) -> int:
     out = ctypes.c_int32(0)
     _check(lib().loca_device_status(ctypes.byref(out), _stream(stream)), "loca_device_status")
     return out.value
+
+
+def loca_set_wait_limit(ns: int):
+    """Test hook: how long a device wait of the single-CTA tensor-core kernels may take before it
+    gives up with LOCA_ERR_TIMEOUT (0 restores the default of 4 s)."""
+    _check(lib().loca_set_wait_limit(int(ns)), "loca_set_wait_limit")
 
 
 def loca_error(logits, label_cols, y, E, w=None, ce=None, normaliser=0, stream=None):

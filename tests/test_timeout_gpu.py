@@ -1,0 +1,78 @@
+"""The failure path of the bounded device waits, exercised without faulting or hanging the GPU.
+
+A wait limit of 1 microsecond (the loca_set_wait_limit test hook) makes the first wait of the
+tensor-core kernels that does not succeed at once give up: the kernel must record
+LOCA_ERR_TIMEOUT in the device status word, let its copies and MMAs in flight land, free its
+tensor memory and return.  The CUDA context must stay usable: with the default limit restored,
+the same call then gives results bit-identical to a call made before the failure, and the status
+word reads OK.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+pytestmark = pytest.mark.gpu
+
+LOCA_ERR_TIMEOUT = 6
+
+
+@pytest.fixture(scope="module")
+def lc():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    from paper_2608_03020_gb300 import _build
+
+    _build.build()
+    from paper_2608_03020_gb300 import loca
+
+    loca.lib()
+    yield loca
+    loca.loca_set_wait_limit(0)
+
+
+def _kspace_call(lc, X, A, E, P, Q):
+    L, N, d = X.shape
+    k, C = A.shape[2], E.shape[1]
+    G = torch.empty((L, k, k), device="cuda")
+    SC = torch.empty((L, C, k), device="cuda")
+    xsq = torch.empty((L,), dtype=torch.float64, device="cuda")
+    lc.loca_kspace_accumulate(X, A, E, P, Q, 0.01, G, SC, xsq, zero_first=True)
+    torch.cuda.synchronize()
+    return G, SC, xsq
+
+
+def _targets_call(lc, E, P, Q, L, N, d):
+    T = torch.empty((L, N, d), dtype=torch.bfloat16, device="cuda")
+    tsq = torch.empty((L,), dtype=torch.float64, device="cuda")
+    lc.loca_targets(E, P, Q, T, tsq=tsq)
+    torch.cuda.synchronize()
+    return T, tsq
+
+
+def test_wait_timeout_is_reported_and_the_context_recovers(lc):
+    g = torch.Generator(device="cuda")
+    g.manual_seed(5)
+    L, N, d, k, C, r = 4, 32768, 1024, 16, 4, 16
+    X = torch.randn((L, N, d), device="cuda", generator=g).to(torch.bfloat16)
+    A = torch.randn((L, d, k), device="cuda", generator=g) * 0.03
+    E = torch.randn((N, C), device="cuda", generator=g)
+    P = torch.randn((L, C, r), device="cuda", generator=g) * 0.25
+    Q = torch.randn((L, r, d), device="cuda", generator=g) * 0.25
+    lc.loca_set_wait_limit(0)
+    assert lc.loca_device_status() == 0
+    ref_k = _kspace_call(lc, X, A, E, P, Q)
+    ref_t = _targets_call(lc, E, P, Q, L, N, d)
+    assert lc.loca_device_status() == 0
+    for call in ("kspace", "targets"):
+        lc.loca_set_wait_limit(1000)  # 1 us: a wait that does not succeed at once gives up
+        if call == "kspace":
+            _kspace_call(lc, X, A, E, P, Q)
+        else:
+            _targets_call(lc, E, P, Q, L, N, d)
+        assert lc.loca_device_status() == LOCA_ERR_TIMEOUT, call
+        lc.loca_set_wait_limit(0)
+        again_k = _kspace_call(lc, X, A, E, P, Q)
+        again_t = _targets_call(lc, E, P, Q, L, N, d)
+        assert lc.loca_device_status() == 0, call
+        for a, b in zip(ref_k + ref_t, again_k + again_t):
+            assert torch.equal(a, b), call
