@@ -33,6 +33,7 @@ __all__ = [
     "rms",
     "head_error",
     "feedback_targets",
+    "alignment",
     "scaled_step",
     "accumulate_stats",
     "project_stats",
@@ -112,6 +113,24 @@ def feedback_targets(E, P, Q):
     T = np.stack([(E @ P[l]) @ Q[l] for l in range(L)])
     tsq = np.array([np.sum(T[l] * T[l]) for l in range(L)])
     return T, tsq
+
+
+def alignment(E, P, Q, G):
+    """In-probe alignment diagnostic (supplement, "One-shot calibration": the cosine between
+    the stacked feedback predictions and the stacked exact probe gradients of each block).
+
+    ``alpha_l = <G_l, T_l>_F / (||G_l||_F ||T_l||_F)`` with ``T_l = E P_l Q_l`` (the
+    predictions of :func:`feedback_targets`) and ``G_l`` (``Np x d``) the exact hidden-state
+    gradients at the same probe positions.  0 where either matrix is zero.
+    """
+    T, tsq = feedback_targets(E, P, Q)
+    G = np.asarray(G, dtype=np.float64)
+    out = np.zeros(T.shape[0])
+    for l in range(T.shape[0]):
+        gg = float(np.sum(G[l] * G[l]))
+        if gg > 0.0 and tsq[l] > 0.0:
+            out[l] = float(np.sum(G[l] * T[l])) / np.sqrt(gg * tsq[l])
+    return out
 
 
 def scaled_step(eta, X_l, T_l):

@@ -519,3 +519,28 @@ def test_linear_network_targets_equal_backprop_gradients():
     T, _ = O.feedback_targets(E, P, Q)
     for l in range(Ln):
         assert _rel(T[l], Gp[l]) < 1e-7
+
+
+def test_alignment_special_cases():
+    """The alignment cosine: 1 for gradients equal to the predictions up to a positive scale,
+    -1 for the opposite direction, 0 for gradients orthogonal to every prediction (built by
+    projecting the predictions' row space out), and the mean of a hand-computed per-block cosine
+    otherwise; it ignores the scale of P."""
+    rng = np.random.default_rng(4)
+    Np, C, r, d, L = 50, 3, 2, 7, 2
+    E = rng.standard_normal((Np, C))
+    P = rng.standard_normal((L, C, r))
+    Q = rng.standard_normal((L, r, d))
+    T = np.stack([E @ P[l] @ Q[l] for l in range(L)])
+    assert np.allclose(O.alignment(E, P, Q, 3.0 * T), 1.0, atol=1e-12)
+    assert np.allclose(O.alignment(E, P, Q, -0.5 * T), -1.0, atol=1e-12)
+    G = rng.standard_normal((L, Np, d))
+    for l in range(L):
+        Qo, _ = np.linalg.qr(Q[l].T)  # orthonormal basis of the rows of T_l (in R^d)
+        G[l] -= (G[l] @ Qo) @ Qo.T
+    assert np.allclose(O.alignment(E, P, Q, G), 0.0, atol=1e-12)
+    G = rng.standard_normal((L, Np, d))
+    want = [float(np.dot(G[l].ravel(), T[l].ravel()) / np.linalg.norm(G[l]) / np.linalg.norm(T[l])) for l in range(L)]
+    assert np.allclose(O.alignment(E, P, Q, G), want, rtol=1e-12)
+    assert np.allclose(O.alignment(E, 5.0 * P, Q, G), want, rtol=1e-12)
+    assert np.all(O.alignment(E, 0.0 * P, Q, G) == 0.0)
