@@ -450,6 +450,34 @@ int loca_accumulate_streamed(const void* X_host, void* staging, const void* T, i
   return LOCA_OK;
 }
 
+int loca_alignment_workspace_size(int64_t Np, int64_t d, int32_t L, size_t* bytes) {
+  if (!bytes) return fail(LOCA_ERR_INVALID_ARG, "bytes is NULL");
+  if (Np < 0 || d < 1 || L < 1) return fail(LOCA_ERR_SHAPE, "need Np >= 0, d >= 1, L >= 1");
+  *bytes = align_workspace_bytes(Np, d, L);
+  return LOCA_OK;
+}
+
+int loca_alignment(const float* E_probe, const float* G_probe, int64_t Np, int32_t m, int64_t d, int32_t L,
+                   const float* P, const float* Q, int32_t r, double* alpha, void* workspace,
+                   size_t workspace_bytes, void* stream) {
+  g_msg[0] = 0;
+  if (Np < 0 || d < 1 || L < 1 || L > 65535 || Np > (int64_t(1) << 31))
+    return fail(LOCA_ERR_SHAPE, "need 0 <= Np < 2^31, d >= 1, 1 <= L <= 65535");
+  if (m < 1 || m > align_max_m()) return fail(LOCA_ERR_SHAPE, "need 1 <= m <= %d, got m=%d", align_max_m(), m);
+  if (r < 1 || r > align_max_r()) return fail(LOCA_ERR_SHAPE, "need 1 <= r <= %d, got r=%d", align_max_r(), r);
+  if ((Np > 0 && (!E_probe || !G_probe)) || !P || !Q || !alpha)
+    return fail(LOCA_ERR_INVALID_ARG, "E_probe, G_probe, P, Q and alpha are required");
+  if ((E_probe && !aligned(E_probe, 4)) || (G_probe && !aligned(G_probe, 4)) || !aligned(P, 4) || !aligned(Q, 4) ||
+      !aligned(alpha, 8))
+    return fail(LOCA_ERR_ALIGNMENT, "pointers must be aligned to their element size");
+  const int rc = check_ws(workspace, workspace_bytes, align_workspace_bytes(Np, d, L));
+  if (rc != LOCA_OK) return rc;
+  cudaError_t e = launch_alignment(E_probe, G_probe, Np, m, d, L, P, Q, r, alpha, workspace,
+                                   static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "loca_alignment launch");
+  return LOCA_OK;
+}
+
 int loca_kspace_workspace_size(int32_t L, int64_t N, int64_t d, int32_t k, int32_t C, int32_t r, size_t* bytes) {
   if (!bytes) return fail(LOCA_ERR_INVALID_ARG, "bytes is NULL");
   if (L < 1 || N < 0 || d < 1 || k < 1 || k > 32 || C < 1 || C > kspace_max_C() || r < 1 || r > kspace_max_r())

@@ -66,6 +66,13 @@ cudaError_t launch_gram_cross_tc(const void* X, const void* T, int L, int64_t N,
 // statistics): 4 s unless loca_set_wait_limit changed it.
 unsigned long long wait_limit_ns();
 
+// ---- alignment diagnostic (align.cu)
+int align_max_m();
+int align_max_r();
+size_t align_workspace_bytes(int64_t Np, int64_t d, int L);
+cudaError_t launch_alignment(const float* E, const float* G, int64_t Np, int m, int64_t d, int L, const float* P,
+                             const float* Q, int r, double* alpha, void* workspace, cudaStream_t s);
+
 // ---- k-space statistics and solve (kspace.cu)
 struct KspaceWs {
   size_t W, M, part, ete, flags, total;

@@ -47,6 +47,8 @@ SIGNATURES = [
      [_P, _P, ctypes.c_int, _I32, _I64, _I64, _P, _F, ctypes.c_int, _P, _P, _P, _P]),
     ("loca_accumulate_streamed", ctypes.c_int,
      [_P, _P, _P, ctypes.c_int, _I32, _I64, _I64, _I32, _P, _F, ctypes.c_int, _P, _P, _P, _P, _SZ, _P]),
+    ("loca_alignment_workspace_size", ctypes.c_int, [_I64, _I64, _I32, ctypes.POINTER(_SZ)]),
+    ("loca_alignment", ctypes.c_int, [_P, _P, _I64, _I32, _I64, _I32, _P, _P, _I32, _P, _P, _SZ, _P]),
     ("loca_kspace_workspace_size", ctypes.c_int, [_I32, _I64, _I64, _I32, _I32, _I32, ctypes.POINTER(_SZ)]),
     ("loca_kspace_accumulate", ctypes.c_int,
      [_P, ctypes.c_int, _I32, _I64, _I64, _P, _I32, _P, _I32, _P, _P, _I32, _F, ctypes.c_int, _P, _P, _P, _P, _P,
@@ -306,6 +308,27 @@ def loca_accumulate_streamed(X_host, staging, T, tsq, eta, gram, cross, xsq_tota
                                         int(bool(zero_first)), _ptr(gram), _ptr(cross), _ptr(xsq_total),
                                         _ptr(ws), nbytes, _stream(stream))
     _check(rc, "loca_accumulate_streamed")
+
+
+def loca_alignment(E_probe, G_probe, P, Q, alpha, workspace=None, stream=None):
+    """Per-block cosine between the feedback predictions E P_l Q_l and the probe gradients."""
+    _dev(E_probe, "E_probe", torch.float32, 2)
+    _dev(G_probe, "G_probe", torch.float32, 3)
+    _dev(P, "P", torch.float32, 3)
+    _dev(Q, "Q", torch.float32, 3)
+    _dev(alpha, "alpha", torch.float64, 1)
+    Np, m = E_probe.shape
+    L, _, d = G_probe.shape
+    r = P.shape[2]
+    if (tuple(G_probe.shape) != (L, Np, d) or tuple(P.shape) != (L, m, r) or tuple(Q.shape) != (L, r, d)
+            or alpha.numel() != L):
+        raise ValueError("shape mismatch among E_probe, G_probe, P, Q, alpha")
+    out = ctypes.c_size_t(0)
+    _check(lib().loca_alignment_workspace_size(Np, d, L, ctypes.byref(out)), "loca_alignment_workspace_size")
+    ws = _workspace(out.value, G_probe.device, workspace)
+    rc = lib().loca_alignment(_ptr(E_probe), _ptr(G_probe), Np, m, d, L, _ptr(P), _ptr(Q), r, _ptr(alpha), _ptr(ws),
+                              out.value, _stream(stream))
+    _check(rc, "loca_alignment")
 
 
 def kspace_workspace_size(L, N, d, k, C, r) -> int:

@@ -146,3 +146,60 @@ def test_calib_reports_beta_below_rounding(lc):
     else:
         assert st == 9
         assert torch.count_nonzero(P) == 0 and torch.count_nonzero(Q) == 0
+
+
+@pytest.mark.parametrize("Np,m,d,L,r", [(3000, 4, 328, 3, 4), (1500, 16, 1024, 2, 16), (700, 64, 96, 1, 32)])
+def test_alignment_matches_oracle(lc, Np, m, d, L, r):
+    """Supplement, one-shot calibration: the in-probe cosine of each block against the oracle's.
+    fp32 products summed in fp32 over 1024 tokens per thread, fp64 across: relative 1e-5."""
+    rng = np.random.default_rng(Np + d)
+    E = rng.standard_normal((Np, m)).astype(np.float32)
+    P = rng.standard_normal((L, m, r)).astype(np.float32)
+    Q = rng.standard_normal((L, r, d)).astype(np.float32)
+    T = np.stack([E.astype(np.float64) @ P[l] @ Q[l] for l in range(L)])
+    # gradients partly aligned with the predictions (alpha away from 0 and 1)
+    G = (0.5 * T / np.sqrt(np.mean(T * T)) + rng.standard_normal((L, Np, d))).astype(np.float32)
+    alpha = torch.empty((L,), dtype=torch.float64, device="cuda")
+    lc.loca_alignment(_dev(E), _dev(G), _dev(P), _dev(Q), alpha)
+    torch.cuda.synchronize()
+    ref = O.alignment(E, P, Q, G)
+    assert np.allclose(alpha.cpu().numpy(), ref, rtol=1e-5, atol=1e-7), (alpha.cpu().numpy(), ref)
+
+
+def test_alignment_of_calibrated_and_random_feedback(lc):
+    """On the all-linear network the calibrated feedback reproduces the gradients (alpha ~ 1);
+    random factors of the same shapes give alpha ~ 0 (the paper's contrast: -0.005 for random
+    feedback, 0.3-0.5 after calibration on real models)."""
+    rng = np.random.default_rng(33)
+    N, d, C, Ln = 4096, 64, 4, 3
+    W = [rng.standard_normal((d, d)) / math.sqrt(d) for _ in range(Ln)]
+    Wu = rng.standard_normal((C, d))
+    h = rng.standard_normal((N, d))
+    for m_ in range(Ln):
+        h = h @ W[m_].T
+    z = (h @ Wu.T).astype(np.float32)
+    y = rng.integers(0, C, N).astype(np.int32)
+    E = torch.empty((N, C), device="cuda")
+    lc.loca_error(_dev(z), _dev(np.arange(C, dtype=np.int32), torch.int32), _dev(y, torch.int32), E)
+    torch.cuda.synchronize()
+    E_h = E.cpu().numpy().astype(np.float64)
+    grads, M = [], Wu.copy()
+    for l in range(Ln, 0, -1):
+        grads.append(E_h @ M)
+        M = M @ W[l - 1]
+    G = _dev(np.stack(grads[::-1]).astype(np.float32))
+    P = torch.empty((Ln, C, C), device="cuda")
+    Q = torch.empty((Ln, C, d), device="cuda")
+    lc.loca_calib_fit(E, G, 1e-5 * float(torch.sum(E * E).item()) / C, C, P, Q)
+    alpha = torch.empty((Ln,), dtype=torch.float64, device="cuda")
+    lc.loca_alignment(E, G, P, Q, alpha)
+    torch.cuda.synchronize()
+    assert np.all(alpha.cpu().numpy() > 0.9999), alpha
+    Pr = _dev(rng.standard_normal((Ln, C, C)).astype(np.float32))
+    Qr = _dev(rng.standard_normal((Ln, C, d)).astype(np.float32))
+    lc.loca_alignment(E, G, Pr, Qr, alpha)
+    torch.cuda.synchronize()
+    a = alpha.cpu().numpy()
+    assert np.all(np.abs(a) < 0.5), a
+    ref = O.alignment(E_h, Pr.cpu().numpy(), Qr.cpu().numpy(), G.cpu().numpy())
+    assert np.allclose(a, ref, rtol=1e-5, atol=1e-6)
