@@ -206,8 +206,8 @@ def host_sample(w, seed=0, tokens=None):
 
 
 def run_reference(args, w):
-    host = host_sample(w, tokens=4096)
-    tokens = 2048
+    tokens = min(2048, w.N)  # bounded sample per step, capped at the workload's N
+    host = host_sample(w, tokens=tokens)
     for _ in range(args.warmup):
         oracle_sample(w, tokens, host)
     times = [oracle_sample(w, tokens, host) for _ in range(args.steps)]
