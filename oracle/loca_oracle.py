@@ -42,6 +42,7 @@ __all__ = [
     "ridge_solve",
     "calib_fit",
     "calib_fit_dual",
+    "calib_fit_rsvd",
     "loca_pass",
 ]
 
@@ -314,6 +315,71 @@ def calib_fit_dual(E_probe, G_probe, beta):
     L, Np, d = Gp.shape
     K = E @ E.T + beta * np.eye(Np)
     return np.stack([E.T @ np.linalg.solve(K, Gp[l]) for l in range(L)])
+
+
+def calib_fit_rsvd(E_probe, G_probe, beta, r, Omega, q):
+    """Rank-r truncation of the feedback ridge fit (Eq. 5; S5) for error spaces too wide to
+    form and decompose ``F_hat_l^T`` (the paper's ``m = d`` form ``e = W_u^T eps``), by
+    randomized subspace iteration: Halko, Martinsson and Tropp, "Finding structure with
+    randomness" (SIAM Review 53, 2011), Algorithm 4.4 (range finder with ``q`` power
+    iterations, an orthonormal basis taken after every product) followed by Algorithm 5.1
+    (SVD of the matrix projected on that basis).  It approximates :func:`calib_fit`; with
+    ``ell >= rank(F_hat_l^T)`` it is exact.
+
+    ``F_hat_l^T = (E^T E + beta I_m)^{-1} E^T G_l`` (``m x d``) is only applied to blocks
+    of ``ell = Omega.shape[1]`` vectors, each time by solving with ``E^T E + beta I_m``:
+
+        F^T x = (E^T E + beta I)^{-1} E^T (G_l x),     F y = G_l^T E (E^T E + beta I)^{-1} y.
+
+    Steps: ``Y = F^T Omega``, ``Q_Y = orth(Y)``; ``q`` times ``Z = orth(F Q_Y)``,
+    ``Q_Y = orth(F^T Z)``; then ``B^T = F Q_Y`` (``d x ell``), ``B = U_B S V^T`` and
+    ``U = Q_Y U_B``; ``P_l = U_r S_r``, ``Q_l = V_r^T``.  ``orth`` is any orthonormal basis
+    of the columns' span (here a reduced QR).  Signs as in :func:`calib_fit` (the entry of
+    largest magnitude in each ``Q_l`` row is positive); singular values at or below
+    ``1e-12 sigma_1`` count as zero (zero ``Q_l`` row and ``P_l`` column).  ``Omega``
+    (``d x ell``) is the caller's Gaussian test matrix, the same for every block.
+
+    Returns ``P`` (``L x m x r``), ``Q`` (``L x r x d``) and ``sigma`` (``L x r``).
+    """
+    E = np.asarray(E_probe, dtype=np.float64)
+    Gp = np.asarray(G_probe, dtype=np.float64)
+    Om = np.asarray(Omega, dtype=np.float64)
+    L, Np, d = Gp.shape
+    m = E.shape[1]
+    K = E.T @ E + beta * np.eye(m)
+
+    def orth(Y):
+        return np.linalg.qr(Y, mode="reduced")[0]
+
+    P = np.zeros((L, m, r))
+    Q = np.zeros((L, r, d))
+    sig = np.zeros((L, r))
+    for l in range(L):
+        G = Gp[l]
+
+        def Ft(X):  # F_hat^T X
+            return np.linalg.solve(K, E.T @ (G @ X))
+
+        def F(Y):  # F_hat Y
+            return G.T @ (E @ np.linalg.solve(K, Y))
+
+        QY = orth(Ft(Om))
+        for _ in range(q):
+            Z = orth(F(QY))
+            QY = orth(Ft(Z))
+        Bt = F(QY)
+        UB, s, Vt = np.linalg.svd(Bt.T, full_matrices=False)
+        U = QY @ UB
+        for i in range(min(r, s.size)):
+            if not s[i] > 1e-12 * s[0]:
+                break
+            u, v = U[:, i].copy(), Vt[i].copy()
+            if v[np.argmax(np.abs(v))] < 0:
+                u, v = -u, -v
+            P[l, :, i] = u * s[i]
+            Q[l, i] = v
+            sig[l, i] = s[i]
+    return P, Q, sig
 
 
 def loca_pass(z, label_cols, y, X, P, Q, A, eta, lambda_rel, w=None, normaliser=0,

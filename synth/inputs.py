@@ -23,7 +23,10 @@ Recipe (seed 0 unless stated):
   (orthonormal columns).
 * Probe pairs for the calibration fit: ``E_probe ~ N(0, 1)`` (``Np x m``) and
   ``G_probe_l = E_probe M_l + 0.1 * rms(E_probe M_l) * noise`` with ``M_l`` a planted
-  rank-``min(rank, m)`` map.
+  rank-``min(rank, m)`` map.  For the paper's d-wide error space (``m = d``) the columns
+  of ``E_probe`` optionally get LogNormal(0, 0.5) scales, so that ``E^T E`` is
+  anisotropic like an unembedded error (``e_scales=True``).
+* Test matrix of the randomized top-r fit: ``Omega ~ N(0, 1)`` (``d x ell``).
 
 Host generation (numpy) serves the small shapes the oracle runs in full; device
 generation (torch on CUDA) serves the full-size shapes, whose small factors
@@ -40,7 +43,7 @@ from dataclasses import dataclass
 import numpy as np
 
 # tensor ids used to derive independent streams from one seed
-_S_SCALE, _S_X, _S_HEAD, _S_Y, _S_COLS, _S_P, _S_Q, _S_A, _S_Z, _S_PE, _S_PM, _S_PN, _S_OUT, _S_BPREV = range(1, 15)
+_S_SCALE, _S_X, _S_HEAD, _S_Y, _S_COLS, _S_P, _S_Q, _S_A, _S_Z, _S_PE, _S_PM, _S_PN, _S_OUT, _S_BPREV, _S_OMEGA, _S_PSC = range(1, 17)
 
 
 @dataclass(frozen=True)
@@ -168,21 +171,66 @@ def host_inputs(w: Workload, seed: int = 0) -> dict:
     return f
 
 
+def probe_error_scales(m: int, seed: int = 0) -> np.ndarray:
+    """Column scales of ``E_probe`` for ``e_scales=True`` (LogNormal(0, 0.5), ``m``)."""
+    return _rng(seed, _S_PSC).lognormal(0.0, 0.5, size=m)
+
+
+def planted_factors(m: int, d: int, rank: int, seed: int, l: int) -> tuple[np.ndarray, np.ndarray]:
+    """The two factors of block ``l``'s planted map ``M_l = a b / sqrt(rho)``, ``rho = min(rank, m)``."""
+    rho = min(rank, m)
+    g = _rng(seed, _S_PM, l)
+    return g.standard_normal(size=(m, rho)), g.standard_normal(size=(rho, d))
+
+
 def host_probe_pairs(Np: int, m: int, d: int, L: int, rank: int, noise: float = 0.1,
-                     seed: int = 0) -> dict:
+                     seed: int = 0, e_scales: bool = False) -> dict:
     """Probe pairs for the calibration fit: ``E_probe`` (``Np x m``), ``G_probe`` (``L x Np x d``),
     and the planted maps ``M`` (``L x m x d``, rank ``min(rank, m)``)."""
     E = _rng(seed, _S_PE).standard_normal(size=(Np, m))
+    if e_scales:
+        E = E * probe_error_scales(m, seed)[None, :]
     rho = min(rank, m)
     M = np.empty((L, m, d))
     G = np.empty((L, Np, d))
     for l in range(L):
-        g = _rng(seed, _S_PM, l)
-        M[l] = (g.standard_normal(size=(m, rho)) @ g.standard_normal(size=(rho, d))) / math.sqrt(rho)
+        a, b = planted_factors(m, d, rank, seed, l)
+        M[l] = (a @ b) / math.sqrt(rho)
         clean = E @ M[l]
         nz = _rng(seed, _S_PN, l).standard_normal(size=(Np, d))
         G[l] = clean + noise * math.sqrt(float(np.mean(clean ** 2))) * nz
     return dict(E_probe=E.astype(np.float32), G_probe=G.astype(np.float32), M=M)
+
+
+def device_probe_pairs(Np: int, m: int, d: int, L: int, rank: int, noise: float = 0.1, seed: int = 0,
+                       e_scales: bool = True, device="cuda") -> dict:
+    """Full-size probe pairs drawn on ``device`` with the recipe of :func:`host_probe_pairs`
+    (seeded CUDA generator for the ``Np``-row arrays; the planted factors and column scales
+    from the host streams).  Returns fp32 ``E_probe`` (``Np x m``) and ``G_probe``
+    (``L x Np x d``)."""
+    import torch
+
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed) * 1_000_003 + _S_PE)
+    E = torch.randn((Np, m), generator=gen, device=device, dtype=torch.float32)
+    if e_scales:
+        E *= torch.from_numpy(probe_error_scales(m, seed).astype(np.float32)).to(device)[None, :]
+    rho = min(rank, m)
+    G = torch.empty((L, Np, d), device=device, dtype=torch.float32)
+    for l in range(L):
+        a, b = planted_factors(m, d, rank, seed, l)
+        Ml = torch.from_numpy(((a @ b) / math.sqrt(rho)).astype(np.float32)).to(device)
+        clean = E @ Ml
+        gen.manual_seed(int(seed) * 1_000_003 + 7919 * (l + 1) + _S_PN)
+        nz = torch.randn((Np, d), generator=gen, device=device, dtype=torch.float32)
+        G[l] = clean + noise * torch.sqrt(torch.mean(clean * clean)) * nz
+        del Ml, clean, nz
+    return dict(E_probe=E, G_probe=G)
+
+
+def omega_matrix(d: int, ell: int, seed: int = 0) -> np.ndarray:
+    """Gaussian test matrix ``Omega`` (``d x ell``, fp32) of the randomized top-r fit."""
+    return _rng(seed, _S_OMEGA).standard_normal(size=(d, ell)).astype(np.float32)
 
 
 def device_inputs(w: Workload, seed: int = 0, device="cuda", x_source: str = "device",

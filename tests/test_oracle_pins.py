@@ -477,6 +477,69 @@ def test_calib_zero_pads_missing_rank():
     assert np.all(P[0, :, 2:] == 0) and np.all(Q[0, 2:] == 0) and np.all(sig[0, 2:] == 0)
 
 
+def test_rsvd_full_width_sketch_is_the_exact_fit():
+    """With ell = m the sketch spans the whole error space, so the Rayleigh-Ritz step of the
+    randomized fit is the exact truncated SVD of calib_fit (any q)."""
+    pp = S.host_probe_pairs(Np=40, m=10, d=16, L=2, rank=10, noise=0.3, seed=21)
+    Om = S.omega_matrix(16, 10, seed=21)
+    P0, Q0, s0, _ = O.calib_fit(pp["E_probe"], pp["G_probe"], 0.5, 4)
+    for q in (0, 1):
+        P, Q, s = O.calib_fit_rsvd(pp["E_probe"], pp["G_probe"], 0.5, 4, Om, q)
+        assert _rel(s, s0) < 1e-11
+        assert _rel(P, P0) < 1e-9 and _rel(Q, Q0) < 1e-9
+
+
+def test_rsvd_exact_on_a_fit_of_low_rank():
+    """Noise-free pairs: F_hat^T = (E^T E + beta I)^-1 E^T E M has the planted rank 3 < ell, so a
+    sketch of width 5 holds its whole range and the fit equals the exact one; the two
+    singular values beyond the rank are zero (zero rows of Q, zero columns of P)."""
+    pp = S.host_probe_pairs(Np=60, m=20, d=24, L=2, rank=3, noise=0.0, seed=22)
+    E = pp["E_probe"].astype(np.float64)
+    G = np.stack([E @ pp["M"][l] for l in range(2)])  # exact rank 3 (no fp32 storage rounding)
+    Om = S.omega_matrix(24, 5, seed=22)
+    P0, Q0, s0, _ = O.calib_fit(E, G, 0.2, 3)
+    P, Q, s = O.calib_fit_rsvd(E, G, 0.2, 5, Om, 0)
+    for l in range(2):
+        assert _rel(P[l, :, :3] @ Q[l, :3], P0[l] @ Q0[l]) < 1e-9
+    assert _rel(s[:, :3], s0) < 1e-10
+    assert np.all(s[:, 3:] == 0) and np.all(Q[:, 3:] == 0) and np.all(P[:, :, 3:] == 0)
+
+
+def test_rsvd_ritz_values_interlace_and_truncation_is_near_optimal():
+    """On a full-rank noisy fit: Ritz values of a projection lie below the singular values
+    (sigma_i(Q_Y^T F^T) <= sigma_i(F^T)); no rank-r map beats the truncated SVD in
+    Frobenius norm (Eckart-Young), and the randomized error approaches that optimum as q
+    grows; Q has orthonormal rows."""
+    pp = S.host_probe_pairs(Np=90, m=30, d=30, L=1, rank=6, noise=0.3, seed=23, e_scales=True)
+    Om = S.omega_matrix(30, 8, seed=23)
+    _, _, s_all, Fh = O.calib_fit(pp["E_probe"], pp["G_probe"], 0.4, 30)
+    r = 4
+    opt = float(np.sum(s_all[0, r:] ** 2))
+    errs = []
+    for q in range(4):
+        P, Q, s = O.calib_fit_rsvd(pp["E_probe"], pp["G_probe"], 0.4, r, Om, q)
+        assert np.all(s[0] <= s_all[0, :r] * (1 + 1e-12))
+        assert np.allclose(Q[0] @ Q[0].T, np.eye(r), atol=1e-12)
+        err = float(np.sum((Fh[0] - P[0] @ Q[0]) ** 2))
+        assert err >= opt * (1 - 1e-12)
+        errs.append(err)
+    assert errs[3] <= errs[0] and errs[3] <= opt * 1.01
+
+
+def test_rsvd_converges_to_the_truncation_on_a_gapped_spectrum():
+    """Planted rank r with little noise gives sigma_{r+1} << sigma_r; subspace iteration
+    then converges like (sigma_{ell+1} / sigma_r)^(2q+1), so two power iterations already
+    give the exact rank-r truncation to rounding."""
+    pp = S.host_probe_pairs(Np=120, m=40, d=48, L=2, rank=4, noise=0.02, seed=24, e_scales=True)
+    Om = S.omega_matrix(48, 8, seed=24)
+    P0, Q0, s0, _ = O.calib_fit(pp["E_probe"], pp["G_probe"], 0.1, 4)
+    P, Q, s = O.calib_fit_rsvd(pp["E_probe"], pp["G_probe"], 0.1, 4, Om, 2)
+    assert _rel(s, s0) < 1e-10
+    for l in range(2):
+        assert _rel(P[l] @ Q[l], P0[l] @ Q0[l]) < 1e-8
+    assert _rel(P, P0) < 1e-8 and _rel(Q, Q0) < 1e-8
+
+
 def test_linear_network_targets_equal_backprop_gradients():
     """Check 4: on an all-linear tokenwise network h_l = W_l h_{l-1}, z = W_u h_L, the true
     hidden-state gradient is g_l = (W_L ... W_{l+1})^T W_u^T eps (S3), exactly linear in the
