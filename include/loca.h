@@ -357,6 +357,42 @@ int loca_calib_fit(const float* E_probe, const float* G_probe, int64_t Np, int32
                    int32_t L, float beta, int32_t r, float* P, float* Q, float* sigma,
                    void* workspace, size_t workspace_bytes, void* stream);
 
+/*
+ * loca_calib_fit_rsvd — the rank-r feedback fit of loca_calib_fit for error spaces too wide
+ * to form and decompose F_hat_l^T (m x d), e.g. the paper's e = W_u^T eps with m = d (Eq. 5;
+ * Theorem "Feedback ridge solution" and Lemma "Rank-truncation error", S5).  The top-r SVD
+ * of F_hat_l^T = (E^T E + beta I_m)^-1 E^T G_l comes from randomized subspace iteration
+ * (Halko, Martinsson and Tropp, SIAM Review 53 (2011), Algorithm 4.4 with q power
+ * iterations, then Algorithm 5.1), which applies F_hat^T and F_hat only to ell vectors at a
+ * time through a Cholesky factor of E^T E + beta I (shared by all blocks; no inverse):
+ *
+ *   Y = F^T Omega, Q_Y = orth(Y); q times: Z = orth(F Q_Y), Q_Y = orth(F^T Z);
+ *   B = Q_Y^T F^T = U_B S V^T;  P_l = Q_Y U_B,r S_r (m x r),  Q_l = V_r^T (r x d).
+ *
+ * It equals loca_calib_fit's result when ell >= rank(F_hat_l^T); otherwise its error
+ * approaches the truncated SVD's as (sigma_{ell+1} / sigma_r)^(2q+1).  Same sign convention
+ * and zero threshold as loca_calib_fit.
+ *
+ * E_probe  Np x m float; G_probe  L x Np x d float; beta > 0
+ * Omega    d x ell float, device: the caller's Gaussian test matrix, used for every block
+ * 1 <= r <= ell <= 64, ell <= m <= 16384, ell <= d <= 16384, 0 <= q <= 16, 1 <= L <= 65535,
+ * 1 <= Np <= 4194240
+ * P        L x m x r float; Q  L x r x d float; sigma  L x r float or NULL
+ * Arithmetic: products with E and G_l from fp32 products summed in fp32 over 128-term runs
+ * and in fp64 across runs; Cholesky factor, triangular solves, orthonormal bases (Gram-Schmidt
+ * with re-orthogonalisation) and the Rayleigh-Ritz step in fp64.  Workspace (device, at least
+ * loca_calib_fit_rsvd_workspace_size bytes, 256-byte aligned) holds E^T E (m x m fp64,
+ * m rounded up to 64) and the ell-column blocks of every block; its contents are scratch.
+ * If E^T E + beta I is not positive definite in floating point, LOCA_ERR_NUMERIC is written
+ * to the device status word and P, Q and sigma are zero.
+ */
+int loca_calib_fit_rsvd_workspace_size(int64_t Np, int32_t m, int64_t d, int32_t L, int32_t r,
+                                       int32_t ell, size_t* bytes /* host */);
+int loca_calib_fit_rsvd(const float* E_probe, const float* G_probe, int64_t Np, int32_t m, int64_t d,
+                        int32_t L, float beta, int32_t r, int32_t ell, int32_t q, const float* Omega,
+                        float* P, float* Q, float* sigma, void* workspace, size_t workspace_bytes,
+                        void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -14,6 +14,7 @@
 //                  are treated as zero (zero Q row, zero P column).
 #include <cuda_runtime.h>
 
+#include "jacobi.cuh"
 #include "loca_internal.h"
 
 namespace loca {
@@ -177,65 +178,8 @@ __global__ void __launch_bounds__(256) k_calib_solve(const double* __restrict__ 
     if (a > b) sm.A[a][b] = sm.A[b][a];
   }
   __syncthreads();
-  // cyclic Jacobi sweeps (warp 0): rotation J in the (p, q) plane with tan(phi) = t chosen so that
-  // (J^T A J)_pq = 0, i.e. t^2 + 2 theta t - 1 = 0 with theta = (A_qq - A_pp) / (2 A_pq)
-  if (t < 32) {
-    double total = 0.0;
-    for (int a = 0; a < m; ++a)
-      for (int b = 0; b < m; ++b) total += sm.A[a][b] * sm.A[a][b];
-    for (int sweep = 0; sweep < 40; ++sweep) {
-      double off = 0.0;
-      for (int a = 0; a < m; ++a)
-        for (int b = a + 1; b < m; ++b) off += sm.A[a][b] * sm.A[a][b];
-      if (!(off > 1e-30 * total)) break;
-      for (int p = 0; p < m - 1; ++p) {
-        for (int q = p + 1; q < m; ++q) {
-          const double apq = sm.A[p][q];
-          if (fabs(apq) <= 1e-300) continue;
-          const double theta = (sm.A[q][q] - sm.A[p][p]) / (2.0 * apq);
-          const double tt = (theta >= 0 ? 1.0 : -1.0) / (fabs(theta) + sqrt(theta * theta + 1.0));
-          const double c = 1.0 / sqrt(tt * tt + 1.0), s = tt * c;
-          __syncwarp();
-          for (int k = t; k < m; k += 32) {
-            if (k != p && k != q) {
-              const double akp = sm.A[k][p], akq = sm.A[k][q];
-              sm.A[k][p] = c * akp - s * akq;
-              sm.A[k][q] = s * akp + c * akq;
-            }
-            const double vkp = sm.V[k][p], vkq = sm.V[k][q];
-            sm.V[k][p] = c * vkp - s * vkq;
-            sm.V[k][q] = s * vkp + c * vkq;
-          }
-          __syncwarp();
-          for (int k = t; k < m; k += 32) {
-            if (k != p && k != q) {
-              sm.A[p][k] = sm.A[k][p];
-              sm.A[q][k] = sm.A[k][q];
-            }
-          }
-          if (t == 0) {
-            sm.A[p][p] -= tt * apq;
-            sm.A[q][q] += tt * apq;
-            sm.A[p][q] = 0.0;
-            sm.A[q][p] = 0.0;
-          }
-          __syncwarp();
-        }
-      }
-    }
-    if (t == 0) {
-      // order eigenvalues descending (stable: lower index first on ties)
-      for (int i = 0; i < KM; ++i) sm.order[i] = i;
-      for (int i = 0; i < m; ++i) {
-        int best = i;
-        for (int k = i + 1; k < m; ++k)
-          if (sm.A[sm.order[k]][sm.order[k]] > sm.A[sm.order[best]][sm.order[best]]) best = k;
-        const int tmp = sm.order[i];
-        sm.order[i] = sm.order[best];
-        sm.order[best] = tmp;
-      }
-    }
-  }
+  // eigen-decomposition of F^T F^T^T by cyclic Jacobi rotations (warp 0)
+  if (t < 32) jacobi_eig_warp<KM>(sm.A, sm.V, sm.order, m, t);
   __syncthreads();
   const double lam1 = sm.A[sm.order[0]][sm.order[0]];
   const double s1 = lam1 > 0.0 ? sqrt(lam1) : 0.0;

@@ -617,4 +617,46 @@ int loca_calib_fit(const float* E_probe, const float* G_probe, int64_t Np, int32
   return LOCA_OK;
 }
 
+static int check_rsvd_shape(int64_t Np, int32_t m, int64_t d, int32_t L, int32_t r, int32_t ell) {
+  const int64_t wmax = calib_rsvd_max_width();
+  if (Np < 1 || Np > 65535LL * 64 || L < 1 || L > 65535 || r < 1 || ell < r || ell > calib_rsvd_max_ell() ||
+      m < ell || d < ell || m > wmax || d > wmax)
+    return fail(LOCA_ERR_SHAPE,
+                "need 1 <= Np <= 4194240, 1 <= L <= 65535, 1 <= r <= ell <= %d, ell <= m <= %lld, ell <= d <= %lld",
+                calib_rsvd_max_ell(), (long long)wmax, (long long)wmax);
+  return LOCA_OK;
+}
+
+int loca_calib_fit_rsvd_workspace_size(int64_t Np, int32_t m, int64_t d, int32_t L, int32_t r, int32_t ell,
+                                       size_t* bytes) {
+  if (!bytes) return fail(LOCA_ERR_INVALID_ARG, "bytes is NULL");
+  int rc = check_rsvd_shape(Np, m, d, L, r, ell);
+  if (rc != LOCA_OK) return rc;
+  *bytes = calib_rsvd_workspace_bytes(Np, m, d, L, ell, r);
+  return LOCA_OK;
+}
+
+int loca_calib_fit_rsvd(const float* E_probe, const float* G_probe, int64_t Np, int32_t m, int64_t d, int32_t L,
+                        float beta, int32_t r, int32_t ell, int32_t q, const float* Omega, float* P, float* Q,
+                        float* sigma, void* workspace, size_t workspace_bytes, void* stream) {
+  g_msg[0] = 0;
+  int rc = check_rsvd_shape(Np, m, d, L, r, ell);
+  if (rc != LOCA_OK) return rc;
+  if (q < 0 || q > 16) return fail(LOCA_ERR_INVALID_ARG, "need 0 <= q <= 16 power iterations");
+  if (!(beta > 0.f)) return fail(LOCA_ERR_INVALID_ARG, "beta must be > 0");
+  if (!E_probe || !G_probe || !Omega || !P || !Q)
+    return fail(LOCA_ERR_INVALID_ARG, "E_probe, G_probe, Omega, P and Q are required");
+  if (!aligned(E_probe, 4) || !aligned(G_probe, 4) || !aligned(Omega, 4) || !aligned(P, 4) || !aligned(Q, 4) ||
+      (sigma && !aligned(sigma, 4)))
+    return fail(LOCA_ERR_ALIGNMENT, "pointers must be 4-byte aligned");
+  rc = check_ws(workspace, workspace_bytes, calib_rsvd_workspace_bytes(Np, m, d, L, ell, r));
+  if (rc != LOCA_OK) return rc;
+  int32_t* status = device_status_word();
+  if (!status) return fail(LOCA_ERR_CUDA, "cannot resolve the device status word");
+  cudaError_t e = launch_calib_rsvd(E_probe, G_probe, Np, m, d, L, beta, r, ell, q, Omega, P, Q, sigma, workspace,
+                                    status, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "loca_calib_fit_rsvd launch");
+  return LOCA_OK;
+}
+
 }  // extern "C"

@@ -103,4 +103,12 @@ cudaError_t launch_calib_fit(const float* E_probe, const float* G_probe, int64_t
                              int64_t d, int L, float beta, int r, float* P, float* Q, float* sigma,
                              void* workspace, int32_t* status, cudaStream_t s);
 
+// ---- calibration for wide error spaces, randomized subspace iteration (calib_rsvd.cu)
+int calib_rsvd_max_ell();
+int64_t calib_rsvd_max_width();
+size_t calib_rsvd_workspace_bytes(int64_t Np, int64_t m, int64_t d, int L, int ell, int r);
+cudaError_t launch_calib_rsvd(const float* E_probe, const float* G_probe, int64_t Np, int64_t m, int64_t d, int L,
+                              float beta, int r, int ell, int q, const float* Omega, float* P, float* Q,
+                              float* sigma, void* workspace, int32_t* status, cudaStream_t s);
+
 }  // namespace loca

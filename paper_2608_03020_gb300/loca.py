@@ -68,6 +68,9 @@ SIGNATURES = [
     ("loca_calib_fit_workspace_size", ctypes.c_int, [_I64, _I32, _I64, _I32, _I32, ctypes.POINTER(_SZ)]),
     ("loca_calib_fit", ctypes.c_int,
      [_P, _P, _I64, _I32, _I64, _I32, _F, _I32, _P, _P, _P, _P, _SZ, _P]),
+    ("loca_calib_fit_rsvd_workspace_size", ctypes.c_int, [_I64, _I32, _I64, _I32, _I32, _I32, ctypes.POINTER(_SZ)]),
+    ("loca_calib_fit_rsvd", ctypes.c_int,
+     [_P, _P, _I64, _I32, _I64, _I32, _F, _I32, _I32, _I32, _P, _P, _P, _P, _P, _SZ, _P]),
 ]
 
 
@@ -487,6 +490,35 @@ def loca_calib_fit(E_probe, G_probe, beta, r, P, Q, sigma=None, workspace=None, 
     rc = lib().loca_calib_fit(_ptr(E_probe), _ptr(G_probe), Np, m, d, L, float(beta), r, _ptr(P), _ptr(Q),
                               _ptr(sigma), _ptr(ws), nbytes, _stream(stream))
     _check(rc, "loca_calib_fit")
+
+
+def calib_fit_rsvd_workspace_size(Np, m, d, L, r, ell) -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib().loca_calib_fit_rsvd_workspace_size(Np, m, d, L, r, ell, ctypes.byref(out)),
+           "loca_calib_fit_rsvd_workspace_size")
+    return out.value
+
+
+def loca_calib_fit_rsvd(E_probe, G_probe, beta, r, Omega, q, P, Q, sigma=None, workspace=None, stream=None):
+    """Rank-r feedback factors for wide error spaces by randomized subspace iteration:
+    ``Omega`` (d x ell) is the Gaussian test matrix, ``q`` the number of power iterations."""
+    _dev(E_probe, "E_probe", torch.float32, 2)
+    _dev(G_probe, "G_probe", torch.float32, 3)
+    _dev(Omega, "Omega", torch.float32, 2)
+    _dev(P, "P", torch.float32, 3)
+    _dev(Q, "Q", torch.float32, 3)
+    _dev(sigma, "sigma", torch.float32, 2)
+    Np, m = E_probe.shape
+    L, Np2, d = G_probe.shape
+    ell = Omega.shape[1]
+    if (Np2 != Np or Omega.shape[0] != d or tuple(P.shape) != (L, m, r) or tuple(Q.shape) != (L, r, d)
+            or (sigma is not None and tuple(sigma.shape) != (L, r))):
+        raise ValueError("shape mismatch among E_probe, G_probe, Omega, P, Q, sigma")
+    nbytes = calib_fit_rsvd_workspace_size(Np, m, d, L, r, ell)
+    ws = _workspace(nbytes, E_probe.device, workspace)
+    rc = lib().loca_calib_fit_rsvd(_ptr(E_probe), _ptr(G_probe), Np, m, d, L, float(beta), r, ell, int(q),
+                                   _ptr(Omega), _ptr(P), _ptr(Q), _ptr(sigma), _ptr(ws), nbytes, _stream(stream))
+    _check(rc, "loca_calib_fit_rsvd")
 
 
 class Pass:

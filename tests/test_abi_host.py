@@ -134,3 +134,32 @@ def test_validation_codes(L):
     # calibration: beta <= 0
     assert L.loca_calib_fit(fake, fake, 16, 4, 64, 2, ctypes.c_float(0.0), 2, fake, fake, None, fake,
                             1 << 20, None) == 1
+
+
+def test_calib_rsvd_validation(L):
+    fake = ctypes.c_void_p(256)
+    f = ctypes.c_float
+
+    def call(Np=64, m=128, d=96, Lb=2, beta=0.1, r=4, ell=8, q=1, omega=fake, ws_bytes=1 << 40):
+        return L.loca_calib_fit_rsvd(fake, fake, Np, m, d, Lb, f(beta), r, ell, q, omega, fake, fake, None, fake,
+                                     ws_bytes, None)
+
+    assert call(r=9) == 2            # r > ell
+    assert call(ell=65, r=4) == 2    # ell above the limit
+    assert call(m=4) == 2            # m < ell
+    assert call(d=4) == 2            # d < ell
+    assert call(m=16385) == 2        # m above the fp64 vector limit
+    assert call(Np=0) == 2
+    assert call(Np=65535 * 64 + 1) == 2
+    assert call(q=17) == 1
+    assert call(q=-1) == 1
+    assert call(beta=0.0) == 1
+    assert call(omega=None) == 1
+    assert call(ws_bytes=16) == 7    # workspace smaller than required
+    rc, n = _ws(L.loca_calib_fit_rsvd_workspace_size, 8192, 3584, 3584, 28, 16, 32)
+    # E^T E (m x m fp64) plus four ell-column blocks of every block (two m-wide, one d-wide,
+    # one Np-wide) dominate
+    n_cols = 28 * 32
+    floor = 8 * (3584 * 3584 + 2 * 3584 * n_cols + 3584 * n_cols + 8192 * n_cols)
+    assert rc == 0 and floor <= n < floor + (8 << 20) and n % 256 == 0
+    assert _ws(L.loca_calib_fit_rsvd_workspace_size, 8192, 3584, 3584, 28, 33, 32)[0] == 2
