@@ -16,10 +16,16 @@
 //   k_cr_potrf / k_cr_trsm / k_cr_syrk   right-looking blocked Cholesky (64 x 64 tiles, fp64);
 //                 the diagonal kernel also inverts its triangular tile, so the panel and the
 //                 diagonal steps of the solves are tile products
-//   k_cr_tsolve   blocked forward (L Y = W) and backward (L^T X = Y) substitution, fp64
-//   k_cr_orth     orthonormal basis of each block's ell columns: classical Gram-Schmidt with
-//                 one re-orthogonalisation (fp64); a column left with less than 1e-12 of its
-//                 norm after projection is dependent and set to zero
+//   k_cr_tsolve   blocked forward (L Y = W) and backward (L^T X = Y) substitution: fp64 for the
+//                 last F^T (which makes the final basis Q_Y) and for the Rayleigh-Ritz product
+//                 F Q_Y; fp32 (on an fp32 copy of the fp64 factor) inside the power iterations,
+//                 which only steer the subspace: an error there moves the starting vectors of
+//                 the next step, and the exact last F^T damps it by sigma_{ell+1} / sigma_r
+//   k_cr_vtv / k_cr_qr_factor / k_cr_qr_apply
+//                 orthonormal basis of each block's ell columns by Cholesky QR, applied twice
+//                 (fp64): S = V^T V over row chunks on all SMs, S = R^T R, V <- V R^-1.  A column
+//                 whose component outside the span of the earlier ones is below 1e-7 of its norm
+//                 is dependent and set to zero
 //   k_cr_btb / k_cr_ritz_eig / k_cr_ritz_out / k_cr_ritz_sign
 //                 Rayleigh-Ritz: B^T = F Q_Y (d x ell), B B^T = U_B S^2 U_B^T by cyclic Jacobi,
 //                 P_l = Q_Y U_B,r S_r, Q_l = S_r^-1 U_B,r^T B; the entry of largest magnitude of
@@ -37,7 +43,6 @@ namespace {
 constexpr int NB = 64;        // Cholesky / solve tile
 constexpr int NBP = NB + 1;   // padded shared-memory row (fp64: conflict-free column reads)
 constexpr int GM_BM = 64, GM_BN = 64, GM_BK = 32, GM_RUN = 4;
-constexpr int OR_THREADS = 256;
 constexpr int RZ_CH = 256;    // rows per chunk of the Rayleigh-Ritz kernels
 constexpr int kMaxEll = 64;
 constexpr int64_t kMaxWidth = 16384;  // m and d (fp64 vectors of one column in shared memory)
@@ -268,25 +273,24 @@ __global__ void __launch_bounds__(256) k_cr_syrk(double* __restrict__ K, int64_t
     }
 }
 
-// Blocked substitution on W (mp x n, fp64, in place), one step per launch, on column tiles of
-// TW columns (blockIdx.y):
+// Blocked substitution on W (mp x n, in place; T = double or float), one step per launch, on
+// column tiles of TW columns (blockIdx.y):
 //   MODE 0  forward diagonal:  W_ib = L(ib, ib)^-1 W_ib
 //   MODE 1  forward update:    W_tb -= L(tb, ib) W_ib,    tb = ib + 1 + blockIdx.x
 //   MODE 2  backward diagonal: W_ib = L(ib, ib)^-T W_ib
 //   MODE 3  backward update:   W_tb -= L(ib, tb)^T W_ib,  tb = blockIdx.x < ib
-template <int MODE, int TW>
-__global__ void __launch_bounds__(256) k_cr_tsolve(const double* __restrict__ K, int64_t mp,
-                                                  const double* __restrict__ Dinv, double* __restrict__ W,
-                                                  int64_t n, int ib, const int32_t* flag) {
+template <typename T, int MODE, int TW>
+__global__ void __launch_bounds__(256) k_cr_tsolve(const T* __restrict__ K, int64_t mp, const T* __restrict__ Dinv,
+                                                  T* __restrict__ W, int64_t n, int ib, const int32_t* flag) {
   extern __shared__ __align__(16) unsigned char cr_smem[];
-  double(*Mt)[NBP] = reinterpret_cast<double(*)[NBP]>(cr_smem);
-  double(*Rt)[NBP] = reinterpret_cast<double(*)[NBP]>(cr_smem + sizeof(double) * NB * NBP);
+  T(*Mt)[NBP] = reinterpret_cast<T(*)[NBP]>(cr_smem);
+  T(*Rt)[NBP] = reinterpret_cast<T(*)[NBP]>(cr_smem + sizeof(T) * NB * NBP);
   if (failed(flag)) return;
   constexpr bool kTrans = (MODE >= 2);
   constexpr bool kSub = (MODE == 1 || MODE == 3);
   constexpr int QN = TW / 16;
   int tb;
-  const double* mat;
+  const T* mat;
   int64_t ldm;
   if (MODE == 0 || MODE == 2) {
     tb = ib;
@@ -302,19 +306,23 @@ __global__ void __launch_bounds__(256) k_cr_tsolve(const double* __restrict__ K,
     ldm = mp;
   }
   const int64_t c0 = int64_t(blockIdx.y) * TW;
-  load_tile(Mt, mat, ldm);
+  for (int e = threadIdx.x; e < NB * NB; e += 256) Mt[e / NB][e % NB] = mat[int64_t(e / NB) * ldm + e % NB];
   for (int e = threadIdx.x; e < NB * TW; e += 256) {
     const int u = e / TW, c = e % TW;
-    Rt[u][c] = (c0 + c < n) ? W[(int64_t(ib) * NB + u) * n + c0 + c] : 0.0;
+    Rt[u][c] = (c0 + c < n) ? W[(int64_t(ib) * NB + u) * n + c0 + c] : T(0);
   }
   __syncthreads();
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-  double acc[4][QN] = {};
+  T acc[4][QN];
+#pragma unroll
+  for (int p = 0; p < 4; ++p)
+#pragma unroll
+    for (int q = 0; q < QN; ++q) acc[p][q] = T(0);
   for (int u = 0; u < NB; ++u) {
 #pragma unroll
     for (int p = 0; p < 4; ++p) {
       const int r = ty + 16 * p;
-      const double a = kTrans ? Mt[u][r] : Mt[r][u];
+      const T a = kTrans ? Mt[u][r] : Mt[r][u];
 #pragma unroll
       for (int q = 0; q < QN; ++q) acc[p][q] = fma(a, Rt[u][tx + 16 * q], acc[p][q]);
     }
@@ -326,89 +334,133 @@ __global__ void __launch_bounds__(256) k_cr_tsolve(const double* __restrict__ K,
     for (int q = 0; q < QN; ++q) {
       const int64_t c = c0 + tx + 16 * q;
       if (c >= n) continue;
-      double* dst = W + (int64_t(tb) * NB + ty + 16 * p) * n + c;
+      T* dst = W + (int64_t(tb) * NB + ty + 16 * p) * n + c;
       *dst = kSub ? (*dst - acc[p][q]) : acc[p][q];
     }
 }
 
-__device__ __forceinline__ double warp_sum(double v) {
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-  return v;
+template <typename TI, typename TO>
+__global__ void k_cr_cvt(const TI* __restrict__ x, TO* __restrict__ y, int64_t count) {
+  for (int64_t e = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; e < count; e += int64_t(gridDim.x) * blockDim.x)
+    y[e] = TO(x[e]);
 }
 
-// Sum over the CTA in a fixed order (warp shuffles, then the warps' sums in index order).
-__device__ double block_sum(double v, double* scratch) {
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  v = warp_sum(v);
-  __syncthreads();
-  if (lane == 0) scratch[wid] = v;
-  __syncthreads();
-  double s = 0.0;
-  for (int w = 0; w < nw; ++w) s += scratch[w];
-  return s;
-}
+constexpr int QR_STAGE = 64;   // rows staged at a time by k_cr_vtv
+constexpr int QR_CHUNK = 256;  // rows per CTA of k_cr_vtv / k_cr_qr_apply
 
-// Orthonormal basis of block l's ell columns of V (rows x n, columns l ell .. l ell + ell - 1),
-// in place: classical Gram-Schmidt, each column projected out twice.
+// Partial Gram matrices of block l's ell columns of V (rows x n, columns l ell ..):
+// part[l][chunk] (ELLP x ELLP, zero outside ell x ell) = sum over the chunk's rows of v v^T.
 template <int ELLP>
-__global__ void __launch_bounds__(OR_THREADS) k_cr_orth(double* __restrict__ V, int64_t rows, int64_t n, int ell) {
-  extern __shared__ __align__(16) unsigned char cr_smem[];
-  double* vs = reinterpret_cast<double*>(cr_smem);
-  __shared__ double red[ELLP][OR_THREADS / 32];
-  __shared__ double hs[ELLP];
-  __shared__ double scratch[OR_THREADS / 32];
-  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-  double* Vb = V + int64_t(blockIdx.x) * ell;
-  for (int c = 0; c < ell; ++c) {
-    double s2 = 0.0;
-    for (int64_t r = tid; r < rows; r += OR_THREADS) {
-      const double x = Vb[r * n + c];
-      vs[r] = x;
-      s2 = fma(x, x, s2);
-    }
-    const double n0 = sqrt(block_sum(s2, scratch));
-    for (int pass = 0; pass < 2 && c > 0; ++pass) {
-      double h[ELLP];
+__global__ void __launch_bounds__(256) k_cr_vtv(const double* __restrict__ V, int64_t rows, int64_t n, int ell,
+                                               int nch, double* __restrict__ part) {
+  __shared__ double Vs[QR_STAGE][ELLP + 1];
+  constexpr int EPT = (ELLP * ELLP + 255) / 256;
+  const int ch = blockIdx.x, l = blockIdx.y, tid = threadIdx.x;
+  const int64_t r0 = int64_t(ch) * QR_CHUNK;
+  const int64_t r1 = (r0 + QR_CHUNK < rows) ? r0 + QR_CHUNK : rows;
+  double acc[EPT];
 #pragma unroll
-      for (int u = 0; u < ELLP; ++u) h[u] = 0.0;
-      for (int64_t r = tid; r < rows; r += OR_THREADS) {
-        const double vr = vs[r];
-        const double* row = Vb + r * n;
-#pragma unroll
-        for (int u = 0; u < ELLP; ++u)
-          if (u < c) h[u] = fma(row[u], vr, h[u]);
-      }
-#pragma unroll
-      for (int u = 0; u < ELLP; ++u)
-        if (u < c) {
-          const double x = warp_sum(h[u]);
-          if (lane == 0) red[u][wid] = x;
-        }
-      __syncthreads();
-      if (tid < c) {
-        double s = 0.0;
-        for (int w = 0; w < OR_THREADS / 32; ++w) s += red[tid][w];
-        hs[tid] = s;
-      }
-      __syncthreads();
-      for (int64_t r = tid; r < rows; r += OR_THREADS) {
-        double a = vs[r];
-        const double* row = Vb + r * n;
-#pragma unroll
-        for (int u = 0; u < ELLP; ++u)
-          if (u < c) a = fma(-hs[u], row[u], a);
-        vs[r] = a;
-      }
-      __syncthreads();
-    }
-    s2 = 0.0;
-    for (int64_t r = tid; r < rows; r += OR_THREADS) s2 = fma(vs[r], vs[r], s2);
-    const double nrm = sqrt(block_sum(s2, scratch));
-    const double scale = (n0 > 0.0 && nrm > 1e-12 * n0) ? 1.0 / nrm : 0.0;
-    for (int64_t r = tid; r < rows; r += OR_THREADS) Vb[r * n + c] = vs[r] * scale;
+  for (int k = 0; k < EPT; ++k) acc[k] = 0.0;
+  for (int64_t rs = r0; rs < r1; rs += QR_STAGE) {
     __syncthreads();
+    for (int e = tid; e < QR_STAGE * ELLP; e += 256) {
+      const int rr = e / ELLP, c = e % ELLP;
+      Vs[rr][c] = (rs + rr < r1 && c < ell) ? V[(rs + rr) * n + int64_t(l) * ell + c] : 0.0;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < EPT; ++k) {
+      const int e = tid + 256 * k;
+      if (e < ELLP * ELLP) {
+        const int a = e / ELLP, b = e % ELLP;
+        double sacc = acc[k];
+        for (int rr = 0; rr < QR_STAGE; ++rr) sacc = fma(Vs[rr][a], Vs[rr][b], sacc);
+        acc[k] = sacc;
+      }
+    }
   }
+  double* out = part + (int64_t(l) * nch + ch) * ELLP * ELLP;
+#pragma unroll
+  for (int k = 0; k < EPT; ++k) {
+    const int e = tid + 256 * k;
+    if (e < ELLP * ELLP) out[e] = acc[k];
+  }
+}
+
+// Per block: S = sum of the partials (fixed order), S = Lc Lc^T by Cholesky (warp 0) with
+// dependent columns (new component below 1e-7 of the column's norm: pivot <= 1e-14 S_cc) given
+// a zero column in Lc.  Writes Lc with its diagonal replaced by the reciprocals (0 when
+// dependent) to fac[l] (ELLP x ELLP).
+template <int ELLP>
+__global__ void __launch_bounds__(256) k_cr_qr_factor(const double* __restrict__ part, int nch, int ell,
+                                                     double* __restrict__ fac) {
+  extern __shared__ __align__(16) unsigned char cr_smem[];
+  double(*S)[ELLP + 1] = reinterpret_cast<double(*)[ELLP + 1]>(cr_smem);
+  double(*Lc)[ELLP + 1] = reinterpret_cast<double(*)[ELLP + 1]>(cr_smem + sizeof(double) * ELLP * (ELLP + 1));
+  const int l = blockIdx.x, tid = threadIdx.x;
+  for (int e = tid; e < ELLP * ELLP; e += blockDim.x) {
+    double v = 0.0;
+    for (int ch = 0; ch < nch; ++ch) v += part[(int64_t(l) * nch + ch) * ELLP * ELLP + e];
+    S[e / ELLP][e % ELLP] = v;
+    Lc[e / ELLP][e % ELLP] = 0.0;
+  }
+  __syncthreads();
+  if (tid < 32) {
+    const int lane = tid;
+    for (int c = 0; c < ell; ++c) {
+      double dsum = S[c][c];
+      for (int u = 0; u < c; ++u) dsum -= Lc[c][u] * Lc[c][u];
+      const bool dep = !(S[c][c] > 0.0) || !(dsum > 1e-14 * S[c][c]);
+      const double lcc = dep ? 0.0 : sqrt(dsum);
+      __syncwarp();
+      for (int j = c + 1 + lane; j < ell; j += 32) {
+        double v = 0.0;
+        if (!dep) {
+          v = S[j][c];
+          for (int u = 0; u < c; ++u) v -= Lc[j][u] * Lc[c][u];
+          v /= lcc;
+        }
+        Lc[j][c] = v;
+      }
+      if (lane == 0) Lc[c][c] = lcc;
+      __syncwarp();
+    }
+  }
+  __syncthreads();
+  double* F = fac + int64_t(l) * ELLP * ELLP;
+  for (int e = tid; e < ELLP * ELLP; e += blockDim.x) {
+    const int a = e / ELLP, b = e % ELLP;
+    double v = (b < a) ? Lc[a][b] : 0.0;
+    if (a == b) v = (Lc[a][a] > 0.0) ? 1.0 / Lc[a][a] : 0.0;
+    F[e] = v;
+  }
+}
+
+// Per row v of block l's columns: q = v R^-1 with R = Lc^T, i.e. Lc q^T = v^T by forward
+// substitution (dependent columns give q_c = 0).
+template <int ELLP>
+__global__ void __launch_bounds__(QR_CHUNK) k_cr_qr_apply(double* __restrict__ V, int64_t rows, int64_t n, int ell,
+                                                         const double* __restrict__ fac) {
+  __shared__ double F[ELLP][ELLP + 1];
+  const int l = blockIdx.y, tid = threadIdx.x;
+  for (int e = tid; e < ELLP * ELLP; e += QR_CHUNK) F[e / ELLP][e % ELLP] = fac[int64_t(l) * ELLP * ELLP + e];
+  __syncthreads();
+  const int64_t rrow = int64_t(blockIdx.x) * QR_CHUNK + tid;
+  if (rrow >= rows) return;
+  double* v = V + rrow * n + int64_t(l) * ell;
+  double x[ELLP];
+#pragma unroll
+  for (int c = 0; c < ELLP; ++c) x[c] = (c < ell) ? v[c] : 0.0;
+#pragma unroll
+  for (int c = 0; c < ELLP; ++c) {
+    double a = x[c];
+#pragma unroll
+    for (int u = 0; u < c; ++u) a = fma(-F[c][u], x[u], a);
+    x[c] = a * F[c][c];
+  }
+#pragma unroll
+  for (int c = 0; c < ELLP; ++c)
+    if (c < ell) v[c] = x[c];
 }
 
 // Partial Gram matrices of B^T (d x ell per block): part[l][chunk][a][b] = sum over the chunk's
@@ -574,7 +626,7 @@ __global__ void __launch_bounds__(256) k_cr_ritz_sign(float* __restrict__ P, flo
 }
 
 struct RsvdWs {
-  size_t K, Dinv, Ym, Wm, Zd, Tn, part, Ur, sig, amv, ami, flag, total;
+  size_t K, Dinv, Kf, Dinvf, Ym, Wm, Wf, Zd, Tn, qrpart, qrfac, part, Ur, sig, amv, ami, flag, total;
 };
 
 RsvdWs rsvd_ws(int64_t Np, int64_t m, int64_t d, int L, int ell, int r) {
@@ -590,12 +642,19 @@ RsvdWs rsvd_ws(int64_t Np, int64_t m, int64_t d, int L, int ell, int r) {
     o += align256(bytes);
     return at;
   };
+  const int64_t ellp = ell <= 16 ? 16 : (ell <= 32 ? 32 : 64);
+  const int64_t nchqr = ((m > d ? m : d) + QR_CHUNK - 1) / QR_CHUNK;
   w.K = take(sizeof(double) * mp * mp);
   w.Dinv = take(sizeof(double) * nb * NB * NB);
+  w.Kf = take(sizeof(float) * mp * mp);
+  w.Dinvf = take(sizeof(float) * nb * NB * NB);
   w.Ym = take(sizeof(double) * mp * n);
   w.Wm = take(sizeof(double) * mp * n);
+  w.Wf = take(sizeof(float) * mp * n);
   w.Zd = take(sizeof(double) * d * n);
   w.Tn = take(sizeof(double) * Np * n);
+  w.qrpart = take(sizeof(double) * L * nchqr * ellp * ellp);
+  w.qrfac = take(sizeof(double) * L * ellp * ellp);
   w.part = take(sizeof(double) * L * nchd * ell * ell);
   w.Ur = take(sizeof(double) * L * ell * r);
   w.sig = take(sizeof(double) * L * r);
@@ -615,43 +674,60 @@ cudaError_t gemm(const float* A, int64_t lda, int64_t sA, const TB* B, int64_t l
   return cudaGetLastError();
 }
 
-// W (mp x n) <- K^-1 W with K = L L^T (forward, then backward substitution).
-cudaError_t solve(const double* K, int64_t mp, const double* Dinv, double* W, int64_t n, const int32_t* flag,
-                  cudaStream_t s) {
+// W (mp x n) <- K^-1 W with K = L L^T (forward, then backward substitution), in T.
+template <typename T>
+cudaError_t solve(const T* K, int64_t mp, const T* Dinv, T* W, int64_t n, const int32_t* flag, cudaStream_t s) {
   const int nb = int(mp / NB);
+  const size_t smem = sizeof(T) * 2 * NB * NBP;
   const unsigned ct16 = unsigned((n + 15) / 16), ct64 = unsigned((n + 63) / 64);
   for (int ib = 0; ib < nb; ++ib) {
-    k_cr_tsolve<0, 16><<<dim3(1, ct16), 256, kTileSmem, s>>>(K, mp, Dinv, W, n, ib, flag);
-    if (ib + 1 < nb) k_cr_tsolve<1, 64><<<dim3(unsigned(nb - 1 - ib), ct64), 256, kTileSmem, s>>>(K, mp, Dinv, W, n, ib, flag);
+    k_cr_tsolve<T, 0, 16><<<dim3(1, ct16), 256, smem, s>>>(K, mp, Dinv, W, n, ib, flag);
+    if (ib + 1 < nb)
+      k_cr_tsolve<T, 1, 64><<<dim3(unsigned(nb - 1 - ib), ct64), 256, smem, s>>>(K, mp, Dinv, W, n, ib, flag);
   }
   for (int ib = nb - 1; ib >= 0; --ib) {
-    k_cr_tsolve<2, 16><<<dim3(1, ct16), 256, kTileSmem, s>>>(K, mp, Dinv, W, n, ib, flag);
-    if (ib > 0) k_cr_tsolve<3, 64><<<dim3(unsigned(ib), ct64), 256, kTileSmem, s>>>(K, mp, Dinv, W, n, ib, flag);
+    k_cr_tsolve<T, 2, 16><<<dim3(1, ct16), 256, smem, s>>>(K, mp, Dinv, W, n, ib, flag);
+    if (ib > 0) k_cr_tsolve<T, 3, 64><<<dim3(unsigned(ib), ct64), 256, smem, s>>>(K, mp, Dinv, W, n, ib, flag);
   }
   return cudaGetLastError();
 }
 
-template <int ELLP>
-cudaError_t orth(double* V, int64_t rows, int64_t n, int ell, int L, cudaStream_t s) {
-  k_cr_orth<ELLP><<<L, OR_THREADS, size_t(rows) * sizeof(double), s>>>(V, rows, n, ell);
+template <typename TI, typename TO>
+cudaError_t cvt(const TI* x, TO* y, int64_t count, cudaStream_t s) {
+  k_cr_cvt<TI, TO><<<2 * sm_count(), 256, 0, s>>>(x, y, count);
   return cudaGetLastError();
 }
 
-cudaError_t set_smem_attributes(int64_t rows_max) {
-  static const void* fns[] = {
-      reinterpret_cast<const void*>(k_cr_potrf),          reinterpret_cast<const void*>(k_cr_trsm),
-      reinterpret_cast<const void*>(k_cr_syrk),           reinterpret_cast<const void*>(k_cr_tsolve<0, 16>),
-      reinterpret_cast<const void*>(k_cr_tsolve<1, 64>),  reinterpret_cast<const void*>(k_cr_tsolve<2, 16>),
-      reinterpret_cast<const void*>(k_cr_tsolve<3, 64>)};
-  for (const void* f : fns) {
+// Orthonormal basis of every block's ell columns of V (rows x n), in place: Cholesky QR twice.
+template <int ELLP>
+cudaError_t orth(double* V, int64_t rows, int64_t n, int ell, int L, double* qrpart, double* qrfac, cudaStream_t s) {
+  const int nch = int((rows + QR_CHUNK - 1) / QR_CHUNK);
+  const size_t fsmem = 2 * sizeof(double) * ELLP * (ELLP + 1);
+  for (int pass = 0; pass < 2; ++pass) {
+    k_cr_vtv<ELLP><<<dim3(unsigned(nch), unsigned(L)), 256, 0, s>>>(V, rows, n, ell, nch, qrpart);
+    k_cr_qr_factor<ELLP><<<L, 256, fsmem, s>>>(qrpart, nch, ell, qrfac);
+    k_cr_qr_apply<ELLP><<<dim3(unsigned(nch), unsigned(L)), QR_CHUNK, 0, s>>>(V, rows, n, ell, qrfac);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t set_smem_attributes() {
+  static const void* fns64[] = {
+      reinterpret_cast<const void*>(k_cr_potrf), reinterpret_cast<const void*>(k_cr_trsm),
+      reinterpret_cast<const void*>(k_cr_syrk), reinterpret_cast<const void*>(k_cr_tsolve<double, 0, 16>),
+      reinterpret_cast<const void*>(k_cr_tsolve<double, 1, 64>),
+      reinterpret_cast<const void*>(k_cr_tsolve<double, 2, 16>),
+      reinterpret_cast<const void*>(k_cr_tsolve<double, 3, 64>)};
+  for (const void* f : fns64) {
     cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kTileSmem));
     if (e != cudaSuccess) return e;
   }
-  const int orth_smem = int(rows_max * sizeof(double));
-  const void* ofns[] = {reinterpret_cast<const void*>(k_cr_orth<16>), reinterpret_cast<const void*>(k_cr_orth<32>),
-                        reinterpret_cast<const void*>(k_cr_orth<64>)};
-  for (const void* f : ofns) {
-    cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, orth_smem);
+  static const void* fqr[] = {reinterpret_cast<const void*>(k_cr_qr_factor<16>),
+                              reinterpret_cast<const void*>(k_cr_qr_factor<32>),
+                              reinterpret_cast<const void*>(k_cr_qr_factor<64>)};
+  for (const void* f : fqr) {
+    cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         int(2 * sizeof(double) * 64 * 65));
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
@@ -667,12 +743,17 @@ cudaError_t rsvd_t(const float* E, const float* G, int64_t Np, int64_t m, int64_
   const int64_t n = int64_t(L) * ell;
   double* K = reinterpret_cast<double*>(ws + w.K);
   double* Dinv = reinterpret_cast<double*>(ws + w.Dinv);
+  float* Kf = reinterpret_cast<float*>(ws + w.Kf);
+  float* Dinvf = reinterpret_cast<float*>(ws + w.Dinvf);
   double* Ym = reinterpret_cast<double*>(ws + w.Ym);
   double* Wm = reinterpret_cast<double*>(ws + w.Wm);
+  float* Wf = reinterpret_cast<float*>(ws + w.Wf);
   double* Zd = reinterpret_cast<double*>(ws + w.Zd);
   double* Tn = reinterpret_cast<double*>(ws + w.Tn);
+  double* qrpart = reinterpret_cast<double*>(ws + w.qrpart);
+  double* qrfac = reinterpret_cast<double*>(ws + w.qrfac);
   int32_t* flag = reinterpret_cast<int32_t*>(ws + w.flag);
-  cudaError_t e = set_smem_attributes(m > d ? m : d);
+  cudaError_t e = set_smem_attributes();
   if (e != cudaSuccess) return e;
 #define CR_TRY(x)              \
   do {                         \
@@ -694,31 +775,43 @@ cudaError_t rsvd_t(const float* E, const float* G, int64_t Np, int64_t m, int64_
     }
     CR_TRY(cudaGetLastError());
   }
+  if (q > 0) {
+    CR_TRY((cvt<double, float>(K, Kf, mp * mp, s)));
+    CR_TRY((cvt<double, float>(Dinv, Dinvf, int64_t(nb) * NB * NB, s)));
+  }
+  // K^-1 V in place on V (mp x n, fp64): exact (fp64 factor) or inside the power iterations
+  // (fp32 factor on an fp32 copy)
+  auto kinv = [&](double* V, bool exact) -> cudaError_t {
+    if (exact) return solve<double>(K, mp, Dinv, V, n, flag, s);
+    CR_TRY((cvt<double, float>(V, Wf, mp * n, s)));
+    CR_TRY(solve<float>(Kf, mp, Dinvf, Wf, n, flag, s));
+    return cvt<float, double>(Wf, V, mp * n, s);
+  };
   // Ym = F^T X for every block, X (d x ell per block) at column offset l ell of Xd (ld ldx, block
   // stride sx); Tn = G_l X, Ym = K^-1 E^T Tn
-  auto apply_Ft = [&](auto* Xd, int64_t ldx, int64_t sx) -> cudaError_t {
+  auto apply_Ft = [&](auto* Xd, int64_t ldx, int64_t sx, bool exact) -> cudaError_t {
     using TX = std::remove_const_t<std::remove_pointer_t<decltype(Xd)>>;
     CR_TRY((gemm<false, TX>(G, d, Np * d, Xd, ldx, sx, Tn, n, ell, Np, ell, d, L, 0, s)));
     CR_TRY((gemm<true, double>(E, m, 0, Tn, n, 0, Ym, n, 0, m, n, Np, 1, 0, s)));
-    return solve(K, mp, Dinv, Ym, n, flag, s);
+    return kinv(Ym, exact);
   };
   // Zd = F Y for every block, Y = Vm (mp x n, overwritten by K^-1 Y): Tn = E K^-1 Y, Zd = G_l^T Tn
-  auto apply_F = [&](double* Vm) -> cudaError_t {
-    CR_TRY(solve(K, mp, Dinv, Vm, n, flag, s));
+  auto apply_F = [&](double* Vm, bool exact) -> cudaError_t {
+    CR_TRY(kinv(Vm, exact));
     CR_TRY((gemm<false, double>(E, m, 0, Vm, n, 0, Tn, n, 0, Np, n, m, 1, 0, s)));
     return gemm<true, double>(G, d, Np * d, Tn, n, ell, Zd, n, ell, d, ell, Np, L, 0, s);
   };
-  CR_TRY(apply_Ft(Omega, int64_t(ell), int64_t(0)));
-  CR_TRY(orth<ELLP>(Ym, m, n, ell, L, s));
+  CR_TRY(apply_Ft(Omega, int64_t(ell), int64_t(0), q == 0));
+  CR_TRY(orth<ELLP>(Ym, m, n, ell, L, qrpart, qrfac, s));
   for (int it = 0; it < q; ++it) {
-    CR_TRY(apply_F(Ym));
-    CR_TRY(orth<ELLP>(Zd, d, n, ell, L, s));
-    CR_TRY(apply_Ft(static_cast<const double*>(Zd), n, int64_t(ell)));
-    CR_TRY(orth<ELLP>(Ym, m, n, ell, L, s));
+    CR_TRY(apply_F(Ym, false));
+    CR_TRY(orth<ELLP>(Zd, d, n, ell, L, qrpart, qrfac, s));
+    CR_TRY(apply_Ft(static_cast<const double*>(Zd), n, int64_t(ell), it == q - 1));
+    CR_TRY(orth<ELLP>(Ym, m, n, ell, L, qrpart, qrfac, s));
   }
   // Rayleigh-Ritz: B^T = F Q_Y
   CR_TRY(cudaMemcpyAsync(Wm, Ym, sizeof(double) * mp * n, cudaMemcpyDeviceToDevice, s));
-  CR_TRY(apply_F(Wm));
+  CR_TRY(apply_F(Wm, true));
   const int nchd = int((d + RZ_CH - 1) / RZ_CH);
   const int nchq = int(((m > d ? m : d) + RZ_CH - 1) / RZ_CH);
   double* part = reinterpret_cast<double*>(ws + w.part);

@@ -157,9 +157,9 @@ def test_calib_rsvd_validation(L):
     assert call(omega=None) == 1
     assert call(ws_bytes=16) == 7    # workspace smaller than required
     rc, n = _ws(L.loca_calib_fit_rsvd_workspace_size, 8192, 3584, 3584, 28, 16, 32)
-    # E^T E (m x m fp64) plus four ell-column blocks of every block (two m-wide, one d-wide,
-    # one Np-wide) dominate
+    # E^T E (m x m fp64) and its fp32 copy, plus the ell-column blocks of every block (two
+    # m-wide fp64 and one fp32, one d-wide, one Np-wide) dominate
     n_cols = 28 * 32
-    floor = 8 * (3584 * 3584 + 2 * 3584 * n_cols + 3584 * n_cols + 8192 * n_cols)
-    assert rc == 0 and floor <= n < floor + (8 << 20) and n % 256 == 0
+    floor = 12 * 3584 * 3584 + 8 * (2 * 3584 * n_cols + 3584 * n_cols + 8192 * n_cols) + 4 * 3584 * n_cols
+    assert rc == 0 and floor <= n < floor + (16 << 20) and n % 256 == 0
     assert _ws(L.loca_calib_fit_rsvd_workspace_size, 8192, 3584, 3584, 28, 33, 32)[0] == 2
