@@ -178,8 +178,8 @@ __global__ void __launch_bounds__(256) k_calib_solve(const double* __restrict__ 
     if (a > b) sm.A[a][b] = sm.A[b][a];
   }
   __syncthreads();
-  // eigen-decomposition of F^T F^T^T by cyclic Jacobi rotations (warp 0)
-  if (t < 32) jacobi_eig_warp<KM>(sm.A, sm.V, sm.order, m, t);
+  // eigen-decomposition of F^T F^T^T by Jacobi rotations (whole block)
+  jacobi_eig_block<KM>(sm.A, sm.V, sm.order, m);
   __syncthreads();
   const double lam1 = sm.A[sm.order[0]][sm.order[0]];
   const double s1 = lam1 > 0.0 ? sqrt(lam1) : 0.0;

@@ -10,8 +10,8 @@
 //
 // All L blocks share K, so every solve runs on the ell columns of all blocks at once.
 //
-//   k_cr_gemm     fp32 operands, fp32 products summed in fp32 over 128-step runs and in fp64
-//                 across runs (the products with E and G_l; K itself, lower tiles only)
+//   k_cr_gemm     fp32 operands, products summed in fp32 over 32 terms, those sums in fp32 over
+//                 16 and in fp64 beyond (the products with E and G_l; K itself, lower tiles only)
 //   k_cr_pad      K + beta I, padded to a multiple of 64 with an identity block
 //   k_cr_potrf / k_cr_trsm / k_cr_syrk   right-looking blocked Cholesky (64 x 64 tiles, fp64);
 //                 the diagonal kernel also inverts its triangular tile, so the panel and the
@@ -32,8 +32,6 @@
 //                 each Q_l row is made positive; singular values <= 1e-12 sigma_1 count as zero.
 #include <cuda_runtime.h>
 
-#include <type_traits>
-
 #include "jacobi.cuh"
 #include "loca_internal.h"
 
@@ -42,7 +40,7 @@ namespace {
 
 constexpr int NB = 64;        // Cholesky / solve tile
 constexpr int NBP = NB + 1;   // padded shared-memory row (fp64: conflict-free column reads)
-constexpr int GM_BM = 64, GM_BN = 64, GM_BK = 32, GM_RUN = 4;
+constexpr int GM_BM = 64, GM_BN = 64, GM_BK = 32, GM_RUN = 16;
 constexpr int RZ_CH = 256;    // rows per chunk of the Rayleigh-Ritz kernels
 constexpr int kMaxEll = 64;
 constexpr int64_t kMaxWidth = 16384;  // m and d (fp64 vectors of one column in shared memory)
@@ -51,12 +49,13 @@ constexpr size_t kTileSmem = sizeof(double) * 2 * NB * NBP;
 __device__ __forceinline__ bool failed(const int32_t* flag) { return *reinterpret_cast<const volatile int32_t*>(flag) != 0; }
 
 // C_b[i][j] = sum_t A_b(i, t) B_b(t, j);  A_b(i, t) = A[t lda + i] (AT) or A[i lda + t];
-// B_b(t, j) = B[t ldb + j]; batch b = blockIdx.z with element strides sA, sB, sC.
-template <bool AT, typename TB>
+// B_b(t, j) = B[t ldb + j]; batch b = blockIdx.z with element strides sA, sB, sC.  Products are
+// summed in fp32 over 32 terms, those sums in fp32 over 16 (512 terms), and those in fp64.
+template <bool AT, typename TC>
 __global__ void __launch_bounds__(256) k_cr_gemm(const float* __restrict__ A, int64_t lda, int64_t sA,
-                                                const TB* __restrict__ B, int64_t ldb, int64_t sB,
-                                                double* __restrict__ C, int64_t ldc, int64_t sC, int64_t M,
-                                                int64_t N, int64_t Kc, int lower_only) {
+                                                const float* __restrict__ B, int64_t ldb, int64_t sB,
+                                                TC* __restrict__ C, int64_t ldc, int64_t sC, int64_t M, int64_t N,
+                                                int64_t Kc, int lower_only) {
   __shared__ __align__(16) float As[GM_BK][GM_BM + 4];
   __shared__ __align__(16) float Bs[GM_BK][GM_BN + 4];
   const int64_t i0 = int64_t(blockIdx.y) * GM_BM, j0 = int64_t(blockIdx.x) * GM_BN;
@@ -67,13 +66,13 @@ __global__ void __launch_bounds__(256) k_cr_gemm(const float* __restrict__ A, in
   C += b * sC;
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
   double acc[4][4];
-  float part[4][4];
+  float run_sum[4][4];
 #pragma unroll
   for (int p = 0; p < 4; ++p)
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       acc[p][q] = 0.0;
-      part[p][q] = 0.f;
+      run_sum[p][q] = 0.f;
     }
   int run = 0;
   for (int64_t t0 = 0; t0 < Kc; t0 += GM_BK) {
@@ -93,9 +92,14 @@ __global__ void __launch_bounds__(256) k_cr_gemm(const float* __restrict__ A, in
     for (int e = tid; e < GM_BK * GM_BN; e += 256) {
       const int t = e / GM_BN, j = e % GM_BN;
       const int64_t gj = j0 + j, gt = t0 + t;
-      Bs[t][j] = (gj < N && gt < Kc) ? float(B[gt * ldb + gj]) : 0.f;
+      Bs[t][j] = (gj < N && gt < Kc) ? B[gt * ldb + gj] : 0.f;
     }
     __syncthreads();
+    float part[4][4];
+#pragma unroll
+    for (int p = 0; p < 4; ++p)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) part[p][q] = 0.f;
 #pragma unroll 8
     for (int t = 0; t < GM_BK; ++t) {
       const float4 a4 = *reinterpret_cast<const float4*>(&As[t][ty * 4]);
@@ -108,14 +112,18 @@ __global__ void __launch_bounds__(256) k_cr_gemm(const float* __restrict__ A, in
         for (int q = 0; q < 4; ++q) part[p][q] = fmaf(av[p], bv[q], part[p][q]);
     }
     __syncthreads();
+#pragma unroll
+    for (int p = 0; p < 4; ++p)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) run_sum[p][q] += part[p][q];
     if (++run == GM_RUN) {
       run = 0;
 #pragma unroll
       for (int p = 0; p < 4; ++p)
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          acc[p][q] += double(part[p][q]);
-          part[p][q] = 0.f;
+          acc[p][q] += double(run_sum[p][q]);
+          run_sum[p][q] = 0.f;
         }
     }
   }
@@ -124,7 +132,7 @@ __global__ void __launch_bounds__(256) k_cr_gemm(const float* __restrict__ A, in
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const int64_t gi = i0 + ty * 4 + p, gj = j0 + tx * 4 + q;
-      if (gi < M && gj < N) C[gi * ldc + gj] = acc[p][q] + double(part[p][q]);
+      if (gi < M && gj < N) C[gi * ldc + gj] = TC(acc[p][q] + double(run_sum[p][q]));
     }
 }
 
@@ -151,20 +159,23 @@ __device__ __forceinline__ void load_tile(double (*S)[NBP], const double* __rest
 
 // Diagonal tile jb: factor in shared memory (unblocked, right-looking), write the factor back,
 // and write the inverse of the triangular factor to Dinv[jb].  A pivot that is not positive
-// sets the failure flag (E^T E + beta I is not positive definite in floating point).
+// sets the failure flag (E^T E + beta I is not positive definite in floating point).  Thread
+// (ty, tx) of the 16 x 16 grid owns entries (ty + 16 p, tx + 16 q).
 __global__ void __launch_bounds__(256) k_cr_potrf(double* __restrict__ K, int64_t mp, int jb,
                                                  double* __restrict__ Dinv, int32_t* flag) {
   extern __shared__ __align__(16) unsigned char cr_smem[];
   double(*S)[NBP] = reinterpret_cast<double(*)[NBP]>(cr_smem);
   double(*X)[NBP] = reinterpret_cast<double(*)[NBP]>(cr_smem + sizeof(double) * NB * NBP);
+  __shared__ double rinv[NB];
   __shared__ int bad;
   if (failed(flag)) return;
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
   const int64_t o = int64_t(jb) * NB;
   double* Kd = K + o * mp + o;
   for (int e = tid; e < NB * NB; e += 256) {
     const int r = e / NB, c = e % NB;
     S[r][c] = (c <= r) ? Kd[int64_t(r) * mp + c] : 0.0;
+    X[r][c] = (r == c) ? 1.0 : 0.0;
   }
   if (tid == 0) bad = 0;
   __syncthreads();
@@ -175,13 +186,26 @@ __global__ void __launch_bounds__(256) k_cr_potrf(double* __restrict__ K, int64_
       break;
     }
     const double lc = sqrt(piv);
+    const double inv = 1.0 / lc;
     __syncthreads();
-    for (int r = c + tid; r < NB; r += 256) S[r][c] = (r == c) ? lc : S[r][c] / lc;
+    if (tid < NB) {
+      if (tid > c) S[tid][c] *= inv;
+      if (tid == c) {
+        S[c][c] = lc;
+        rinv[c] = inv;
+      }
+    }
     __syncthreads();
-    const int w = NB - c - 1;
-    for (int e = tid; e < w * w; e += 256) {
-      const int rr = c + 1 + e / w, ss = c + 1 + e % w;
-      if (ss <= rr) S[rr][ss] -= S[rr][c] * S[ss][c];
+#pragma unroll
+    for (int p = 0; p < 4; ++p) {
+      const int rr = ty + 16 * p;
+      if (rr <= c) continue;
+      const double lrc = S[rr][c];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int ss = tx + 16 * q;
+        if (ss > c && ss <= rr) S[rr][ss] = fma(-lrc, S[ss][c], S[rr][ss]);
+      }
     }
     __syncthreads();
   }
@@ -193,18 +217,24 @@ __global__ void __launch_bounds__(256) k_cr_potrf(double* __restrict__ K, int64_
     const int r = e / NB, c = e % NB;
     if (c <= r) Kd[int64_t(r) * mp + c] = S[r][c];
   }
-  // inverse of the lower factor, column t by forward substitution on e_t
-  if (tid < NB) {
-    const int t = tid;
-    for (int r = 0; r < t; ++r) X[r][t] = 0.0;
-    X[t][t] = 1.0 / S[t][t];
-    for (int r = t + 1; r < NB; ++r) {
-      double s = 0.0;
-      for (int u = t; u < r; ++u) s += S[r][u] * X[u][t];
-      X[r][t] = -s / S[r][r];
+  // X = L^-1, right-looking on the identity: row c scaled by 1 / L_cc, then removed from the rows
+  // below
+  for (int c = 0; c < NB; ++c) {
+    if (tid <= c) X[c][tid] *= rinv[c];
+    __syncthreads();
+#pragma unroll
+    for (int p = 0; p < 4; ++p) {
+      const int rr = ty + 16 * p;
+      if (rr <= c) continue;
+      const double lrc = S[rr][c];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int u = tx + 16 * q;
+        if (u <= c) X[rr][u] = fma(-lrc, X[c][u], X[rr][u]);
+      }
     }
+    __syncthreads();
   }
-  __syncthreads();
   double* D = Dinv + int64_t(jb) * NB * NB;
   for (int e = tid; e < NB * NB; e += 256) D[e] = X[e / NB][e % NB];
 }
@@ -518,7 +548,7 @@ __global__ void __launch_bounds__(256) k_cr_ritz_eig(const double* __restrict__ 
     if (a > b) A[a][b] = A[b][a];
   }
   __syncthreads();
-  if (tid < 32) jacobi_eig_warp<ELLP>(A, V, order, ell, tid);
+  jacobi_eig_block<ELLP>(A, V, order, ell);
   __syncthreads();
   const double lam1 = A[order[0]][order[0]];
   const double s1 = lam1 > 0.0 ? sqrt(lam1) : 0.0;
@@ -626,7 +656,7 @@ __global__ void __launch_bounds__(256) k_cr_ritz_sign(float* __restrict__ P, flo
 }
 
 struct RsvdWs {
-  size_t K, Dinv, Kf, Dinvf, Ym, Wm, Wf, Zd, Tn, qrpart, qrfac, part, Ur, sig, amv, ami, flag, total;
+  size_t K, Dinv, Kf, Dinvf, Ym, Wm, Wf, Zd, Zf, Tn, qrpart, qrfac, part, Ur, sig, amv, ami, flag, total;
 };
 
 RsvdWs rsvd_ws(int64_t Np, int64_t m, int64_t d, int L, int ell, int r) {
@@ -652,7 +682,8 @@ RsvdWs rsvd_ws(int64_t Np, int64_t m, int64_t d, int L, int ell, int r) {
   w.Wm = take(sizeof(double) * mp * n);
   w.Wf = take(sizeof(float) * mp * n);
   w.Zd = take(sizeof(double) * d * n);
-  w.Tn = take(sizeof(double) * Np * n);
+  w.Zf = take(sizeof(float) * d * n);
+  w.Tn = take(sizeof(float) * Np * n);
   w.qrpart = take(sizeof(double) * L * nchqr * ellp * ellp);
   w.qrfac = take(sizeof(double) * L * ellp * ellp);
   w.part = take(sizeof(double) * L * nchd * ell * ell);
@@ -665,12 +696,12 @@ RsvdWs rsvd_ws(int64_t Np, int64_t m, int64_t d, int L, int ell, int r) {
   return w;
 }
 
-template <bool AT, typename TB>
-cudaError_t gemm(const float* A, int64_t lda, int64_t sA, const TB* B, int64_t ldb, int64_t sB, double* C,
+template <bool AT, typename TC>
+cudaError_t gemm(const float* A, int64_t lda, int64_t sA, const float* B, int64_t ldb, int64_t sB, TC* C,
                  int64_t ldc, int64_t sC, int64_t M, int64_t N, int64_t Kc, int batch, int lower_only,
                  cudaStream_t s) {
   const dim3 grid(unsigned((N + GM_BN - 1) / GM_BN), unsigned((M + GM_BM - 1) / GM_BM), unsigned(batch));
-  k_cr_gemm<AT, TB><<<grid, 256, 0, s>>>(A, lda, sA, B, ldb, sB, C, ldc, sC, M, N, Kc, lower_only);
+  k_cr_gemm<AT, TC><<<grid, 256, 0, s>>>(A, lda, sA, B, ldb, sB, C, ldc, sC, M, N, Kc, lower_only);
   return cudaGetLastError();
 }
 
@@ -749,7 +780,8 @@ cudaError_t rsvd_t(const float* E, const float* G, int64_t Np, int64_t m, int64_
   double* Wm = reinterpret_cast<double*>(ws + w.Wm);
   float* Wf = reinterpret_cast<float*>(ws + w.Wf);
   double* Zd = reinterpret_cast<double*>(ws + w.Zd);
-  double* Tn = reinterpret_cast<double*>(ws + w.Tn);
+  float* Zf = reinterpret_cast<float*>(ws + w.Zf);
+  float* Tn = reinterpret_cast<float*>(ws + w.Tn);
   double* qrpart = reinterpret_cast<double*>(ws + w.qrpart);
   double* qrfac = reinterpret_cast<double*>(ws + w.qrfac);
   int32_t* flag = reinterpret_cast<int32_t*>(ws + w.flag);
@@ -763,7 +795,7 @@ cudaError_t rsvd_t(const float* E, const float* G, int64_t Np, int64_t m, int64_
   CR_TRY(cudaMemsetAsync(flag, 0, sizeof(int32_t) * 64, s));
   CR_TRY(cudaMemsetAsync(Ym, 0, sizeof(double) * mp * n, s));
   // K = E^T E (lower tiles), + beta I, padded
-  CR_TRY((gemm<true, float>(E, m, 0, E, m, 0, K, mp, 0, m, m, Np, 1, 1, s)));
+  CR_TRY((gemm<true, double>(E, m, 0, E, m, 0, K, mp, 0, m, m, Np, 1, 1, s)));
   k_cr_pad<<<4 * sm_count(), 256, 0, s>>>(K, m, mp, double(beta));
   CR_TRY(cudaGetLastError());
   for (int jb = 0; jb < nb; ++jb) {
@@ -779,26 +811,28 @@ cudaError_t rsvd_t(const float* E, const float* G, int64_t Np, int64_t m, int64_
     CR_TRY((cvt<double, float>(K, Kf, mp * mp, s)));
     CR_TRY((cvt<double, float>(Dinv, Dinvf, int64_t(nb) * NB * NB, s)));
   }
-  // K^-1 V in place on V (mp x n, fp64): exact (fp64 factor) or inside the power iterations
-  // (fp32 factor on an fp32 copy)
-  auto kinv = [&](double* V, bool exact) -> cudaError_t {
-    if (exact) return solve<double>(K, mp, Dinv, V, n, flag, s);
-    CR_TRY((cvt<double, float>(V, Wf, mp * n, s)));
-    CR_TRY(solve<float>(Kf, mp, Dinvf, Wf, n, flag, s));
-    return cvt<float, double>(Wf, V, mp * n, s);
-  };
-  // Ym = F^T X for every block, X (d x ell per block) at column offset l ell of Xd (ld ldx, block
-  // stride sx); Tn = G_l X, Ym = K^-1 E^T Tn
-  auto apply_Ft = [&](auto* Xd, int64_t ldx, int64_t sx, bool exact) -> cudaError_t {
-    using TX = std::remove_const_t<std::remove_pointer_t<decltype(Xd)>>;
-    CR_TRY((gemm<false, TX>(G, d, Np * d, Xd, ldx, sx, Tn, n, ell, Np, ell, d, L, 0, s)));
+  // Ym = F^T X for every block, X (d x ell per block, fp32) at column offset l ell of Xf (ld ldx,
+  // block stride sx): Tn = G_l X, Ym = K^-1 E^T Tn (fp64 factor when exact, else the fp32 one on
+  // an fp32 copy)
+  auto apply_Ft = [&](const float* Xf, int64_t ldx, int64_t sx, bool exact) -> cudaError_t {
+    CR_TRY((gemm<false, float>(G, d, Np * d, Xf, ldx, sx, Tn, n, ell, Np, ell, d, L, 0, s)));
     CR_TRY((gemm<true, double>(E, m, 0, Tn, n, 0, Ym, n, 0, m, n, Np, 1, 0, s)));
-    return kinv(Ym, exact);
+    if (exact) return solve<double>(K, mp, Dinv, Ym, n, flag, s);
+    CR_TRY((cvt<double, float>(Ym, Wf, mp * n, s)));
+    CR_TRY(solve<float>(Kf, mp, Dinvf, Wf, n, flag, s));
+    return cvt<float, double>(Wf, Ym, mp * n, s);
   };
-  // Zd = F Y for every block, Y = Vm (mp x n, overwritten by K^-1 Y): Tn = E K^-1 Y, Zd = G_l^T Tn
+  // Zd = F Y for every block, Y = Vm (mp x n, fp64; overwritten when exact): Wf = K^-1 Y in fp32,
+  // Tn = E Wf, Zd = G_l^T Tn
   auto apply_F = [&](double* Vm, bool exact) -> cudaError_t {
-    CR_TRY(kinv(Vm, exact));
-    CR_TRY((gemm<false, double>(E, m, 0, Vm, n, 0, Tn, n, 0, Np, n, m, 1, 0, s)));
+    if (exact) {
+      CR_TRY(solve<double>(K, mp, Dinv, Vm, n, flag, s));
+      CR_TRY((cvt<double, float>(Vm, Wf, mp * n, s)));
+    } else {
+      CR_TRY((cvt<double, float>(Vm, Wf, mp * n, s)));
+      CR_TRY(solve<float>(Kf, mp, Dinvf, Wf, n, flag, s));
+    }
+    CR_TRY((gemm<false, float>(E, m, 0, Wf, n, 0, Tn, n, 0, Np, n, m, 1, 0, s)));
     return gemm<true, double>(G, d, Np * d, Tn, n, ell, Zd, n, ell, d, ell, Np, L, 0, s);
   };
   CR_TRY(apply_Ft(Omega, int64_t(ell), int64_t(0), q == 0));
@@ -806,7 +840,8 @@ cudaError_t rsvd_t(const float* E, const float* G, int64_t Np, int64_t m, int64_
   for (int it = 0; it < q; ++it) {
     CR_TRY(apply_F(Ym, false));
     CR_TRY(orth<ELLP>(Zd, d, n, ell, L, qrpart, qrfac, s));
-    CR_TRY(apply_Ft(static_cast<const double*>(Zd), n, int64_t(ell), it == q - 1));
+    CR_TRY((cvt<double, float>(Zd, Zf, d * n, s)));
+    CR_TRY(apply_Ft(Zf, n, int64_t(ell), it == q - 1));
     CR_TRY(orth<ELLP>(Ym, m, n, ell, L, qrpart, qrfac, s));
   }
   // Rayleigh-Ritz: B^T = F Q_Y

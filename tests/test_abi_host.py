@@ -158,8 +158,8 @@ def test_calib_rsvd_validation(L):
     assert call(ws_bytes=16) == 7    # workspace smaller than required
     rc, n = _ws(L.loca_calib_fit_rsvd_workspace_size, 8192, 3584, 3584, 28, 16, 32)
     # E^T E (m x m fp64) and its fp32 copy, plus the ell-column blocks of every block (two
-    # m-wide fp64 and one fp32, one d-wide, one Np-wide) dominate
+    # m-wide fp64 and one fp32, one d-wide fp64 and its fp32 copy, one Np-wide fp32) dominate
     n_cols = 28 * 32
-    floor = 12 * 3584 * 3584 + 8 * (2 * 3584 * n_cols + 3584 * n_cols + 8192 * n_cols) + 4 * 3584 * n_cols
+    floor = 12 * 3584 * 3584 + (8 * 2 * 3584 + 4 * 3584 + 12 * 3584 + 4 * 8192) * n_cols
     assert rc == 0 and floor <= n < floor + (16 << 20) and n % 256 == 0
     assert _ws(L.loca_calib_fit_rsvd_workspace_size, 8192, 3584, 3584, 28, 33, 32)[0] == 2
