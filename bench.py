@@ -62,6 +62,7 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-kspace", action="store_true", help="skip the k-space statistics measurement")
     ap.add_argument("--no-vocab", action="store_true", help="skip the wide-vocabulary head-error measurement")
+    ap.add_argument("--no-calib", action="store_true", help="skip the one-shot d-wide feedback-fit measurement")
     ap.add_argument("--e2e-group", type=int, default=2, help="blocks per host-to-device copy in the e2e leg")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -435,6 +436,37 @@ def main():
         del zv, Ev, cev
         torch.cuda.empty_cache()
 
+    # the one-shot feedback fit in the paper's d-wide error space (m = d) at the 7B width: every
+    # block's rank-16 map from Np = 8192 probe pairs, randomized subspace iteration with a sketch
+    # of 32 and two power iterations (untimed in the step; reported on its own)
+    calib = None
+    if not args.no_calib and world == 1:
+        Np_c, m_c, r_c, ell_c, q_c = 8192, d, 16, 32, 2
+        pc = S.device_probe_pairs(Np_c, m_c, d, L, rank=8, seed=1, device=dev)
+        Ec, Gc = pc["E_probe"], pc["G_probe"]
+        Om = torch.from_numpy(S.omega_matrix(d, ell_c, seed=1)).to(dev)
+        beta_c = 1e-3 * float(torch.sum(Ec.double() ** 2).item()) / m_c
+        Pc = torch.empty((L, m_c, r_c), **f32)
+        Qc = torch.empty((L, r_c, d), **f32)
+        wsc = torch.empty(lc.calib_fit_rsvd_workspace_size(Np_c, m_c, d, L, r_c, ell_c), dtype=torch.uint8,
+                          device=dev)
+        lc.loca_calib_fit_rsvd(Ec, Gc, beta_c, r_c, Om, q_c, Pc, Qc, workspace=wsc, stream=stream)
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(3):
+            lc.loca_calib_fit_rsvd(Ec, Gc, beta_c, r_c, Om, q_c, Pc, Qc, workspace=wsc, stream=stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        if lc.loca_device_status() != 0:
+            raise SystemExit("the feedback fit reported a device error")
+        calib = {"workload": "qwen2.5-7b feedback fit, d-wide error space", "Np": Np_c, "m": m_c, "d": d, "L": L,
+                 "r": r_c, "ell": ell_c, "q": q_c, "ms": a.elapsed_time(b) / 3,
+                 "method": "randomized subspace iteration + Rayleigh-Ritz (loca_calib_fit_rsvd)"}
+        del Ec, Gc, pc, wsc, Pc, Qc
+        torch.cuda.empty_cache()
+
     # end to end through the public API: host inputs copied in, adapters copied out, per step
     e2e = None
     if not args.no_e2e:
@@ -522,6 +554,7 @@ def main():
             "e2e": e2e,
             "kspace": kspace,
             "head_error_vocab": vocab,
+            "calibration": calib,
             "cpu_baseline": cpu,
             "clocks": clk.summary(),
         }

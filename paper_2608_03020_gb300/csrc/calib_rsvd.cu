@@ -50,14 +50,17 @@ __device__ __forceinline__ bool failed(const int32_t* flag) { return *reinterpre
 
 // C_b[i][j] = sum_t A_b(i, t) B_b(t, j);  A_b(i, t) = A[t lda + i] (AT) or A[i lda + t];
 // B_b(t, j) = B[t ldb + j]; batch b = blockIdx.z with element strides sA, sB, sC.  Products are
-// summed in fp32 over 32 terms, those sums in fp32 over 16 (512 terms), and those in fp64.
+// summed in fp32 over 32 terms, those sums in fp32 over 16 (512 terms), and those in fp64.  The
+// next 32-term slab is loaded into registers while the current one is multiplied, then stored
+// to the other shared-memory buffer (one barrier per slab).
 template <bool AT, typename TC>
 __global__ void __launch_bounds__(256) k_cr_gemm(const float* __restrict__ A, int64_t lda, int64_t sA,
                                                 const float* __restrict__ B, int64_t ldb, int64_t sB,
                                                 TC* __restrict__ C, int64_t ldc, int64_t sC, int64_t M, int64_t N,
                                                 int64_t Kc, int lower_only) {
-  __shared__ __align__(16) float As[GM_BK][GM_BM + 4];
-  __shared__ __align__(16) float Bs[GM_BK][GM_BN + 4];
+  __shared__ __align__(16) float As[2][GM_BK][GM_BM + 4];
+  __shared__ __align__(16) float Bs[2][GM_BK][GM_BN + 4];
+  constexpr int LPT = GM_BK * GM_BM / 256;
   const int64_t i0 = int64_t(blockIdx.y) * GM_BM, j0 = int64_t(blockIdx.x) * GM_BN;
   if (lower_only && j0 > i0) return;
   const int64_t b = blockIdx.z;
@@ -65,6 +68,37 @@ __global__ void __launch_bounds__(256) k_cr_gemm(const float* __restrict__ A, in
   B += b * sB;
   C += b * sC;
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  float ra[LPT], rb[LPT];
+  auto gload = [&](int64_t t0) {
+#pragma unroll
+    for (int k = 0; k < LPT; ++k) {
+      const int e = tid + 256 * k;
+      int t, i;
+      if (AT) {
+        t = e / GM_BM;
+        i = e % GM_BM;
+      } else {
+        i = e / GM_BK;
+        t = e % GM_BK;
+      }
+      const int64_t gi = i0 + i, gt = t0 + t;
+      ra[k] = (gi < M && gt < Kc) ? (AT ? A[gt * lda + gi] : A[gi * lda + gt]) : 0.f;
+      const int tb = e / GM_BN, jb = e % GM_BN;
+      const int64_t gj = j0 + jb, gtb = t0 + tb;
+      rb[k] = (gj < N && gtb < Kc) ? B[gtb * ldb + gj] : 0.f;
+    }
+  };
+  auto sstore = [&](int buf) {
+#pragma unroll
+    for (int k = 0; k < LPT; ++k) {
+      const int e = tid + 256 * k;
+      if (AT)
+        As[buf][e / GM_BM][e % GM_BM] = ra[k];
+      else
+        As[buf][e % GM_BK][e / GM_BK] = ra[k];
+      Bs[buf][e / GM_BN][e % GM_BN] = rb[k];
+    }
+  };
   double acc[4][4];
   float run_sum[4][4];
 #pragma unroll
@@ -74,36 +108,22 @@ __global__ void __launch_bounds__(256) k_cr_gemm(const float* __restrict__ A, in
       acc[p][q] = 0.0;
       run_sum[p][q] = 0.f;
     }
-  int run = 0;
+  gload(0);
+  sstore(0);
+  __syncthreads();
+  int run = 0, buf = 0;
   for (int64_t t0 = 0; t0 < Kc; t0 += GM_BK) {
-    if (AT) {
-      for (int e = tid; e < GM_BK * GM_BM; e += 256) {
-        const int t = e / GM_BM, i = e % GM_BM;
-        const int64_t gi = i0 + i, gt = t0 + t;
-        As[t][i] = (gi < M && gt < Kc) ? A[gt * lda + gi] : 0.f;
-      }
-    } else {
-      for (int e = tid; e < GM_BK * GM_BM; e += 256) {
-        const int i = e / GM_BK, t = e % GM_BK;
-        const int64_t gi = i0 + i, gt = t0 + t;
-        As[t][i] = (gi < M && gt < Kc) ? A[gi * lda + gt] : 0.f;
-      }
-    }
-    for (int e = tid; e < GM_BK * GM_BN; e += 256) {
-      const int t = e / GM_BN, j = e % GM_BN;
-      const int64_t gj = j0 + j, gt = t0 + t;
-      Bs[t][j] = (gj < N && gt < Kc) ? B[gt * ldb + gj] : 0.f;
-    }
-    __syncthreads();
+    const bool more = t0 + GM_BK < Kc;
+    if (more) gload(t0 + GM_BK);
     float part[4][4];
 #pragma unroll
     for (int p = 0; p < 4; ++p)
 #pragma unroll
       for (int q = 0; q < 4; ++q) part[p][q] = 0.f;
-#pragma unroll 8
+#pragma unroll
     for (int t = 0; t < GM_BK; ++t) {
-      const float4 a4 = *reinterpret_cast<const float4*>(&As[t][ty * 4]);
-      const float4 b4 = *reinterpret_cast<const float4*>(&Bs[t][tx * 4]);
+      const float4 a4 = *reinterpret_cast<const float4*>(&As[buf][t][ty * 4]);
+      const float4 b4 = *reinterpret_cast<const float4*>(&Bs[buf][t][tx * 4]);
       const float av[4] = {a4.x, a4.y, a4.z, a4.w};
       const float bv[4] = {b4.x, b4.y, b4.z, b4.w};
 #pragma unroll
@@ -111,7 +131,9 @@ __global__ void __launch_bounds__(256) k_cr_gemm(const float* __restrict__ A, in
 #pragma unroll
         for (int q = 0; q < 4; ++q) part[p][q] = fmaf(av[p], bv[q], part[p][q]);
     }
+    if (more) sstore(buf ^ 1);
     __syncthreads();
+    buf ^= 1;
 #pragma unroll
     for (int p = 0; p < 4; ++p)
 #pragma unroll
