@@ -183,3 +183,35 @@ def test_rsvd_full_size_sampled_block(lc):
     assert np.max(np.abs(sig[0] - sr[0])) < 1e-5 * sr[0, 0]
     assert np.allclose(Q[0] @ Q[0].T, np.eye(r), atol=1e-5)
     assert np.all(np.isfinite(P)) and np.all(np.isfinite(Q))
+
+
+def test_d_wide_fit_feeds_the_label_restricted_targets(lc):
+    """The paper's d-wide error space through the hot path: probe errors e = W^T eps (rows
+    E_d = E_C W, W the head's C label rows, orthonormal here), fitted on the GPU with m = d and
+    folded through the head (P_C = W P_d), give the label-space fit (push-through identity, same
+    beta); loca_targets with the folded factors then gives the targets of the label-space fit."""
+    Np, C, d, L, r = 2048, 4, 512, 2, 4
+    pp = S.host_probe_pairs(Np=Np, m=C, d=d, L=L, rank=C, seed=41)
+    E_C, G = pp["E_probe"], pp["G_probe"]
+    rng = np.random.default_rng(41)
+    W = np.linalg.qr(rng.standard_normal((d, C)))[0].T.astype(np.float32)  # C x d
+    E_d = (E_C.astype(np.float64) @ W).astype(np.float32)
+    beta = 0.05 * float(np.sum(E_d.astype(np.float64) ** 2)) / d
+    P_d, Q_d, s_d = _fit(lc, _dev(E_d), _dev(G), beta, r, _dev(S.omega_matrix(d, 8, seed=41)), 1)
+    P_fold = np.einsum("cj,ljs->lcs", W.astype(np.float64), P_d)
+    P_C, Q_C, s_C, _ = O.calib_fit(E_C, G, beta, r)
+    for l in range(L):
+        assert _rel(P_fold[l] @ Q_d[l], P_C[l] @ Q_C[l]) < 1e-4, l
+        assert np.max(np.abs(s_d[l] - s_C[l])) < 1e-5 * s_C[l, 0]
+    # targets on fresh tokens: folded d-wide factors vs the GPU's label-space fit
+    Pg = torch.empty((L, C, r), device="cuda")
+    Qg = torch.empty((L, r, d), device="cuda")
+    lc.loca_calib_fit(_dev(E_C), _dev(G), beta, r, Pg, Qg)
+    E_run = _dev(rng.standard_normal((4096, C)).astype(np.float32))
+    T1 = torch.empty((L, 4096, d), device="cuda")
+    T2 = torch.empty((L, 4096, d), device="cuda")
+    lc.loca_targets(E_run, _dev(P_fold.astype(np.float32)), _dev(Q_d.astype(np.float32)), T1)
+    lc.loca_targets(E_run, Pg, Qg, T2)
+    torch.cuda.synchronize()
+    for l in range(L):
+        assert _rel(T1[l].cpu().numpy(), T2[l].cpu().numpy().astype(np.float64)) < 1e-4, l

@@ -540,6 +540,27 @@ def test_rsvd_converges_to_the_truncation_on_a_gapped_spectrum():
     assert _rel(P, P0) < 1e-8 and _rel(Q, Q0) < 1e-8
 
 
+def test_d_wide_fit_folded_through_the_head_is_the_label_space_fit():
+    """Reading of the head fold: with the paper's d-wide error e = W^T eps (rows E_d = E_C W, W the
+    head's C label rows, orthonormal here), the push-through identity gives
+    (W^T A W + beta I)^-1 W^T = W^T (A + beta I)^-1 for A = E_C^T E_C, so F_hat_d^T = W^T F_hat_C^T:
+    the d-wide fit, folded as P_C = W P_d, is the label-space fit (same beta), for the exact and
+    the randomized fit alike (rank <= C <= ell)."""
+    rng = np.random.default_rng(31)
+    Np, C, d, L, beta = 60, 3, 24, 2, 0.3
+    W = np.linalg.qr(rng.standard_normal((d, C)))[0].T  # C x d, orthonormal rows
+    E_C = rng.standard_normal((Np, C))
+    G = rng.standard_normal((L, Np, d))
+    E_d = E_C @ W
+    P_C, Q_C, s_C, _ = O.calib_fit(E_C, G, beta, C)
+    P_d, Q_d, s_d, _ = O.calib_fit(E_d, G, beta, C)
+    Pr, Qr, sr = O.calib_fit_rsvd(E_d, G, beta, C, S.omega_matrix(d, 5, seed=31), 0)
+    for l in range(L):
+        assert _rel(W @ P_d[l], P_C[l]) < 1e-10 and _rel(Q_d[l], Q_C[l]) < 1e-10
+        assert _rel(W @ Pr[l], P_C[l]) < 1e-10 and _rel(Qr[l], Q_C[l]) < 1e-10
+    assert _rel(s_d, s_C) < 1e-12 and _rel(sr, s_C) < 1e-12
+
+
 def test_linear_network_targets_equal_backprop_gradients():
     """Check 4: on an all-linear tokenwise network h_l = W_l h_{l-1}, z = W_u h_L, the true
     hidden-state gradient is g_l = (W_L ... W_{l+1})^T W_u^T eps (S3), exactly linear in the
