@@ -2,9 +2,10 @@
 """Throughput of one LoCA Stage-II pass on GB300: tokens/s/block at the Qwen2.5-7B shape.
 
 A step is one pass of the whole hot path over one batch of synthetic inputs resident in HBM:
-  loca_error -> loca_targets -> loca_batch_step -> loca_gram_cross -> loca_ridge_solve
-(head error, feedback targets, scale-normalised step, Gram / cross statistics on the tensor
-cores, projected ridge solves for every block and every candidate lambda).
+  loca_error -> loca_targets -> loca_gram_cross -> loca_step_from_gram -> loca_ridge_solve
+(head error, feedback targets, Gram / cross statistics on the tensor cores, the
+scale-normalised step from tr(Gram) = ||X||^2 of the one mini-batch, projected ridge solves for
+every block and every candidate lambda with the step applied to the cross product).
 
 value     = N * L / (seconds per step)            tokens per second per block (higher is better)
 e2e       = the same metric with the inputs copied from pinned host memory and the adapters
@@ -271,11 +272,11 @@ def main():
     B = torch.empty((nl, L, d, k), **f32)
     info = torch.empty((nl, L), dtype=torch.int32, device=dev)
     ws_t = torch.empty(lc.targets_workspace_size(N, L, d), dtype=torch.uint8, device=dev)
-    ws_b = torch.empty(lc.batch_step_workspace_size(L), dtype=torch.uint8, device=dev)
+    ones = torch.ones((L,), **f32)
     ws_g = torch.empty(lc.gram_cross_workspace_size(), dtype=torch.uint8, device=dev)
     ws_s = torch.empty(lc.ridge_solve_workspace_size(L, d, k), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
-    launches_per_step = 1 + 2 + 2 + 1 + 2  # error; targets+reduce; sumsq+step; gram/cross; project+solve
+    launches_per_step = 1 + 2 + 1 + 1 + 2  # error; targets+reduce; gram/cross; step; project+solve
 
     def step(ev=None):
         if ev is not None:
@@ -286,13 +287,16 @@ def main():
         lc.loca_targets(E, P, Q, T, tsq=tsq, workspace=ws_t, stream=stream)
         if ev is not None:
             ev[2].record(stream)
-        lc.loca_batch_step(X, tsq, w.eta, xsq, alpha, zero_first=True, workspace=ws_b, stream=stream)
+        # one mini-batch: the cross product at alpha = 1, the step from the Gram trace, alpha
+        # applied to the cross product in the solve (X is read by the Gram kernel only)
+        lc.loca_gram_cross(X, T, ones, gram, cross, zero_first=True, workspace=ws_g, stream=stream)
         if ev is not None:
             ev[3].record(stream)
-        lc.loca_gram_cross(X, T, alpha, gram, cross, zero_first=True, workspace=ws_g, stream=stream)
+        lc.loca_step_from_gram(gram, tsq, w.eta, xsq, alpha, stream=stream)
         if ev is not None:
             ev[4].record(stream)
-        lc.loca_ridge_solve(gram, cross, A, w.lambda_rel, B, info, xsq_total=xsq, workspace=ws_s, stream=stream)
+        lc.loca_ridge_solve(gram, cross, A, w.lambda_rel, B, info, xsq_total=xsq, cross_scale=alpha,
+                            workspace=ws_s, stream=stream)
         if ev is not None:
             ev[5].record(stream)
 
@@ -324,7 +328,7 @@ def main():
     ms_total = t_start.elapsed_time(t_end)
     ms_total = max_over_ranks(world, ms_total)
     ms_step = ms_total / args.steps
-    stage_names = ["error", "targets", "batch_step", "gram_cross", "ridge_solve"]
+    stage_names = ["error", "targets", "gram_cross", "step", "ridge_solve"]
     stages = {n: statistics.mean(e[i].elapsed_time(e[i + 1]) for e in evs) for i, n in enumerate(stage_names)}
     status = lc.loca_device_status()
     if status != 0:
@@ -508,6 +512,19 @@ def main():
         e2e_steps = max(1, min(args.steps, 5))
         e2e_step()
         torch.cuda.synchronize()
+
+        # the link's host-to-device rate right before the timed steps: the host memory and its
+        # bandwidth are shared with whatever else runs on the machine
+        def link_gbs():
+            nb = min(group, L) * N * d
+            a_, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a_.record(stream)
+            staging.view(-1)[:nb].copy_(hX.view(-1)[:nb], non_blocking=True)
+            b_.record(stream)
+            torch.cuda.synchronize()
+            return nb * staging.element_size() / (a_.elapsed_time(b_) / 1e3) / 1e9
+
+        link_before = link_gbs()
         barrier(world)
         a = torch.cuda.Event(enable_timing=True)
         b = torch.cuda.Event(enable_timing=True)
@@ -517,9 +534,11 @@ def main():
         b.record(stream)
         torch.cuda.synchronize()
         ms_e2e = max_over_ranks(world, a.elapsed_time(b)) / e2e_steps
+        link_after = link_gbs()
         e2e = {"value": world * N * L / (ms_e2e / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e, "steps": e2e_steps,
-               "x_from_host": f"loca_accumulate_streamed, {group} blocks per copy"}
+               "x_from_host": f"loca_accumulate_streamed, {group} blocks per copy",
+               "h2d_link_gbs_before_after": [round(link_before, 1), round(link_after, 1)]}
         if int(info.abs().sum().item()) != 0 or lc.loca_device_status() != 0:
             raise SystemExit("the end-to-end steps reported a device error or a non-PD system")
         del hX, hz, staging

@@ -305,26 +305,46 @@ int loca_accumulate_noalloc(const void* X, const void* T, int dtype, int32_t L, 
                             double* xsq_total, void* stream);
 
 /*
+ * loca_step_from_gram — the step of Eq. 10 for a pass with one mini-batch, without reading X:
+ * that batch's Gram (loca_gram_cross with zero_first = 1) holds X_l^T X_l, whose trace is
+ * ||X_l||_F^2, so
+ *
+ *   xsq_total[l] = tr(gram_l),   alpha[l] = -eta sqrt(xsq_total[l] / tsq[l])   (0 if tsq[l] == 0)
+ *
+ * (RMS ratio of Eq. 10; N d cancels).  With the cross product accumulated at alpha = 1, pass
+ * alpha to loca_ridge_solve as cross_scale: the same C_l as loca_batch_step + loca_gram_cross.
+ * gram  L x d x d float (device); tsq  L double; xsq_total  L double (output); alpha  L float
+ * (output).  The trace is summed in fp64 in a fixed order.  Only valid when gram holds exactly
+ * one mini-batch; for several, use loca_batch_step before each loca_gram_cross.
+ */
+int loca_step_from_gram(const float* gram, int32_t L, int64_t d, const double* tsq, float eta,
+                        double* xsq_total, float* alpha, void* stream);
+
+/*
  * loca_ridge_solve — closed-form block minimisers for every block l and every ridge
  * candidate j (Eq. 8; Theorem S6; positive-definite solve without an inverse, S7):
  *
  *   G_l   = A_l^T gram_l A_l                              (k x k, Eq. 9 with p = A_l^T x)
- *   C_l   = B_prev,l G_l + cross_l A_l                    (d x k; = sum_n rho_n p_n^T with
+ *   C_l   = B_prev,l G_l + s_l cross_l A_l                (d x k; = sum_n rho_n p_n^T with
  *                                                         rho = B^(t) p - eta_bar q, Eq. 6)
+ *   s_l   = cross_scale[l], or 1 when cross_scale is NULL (a pass with one mini-batch may
+ *           accumulate cross with alpha = 1 and apply alpha_l here; see loca_step_from_gram)
  *   lam   = lambda_rel[j] * xsq_total[l] / d              (xsq_total != NULL; = tr(gram_l)/d)
  *         = lambda_rel[j]                                 (xsq_total == NULL: absolute)
  *   B[j, l] = C_l (G_l + lam I)^-1   via Cholesky (fp64) and two triangular substitutions
  *
- * gram, cross   L x d x d float;  A  L x d x k float;  B_prev  L x d x k float or NULL (0)
+ * gram, cross   L x d x d float;  cross_scale  L float (device) or NULL
+ * A             L x d x k float;  B_prev  L x d x k float or NULL (0)
  * lambda_rel    HOST array of nl > 0 positive floats, nl <= 16
  * B             nl x L x d x k float output;  info  nl x L int32 output: 0, or p > 0 when
  *               the p-th pivot of G_l + lam I is not positive (B[j, l] is then zero)
  * G_out         L x k x k float output or NULL;  C_out  L x d x k float output or NULL
- * k in [1, 64].
+ * 1 <= k <= min(d, 32); 1 <= nl <= 16.
  */
 int loca_ridge_solve_workspace_size(int32_t L, int64_t d, int32_t k, size_t* bytes /* host */);
-int loca_ridge_solve(const float* gram, const float* cross, const double* xsq_total,
-                     const float* A, const float* B_prev, const float* lambda_rel /* host */,
+int loca_ridge_solve(const float* gram, const float* cross, const float* cross_scale,
+                     const double* xsq_total, const float* A, const float* B_prev,
+                     const float* lambda_rel /* host */,
                      int32_t nl, int32_t L, int64_t d, int32_t k, float* B, int32_t* info,
                      float* G_out, float* C_out, void* workspace, size_t workspace_bytes,
                      void* stream);

@@ -127,7 +127,7 @@ struct SolveWs {
 };
 SolveWs solve_ws(int32_t L, int64_t d, int32_t k) {
   SolveWs w{};
-  const size_t one = align256(sizeof(float) * size_t(L) * size_t(d) * size_t(k));
+  const size_t one = align256(sizeof(float) * size_t(project_split()) * size_t(L) * size_t(d) * size_t(k));
   w.ga = 0;
   w.ca = one;
   w.total = 2 * one;
@@ -559,9 +559,9 @@ int loca_ridge_solve_workspace_size(int32_t L, int64_t d, int32_t k, size_t* byt
   return LOCA_OK;
 }
 
-int loca_ridge_solve(const float* gram, const float* cross, const double* xsq_total, const float* A,
-                     const float* B_prev, const float* lambda_rel, int32_t nl, int32_t L, int64_t d,
-                     int32_t k, float* B, int32_t* info, float* G_out, float* C_out,
+int loca_ridge_solve(const float* gram, const float* cross, const float* cross_scale, const double* xsq_total,
+                     const float* A, const float* B_prev, const float* lambda_rel, int32_t nl, int32_t L,
+                     int64_t d, int32_t k, float* B, int32_t* info, float* G_out, float* C_out,
                      void* workspace, size_t workspace_bytes, void* stream) {
   g_msg[0] = 0;
   if (L < 1 || L > 65535 || d < 1) return fail(LOCA_ERR_SHAPE, "need 1 <= L <= 65535, d >= 1");
@@ -573,7 +573,7 @@ int loca_ridge_solve(const float* gram, const float* cross, const double* xsq_to
     if (!(lambda_rel[j] > 0.f)) return fail(LOCA_ERR_INVALID_ARG, "lambda_rel[%d] must be > 0", j);
   if (!aligned(gram, 4) || !aligned(cross, 4) || !aligned(A, 4) || !aligned(B, 4) ||
       !aligned(info, 4) || (B_prev && !aligned(B_prev, 4)) || (xsq_total && !aligned(xsq_total, 8)) ||
-      (G_out && !aligned(G_out, 4)) || (C_out && !aligned(C_out, 4)))
+      (G_out && !aligned(G_out, 4)) || (C_out && !aligned(C_out, 4)) || (cross_scale && !aligned(cross_scale, 4)))
     return fail(LOCA_ERR_ALIGNMENT, "pointers must be aligned to their element size");
   const SolveWs lay = solve_ws(L, d, k);
   int rc = check_ws(workspace, workspace_bytes, lay.total);
@@ -583,8 +583,22 @@ int loca_ridge_solve(const float* gram, const float* cross, const double* xsq_to
   float* CA = reinterpret_cast<float*>(ws_at(workspace, lay.ca));
   cudaError_t e = launch_project_rows(gram, cross, A, L, d, k, GA, CA, s);
   if (e != cudaSuccess) return cuda_fail(e, "loca_ridge_solve: projection");
-  e = launch_chol_solve(GA, CA, A, B_prev, xsq_total, lambda_rel, nl, L, d, k, B, info, G_out, C_out, s);
+  e = launch_chol_solve(GA, CA, A, B_prev, xsq_total, cross_scale, lambda_rel, nl, L, d, k, B, info, G_out,
+                        C_out, s);
   if (e != cudaSuccess) return cuda_fail(e, "loca_ridge_solve: solve");
+  return LOCA_OK;
+}
+
+int loca_step_from_gram(const float* gram, int32_t L, int64_t d, const double* tsq, float eta, double* xsq_total,
+                        float* alpha, void* stream) {
+  g_msg[0] = 0;
+  if (L < 1 || L > 65535 || d < 1) return fail(LOCA_ERR_SHAPE, "need 1 <= L <= 65535, d >= 1");
+  if (!gram || !tsq || !xsq_total || !alpha)
+    return fail(LOCA_ERR_INVALID_ARG, "gram, tsq, xsq_total and alpha are required");
+  if (!aligned(gram, 4) || !aligned(tsq, 8) || !aligned(xsq_total, 8) || !aligned(alpha, 4))
+    return fail(LOCA_ERR_ALIGNMENT, "pointers must be aligned to their element size");
+  cudaError_t e = launch_step_from_gram(gram, L, d, tsq, eta, xsq_total, alpha, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "loca_step_from_gram launch");
   return LOCA_OK;
 }
 

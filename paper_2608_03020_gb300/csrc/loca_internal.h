@@ -52,6 +52,9 @@ int sumsq_num_partials();
 cudaError_t launch_sumsq_and_step(const void* X, int dtype, int L, int64_t N, int64_t d,
                                   const double* tsq, float eta, int zero_first, double* xsq_total,
                                   double* partials, float* alpha, cudaStream_t s);
+// alpha_l and xsq_total[l] from tr(Gram_l) of a pass with one mini-batch (no read of X).
+cudaError_t launch_step_from_gram(const float* gram, int L, int64_t d, const double* tsq, float eta,
+                                  double* xsq_total, float* alpha, cudaStream_t s);
 // fp32-input Gram / cross (fp64 accumulation).
 cudaError_t launch_gram_cross_f32(const float* X, const float* T, int L, int64_t N, int64_t d,
                                   const float* alpha, int zero_first, float* gram, float* cross,
@@ -90,11 +93,13 @@ cudaError_t launch_kspace_solve(const float* G, const float* SC, const double* x
                                 cudaStream_t s);
 
 // ---- ridge solve (solve.cu)
+// GA / CA are project_split() partial products each (L x d x k fp32 apiece), summed by the solve.
+int project_split();
 cudaError_t launch_project_rows(const float* gram, const float* cross, const float* A, int L,
                                 int64_t d, int k, float* GA, float* CA, cudaStream_t s);
 cudaError_t launch_chol_solve(const float* GA, const float* CA, const float* A, const float* B_prev,
-                              const double* xsq_total, const float* lambda_rel, int nl, int L,
-                              int64_t d, int k, float* B, int32_t* info, float* G_out,
+                              const double* xsq_total, const float* cross_scale, const float* lambda_rel,
+                              int nl, int L, int64_t d, int k, float* B, int32_t* info, float* G_out,
                               float* C_out, cudaStream_t s);
 
 // ---- calibration (calib.cu)

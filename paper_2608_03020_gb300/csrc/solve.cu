@@ -1,12 +1,16 @@
 // Projected statistics and batched positive-definite solves (Eqs. 8 and 9; Theorem S6; S7).
 //
-// k_project_rows  GA_l = Gram_l A_l, CA_l = Cross_l A_l (d x k each).  One thread per row of the
-//                 stacked [Gram_l; Cross_l]; each thread streams its row with 32-byte loads while
-//                 the block shares A_l through shared memory (broadcast reads).  Bound: the HBM
+// k_project_rows  GA_l = Gram_l A_l, CA_l = Cross_l A_l (d x k each), as PR_SPLIT partial
+//                 products over quarters of the column range (GA = sum_z GA_z, summed in a fixed
+//                 order by k_chol_solve).  One thread per row of the stacked [Gram_l; Cross_l] and
+//                 column quarter; each thread streams its stretch of the row with 32-byte loads
+//                 while the block shares A_l through shared memory (broadcast reads).  The split
+//                 gives 4x as many, 4x shorter CTAs, so the last wave is small.  Bound: the HBM
 //                 read of Gram and Cross (8 d^2 bytes per block), k fp32 FMAs per element read.
 // k_chol_solve    one thread block per (ridge candidate j, block l):
 //                 G_l = A_l^T GA_l (k x k), lambda from the trace, Cholesky of G_l + lambda I in
-//                 fp64 in shared memory, then every row i of C_l = B_prev,l G_l + CA_l is solved
+//                 fp64 in shared memory, then every row i of C_l = B_prev,l G_l + s_l CA_l
+//                 (s_l = cross_scale[l], or 1) is solved
 //                 by a forward and a back substitution:  B[j, l, i] = C_l[i] (G_l + lambda I)^-1.
 //                 k is padded to a compile-time size with an identity block (its solution
 //                 columns are zero), so each row's solve stays in registers.
@@ -18,6 +22,7 @@ namespace {
 
 constexpr int PR_THREADS = 256;
 constexpr int PR_JC = 128;  // columns of A staged per step
+constexpr int PR_SPLIT = 4;  // column ranges per row (partial products)
 
 template <int KM>
 __global__ void __launch_bounds__(PR_THREADS) k_project_rows(const float* __restrict__ gram,
@@ -26,7 +31,10 @@ __global__ void __launch_bounds__(PR_THREADS) k_project_rows(const float* __rest
                                                             int k, float* __restrict__ GA,
                                                             float* __restrict__ CA) {
   __shared__ float As[PR_JC][KM];
-  const int l = blockIdx.y;
+  const int l = blockIdx.y, z = blockIdx.z;
+  const int64_t zlen = ((d + PR_SPLIT * PR_JC - 1) / (PR_SPLIT * PR_JC)) * PR_JC;
+  const int64_t jb = int64_t(z) * zlen;
+  const int64_t je = (jb + zlen < d) ? jb + zlen : d;
   const int64_t row = int64_t(blockIdx.x) * PR_THREADS + threadIdx.x;  // in [0, 2d)
   const bool active = row < 2 * d;
   const bool is_gram = row < d;
@@ -37,25 +45,31 @@ __global__ void __launch_bounds__(PR_THREADS) k_project_rows(const float* __rest
   float acc[KM];
 #pragma unroll
   for (int s = 0; s < KM; ++s) acc[s] = 0.f;
-  for (int64_t j0 = 0; j0 < d; j0 += PR_JC) {
+  for (int64_t j0 = jb; j0 < je; j0 += PR_JC) {
     __syncthreads();
     for (int e = threadIdx.x; e < PR_JC * KM; e += PR_THREADS) {
       const int jj = e / KM, s = e % KM;
-      As[jj][s] = (j0 + jj < d && s < k) ? Al[(j0 + jj) * k + s] : 0.f;
+      As[jj][s] = (j0 + jj < je && s < k) ? Al[(j0 + jj) * k + s] : 0.f;
     }
     __syncthreads();
     if (!active) continue;
-    const int64_t jn = (d - j0) < PR_JC ? (d - j0) : PR_JC;
+    const int64_t jn = (je - j0) < PR_JC ? (je - j0) : PR_JC;
     if (vec && jn == PR_JC) {
-#pragma unroll 2
-      for (int jj = 0; jj < PR_JC; jj += 8) {
-        const float4 m0 = __ldg(reinterpret_cast<const float4*>(M + j0 + jj));
-        const float4 m1 = __ldg(reinterpret_cast<const float4*>(M + j0 + jj + 4));
-        const float m[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
+      // 64 columns at a time: all sixteen 16-byte loads of the row stretch are issued before
+      // the multiplications, so each lane keeps 256 bytes in flight
+#pragma unroll 1
+      for (int jh = 0; jh < PR_JC; jh += 64) {
+        float4 m4[16];
 #pragma unroll
-        for (int u = 0; u < 8; ++u)
+        for (int v = 0; v < 16; ++v) m4[v] = __ldg(reinterpret_cast<const float4*>(M + j0 + jh + 4 * v));
 #pragma unroll
-          for (int s = 0; s < KM; ++s) acc[s] = fmaf(m[u], As[jj + u][s], acc[s]);
+        for (int v = 0; v < 16; ++v) {
+          const float m[4] = {m4[v].x, m4[v].y, m4[v].z, m4[v].w};
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+#pragma unroll
+            for (int s = 0; s < KM; ++s) acc[s] = fmaf(m[u], As[jh + 4 * v + u][s], acc[s]);
+        }
       }
     } else {
       for (int jj = 0; jj < jn; ++jj) {
@@ -66,7 +80,8 @@ __global__ void __launch_bounds__(PR_THREADS) k_project_rows(const float* __rest
     }
   }
   if (!active) return;
-  float* out = (is_gram ? GA : CA) + (int64_t(l) * d + i) * k;
+  const int64_t part = int64_t(z) * gridDim.y * d * k;
+  float* out = (is_gram ? GA : CA) + part + (int64_t(l) * d + i) * k;
 #pragma unroll
   for (int s = 0; s < KM; ++s)
     if (s < k) out[s] = acc[s];
@@ -78,7 +93,8 @@ constexpr int CS_ROWS = 64;  // rows of A / GA staged per step when forming G
 template <int KM>
 __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
     const float* __restrict__ GA, const float* __restrict__ CA, const float* __restrict__ A,
-    const float* __restrict__ B_prev, const double* __restrict__ xsq_total, int64_t d, int k, int L,
+    const float* __restrict__ B_prev, const double* __restrict__ xsq_total, const float* __restrict__ cross_scale,
+    int64_t d, int k, int L,
     float l0, float l1, float l2, float l3, float l4, float l5, float l6, float l7, float l8,
     float l9, float l10, float l11, float l12, float l13, float l14, float l15,
     float* __restrict__ B, int32_t* __restrict__ info, float* __restrict__ G_out,
@@ -95,6 +111,7 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
   const float* Al = A + int64_t(l) * d * k;
   const float* GAl = GA + int64_t(l) * d * k;
   const float* CAl = CA + int64_t(l) * d * k;
+  const int64_t zs = int64_t(L) * d * k;  // stride between the PR_SPLIT partial products
 
   // G_l = A_l^T GA_l: thread owns entries e = t, t + 256, ... of the KM x KM matrix
   constexpr int PER = (KM * KM + CS_THREADS - 1) / CS_THREADS;
@@ -107,7 +124,10 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
       const int ii = e / KM, s = e % KM;
       const bool ok = (i0 + ii < d) && s < k;
       As[ii][s] = ok ? Al[(i0 + ii) * k + s] : 0.f;
-      Gs[ii][s] = ok ? GAl[(i0 + ii) * k + s] : 0.f;
+      float gsum = 0.f;
+      if (ok)
+        for (int z = 0; z < PR_SPLIT; ++z) gsum += GAl[z * zs + (i0 + ii) * k + s];
+      Gs[ii][s] = gsum;
     }
     __syncthreads();
 #pragma unroll
@@ -152,10 +172,16 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
 
   float* Bj = B + (int64_t(j) * L + l) * d * k;
   const float* Bp = B_prev ? B_prev + int64_t(l) * d * k : nullptr;
+  const float cs = cross_scale != nullptr ? cross_scale[l] : 1.f;
   for (int64_t i = threadIdx.x; i < d; i += CS_THREADS) {
     float c[KM];
 #pragma unroll
-    for (int s = 0; s < KM; ++s) c[s] = (s < k) ? CAl[i * k + s] : 0.f;
+    for (int s = 0; s < KM; ++s) {
+      float csum = 0.f;
+      if (s < k)
+        for (int z = 0; z < PR_SPLIT; ++z) csum += CAl[z * zs + i * k + s];
+      c[s] = cs * csum;
+    }
     if (Bp != nullptr) {
       float b[KM];
 #pragma unroll
@@ -189,19 +215,19 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
 template <int KM>
 cudaError_t project_t(const float* gram, const float* cross, const float* A, int L, int64_t d,
                       int k, float* GA, float* CA, cudaStream_t s) {
-  const dim3 grid = dim3(unsigned((2 * d + PR_THREADS - 1) / PR_THREADS), unsigned(L));
+  const dim3 grid = dim3(unsigned((2 * d + PR_THREADS - 1) / PR_THREADS), unsigned(L), unsigned(PR_SPLIT));
   k_project_rows<KM><<<grid, PR_THREADS, 0, s>>>(gram, cross, A, d, k, GA, CA);
   return cudaGetLastError();
 }
 
 template <int KM>
 cudaError_t solve_t(const float* GA, const float* CA, const float* A, const float* B_prev,
-                    const double* xsq_total, const float* lr, int nl, int L, int64_t d, int k,
-                    float* B, int32_t* info, float* G_out, float* C_out, cudaStream_t s) {
+                    const double* xsq_total, const float* cross_scale, const float* lr, int nl, int L,
+                    int64_t d, int k, float* B, int32_t* info, float* G_out, float* C_out, cudaStream_t s) {
   float v[16] = {};
   for (int i = 0; i < nl && i < 16; ++i) v[i] = lr[i];
   const dim3 grid = dim3(unsigned(nl), unsigned(L));
-  k_chol_solve<KM><<<grid, CS_THREADS, 0, s>>>(GA, CA, A, B_prev, xsq_total, d, k, L, v[0], v[1],
+  k_chol_solve<KM><<<grid, CS_THREADS, 0, s>>>(GA, CA, A, B_prev, xsq_total, cross_scale, d, k, L, v[0], v[1],
                                                v[2], v[3], v[4], v[5], v[6], v[7], v[8], v[9],
                                                v[10], v[11], v[12], v[13], v[14], v[15], B, info,
                                                G_out, C_out);
@@ -209,6 +235,8 @@ cudaError_t solve_t(const float* GA, const float* CA, const float* A, const floa
 }
 
 }  // namespace
+
+int project_split() { return PR_SPLIT; }
 
 cudaError_t launch_project_rows(const float* gram, const float* cross, const float* A, int L,
                                 int64_t d, int k, float* GA, float* CA, cudaStream_t s) {
@@ -220,12 +248,12 @@ cudaError_t launch_project_rows(const float* gram, const float* cross, const flo
 }
 
 cudaError_t launch_chol_solve(const float* GA, const float* CA, const float* A, const float* B_prev,
-                              const double* xsq_total, const float* lambda_rel, int nl, int L,
-                              int64_t d, int k, float* B, int32_t* info, float* G_out,
+                              const double* xsq_total, const float* cross_scale, const float* lambda_rel,
+                              int nl, int L, int64_t d, int k, float* B, int32_t* info, float* G_out,
                               float* C_out, cudaStream_t s) {
-#define LOCA_SOLVE(KM)                                                                          \
-  return solve_t<KM>(GA, CA, A, B_prev, xsq_total, lambda_rel, nl, L, d, k, B, info, G_out, C_out, \
-                     s)
+#define LOCA_SOLVE(KM)                                                                               \
+  return solve_t<KM>(GA, CA, A, B_prev, xsq_total, cross_scale, lambda_rel, nl, L, d, k, B, info, G_out, \
+                     C_out, s)
   if (k <= 4) LOCA_SOLVE(4);
   if (k <= 8) LOCA_SOLVE(8);
   if (k <= 16) LOCA_SOLVE(16);

@@ -6,6 +6,9 @@
 //               loads into one fp64 partial; k_step sums the G partials in a fixed order.
 // k_step:       alpha_l = -eta sqrt(xsq_b / tsq) (= -eta_bar of Eq. 10, 0 when tsq == 0) and
 //               xsq_total[l] (+)= xsq_b.
+// k_step_from_gram: the same alpha_l and xsq_total[l] = xsq_b for a pass with one mini-batch,
+//               with xsq_b = tr(Gram_l) = ||X_l||_F^2 read off the diagonal of that batch's Gram
+//               (fp64 sum in a fixed order), so no separate read of X is needed.
 // k_gram_cross_f32: Gram_l (+)= X^T X (upper tiles, mirrored) and Cross_l (+)= alpha T^T X for
 //               fp32 inputs with fp64 accumulation: the exact-input path used for tight parity
 //               on small shapes; the bf16 path runs on the tensor cores (gram_tc.cu).
@@ -90,6 +93,28 @@ __global__ void k_step(const double* __restrict__ partials, int G, int L, const 
   const double ts = tsq[l];
   alpha[l] = ts > 0.0 ? float(-double(eta) * sqrt(xb / ts)) : 0.f;
   xsq_total[l] = (zero_first ? 0.0 : xsq_total[l]) + xb;
+}
+
+__global__ void __launch_bounds__(256) k_step_from_gram(const float* __restrict__ gram, int64_t d,
+                                                        const double* __restrict__ tsq, float eta,
+                                                        double* __restrict__ xsq_total,
+                                                        float* __restrict__ alpha) {
+  __shared__ double red[8];
+  const int l = blockIdx.x;
+  const float* Gl = gram + int64_t(l) * d * d;
+  double acc = 0.0;
+  for (int64_t j = threadIdx.x; j < d; j += 256) acc += double(Gl[j * (d + 1)]);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double xb = 0.0;
+    for (int w = 0; w < 8; ++w) xb += red[w];
+    const double ts = tsq[l];
+    alpha[l] = ts > 0.0 ? float(-double(eta) * sqrt(xb / ts)) : 0.f;
+    xsq_total[l] = xb;
+  }
 }
 
 // 64 x 64 output tile per thread block, 4 x 4 per thread, fp64 accumulators.
@@ -192,6 +217,12 @@ cudaError_t launch_gram_cross_f32(const float* X, const float* T, int L, int64_t
   const unsigned nt = unsigned((d + FT - 1) / FT);
   const dim3 grid = dim3(nt, nt, unsigned(2 * L));
   k_gram_cross_f32<<<grid, 256, 0, s>>>(X, T, N, d, alpha, zero_first, gram, cross);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_step_from_gram(const float* gram, int L, int64_t d, const double* tsq, float eta,
+                                  double* xsq_total, float* alpha, cudaStream_t s) {
+  k_step_from_gram<<<L, 256, 0, s>>>(gram, d, tsq, eta, xsq_total, alpha);
   return cudaGetLastError();
 }
 

@@ -64,7 +64,8 @@ SIGNATURES = [
      [_P, _P, ctypes.c_int, _I32, _I64, _I64, _P, ctypes.c_int, _P, _P, _P, _SZ, _P]),
     ("loca_ridge_solve_workspace_size", ctypes.c_int, [_I32, _I64, _I32, ctypes.POINTER(_SZ)]),
     ("loca_ridge_solve", ctypes.c_int,
-     [_P, _P, _P, _P, _P, ctypes.POINTER(_F), _I32, _I32, _I64, _I32, _P, _P, _P, _P, _P, _SZ, _P]),
+     [_P, _P, _P, _P, _P, _P, ctypes.POINTER(_F), _I32, _I32, _I64, _I32, _P, _P, _P, _P, _P, _SZ, _P]),
+    ("loca_step_from_gram", ctypes.c_int, [_P, _I32, _I64, _P, _F, _P, _P, _P]),
     ("loca_calib_fit_workspace_size", ctypes.c_int, [_I64, _I32, _I64, _I32, _I32, ctypes.POINTER(_SZ)]),
     ("loca_calib_fit", ctypes.c_int,
      [_P, _P, _I64, _I32, _I64, _I32, _F, _I32, _P, _P, _P, _P, _SZ, _P]),
@@ -444,10 +445,12 @@ def ridge_solve_workspace_size(L, d, k) -> int:
 
 
 def loca_ridge_solve(gram, cross, A, lambda_rel, B, info, xsq_total=None, B_prev=None, G_out=None, C_out=None,
-                     workspace=None, stream=None):
-    """Closed-form adapters ``B[j, l] = C_l (G_l + lambda_j I)^-1`` for every block and candidate."""
+                     cross_scale=None, workspace=None, stream=None):
+    """Closed-form adapters ``B[j, l] = C_l (G_l + lambda_j I)^-1`` for every block and candidate;
+    ``cross_scale`` (L, optional) multiplies ``cross_l``."""
     _dev(gram, "gram", torch.float32, 3)
     _dev(cross, "cross", torch.float32, 3)
+    _dev(cross_scale, "cross_scale", torch.float32, 1)
     _dev(A, "A", torch.float32, 3)
     _dev(B, "B", torch.float32, 4)
     _dev(info, "info", torch.int32, 2)
@@ -463,9 +466,27 @@ def loca_ridge_solve(gram, cross, A, lambda_rel, B, info, xsq_total=None, B_prev
     lam_arr = (ctypes.c_float * max(nl, 1))(*lam)
     nbytes = ridge_solve_workspace_size(L, d, k)
     ws = _workspace(nbytes, A.device, workspace)
-    rc = lib().loca_ridge_solve(_ptr(gram), _ptr(cross), _ptr(xsq_total), _ptr(A), _ptr(B_prev), lam_arr, nl, L, d,
-                                k, _ptr(B), _ptr(info), _ptr(G_out), _ptr(C_out), _ptr(ws), nbytes, _stream(stream))
+    if cross_scale is not None and tuple(cross_scale.shape) != (L,):
+        raise ValueError("cross_scale must have L entries")
+    rc = lib().loca_ridge_solve(_ptr(gram), _ptr(cross), _ptr(cross_scale), _ptr(xsq_total), _ptr(A), _ptr(B_prev),
+                                lam_arr, nl, L, d, k, _ptr(B), _ptr(info), _ptr(G_out), _ptr(C_out), _ptr(ws), nbytes,
+                                _stream(stream))
     _check(rc, "loca_ridge_solve")
+
+
+def loca_step_from_gram(gram, tsq, eta, xsq_total, alpha, stream=None):
+    """Step of Eq. 10 for a pass with one mini-batch from ``tr(gram_l) = ||X_l||^2``:
+    ``alpha[l] = -eta sqrt(tr(gram_l) / tsq[l])``, ``xsq_total[l] = tr(gram_l)``."""
+    _dev(gram, "gram", torch.float32, 3)
+    _dev(tsq, "tsq", torch.float64, 1)
+    _dev(xsq_total, "xsq_total", torch.float64, 1)
+    _dev(alpha, "alpha", torch.float32, 1)
+    L, d, d2 = gram.shape
+    if d2 != d or tuple(tsq.shape) != (L,) or tuple(xsq_total.shape) != (L,) or tuple(alpha.shape) != (L,):
+        raise ValueError("gram must be L x d x d; tsq, xsq_total, alpha must have L entries")
+    rc = lib().loca_step_from_gram(_ptr(gram), L, d, _ptr(tsq), float(eta), _ptr(xsq_total), _ptr(alpha),
+                                   _stream(stream))
+    _check(rc, "loca_step_from_gram")
 
 
 def calib_fit_workspace_size(Np, m, d, L, r) -> int:

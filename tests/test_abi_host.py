@@ -100,12 +100,15 @@ def test_validation_codes(L):
     assert b"workspace" in L.loca_last_error_string()
     # lambda_rel must be positive
     lam = (ctypes.c_float * 2)(1e-3, 0.0)
-    assert L.loca_ridge_solve(fake, fake, None, fake, None, lam, 2, 2, 64, 4, fake, fake, None, None,
+    assert L.loca_ridge_solve(fake, fake, None, None, fake, None, lam, 2, 2, 64, 4, fake, fake, None, None,
                               fake, 1 << 24, None) == 1
     # k above the supported maximum
     lam = (ctypes.c_float * 1)(1e-3)
-    assert L.loca_ridge_solve(fake, fake, None, fake, None, lam, 1, 2, 64, 33, fake, fake, None, None,
+    assert L.loca_ridge_solve(fake, fake, None, None, fake, None, lam, 1, 2, 64, 33, fake, fake, None, None,
                               fake, 1 << 24, None) == 2
+    # step from the Gram trace: L out of range, missing tsq
+    assert L.loca_step_from_gram(fake, 0, 64, fake, ctypes.c_float(0.01), fake, fake, None) == 2
+    assert L.loca_step_from_gram(fake, 2, 64, None, ctypes.c_float(0.01), fake, fake, None) == 1
     # streamed accumulate: group < 1, missing host X
     assert L.loca_accumulate_streamed(fake, fake, fake, 1, 2, 64, 64, 0, fake, ctypes.c_float(0.01), 1, fake,
                                       fake, fake, fake, 1 << 20, None) == 2

@@ -409,3 +409,70 @@ def test_end_to_end_bf16_small(lc, batches, prev):
     assert rg < 2e-3 and rc < 2e-3 and rb < 2e-3
     assert np.allclose(_np(ps.xsq), ref["xsq_total"], rtol=2e-6)
     assert lc.loca_device_status() == 0
+
+
+def _single_batch_chain(lc, w, f, X, Bp=None):
+    """error -> targets -> Gram / cross at alpha = 1 -> step from the Gram trace -> solve with
+    cross_scale = alpha: the pass with one mini-batch that reads X once (in the Gram kernel)."""
+    act = torch.bfloat16 if w.act_dtype == "bf16" else torch.float32
+    L, N, d, C, r, k = w.L, w.N, w.d, w.C, w.r, w.k
+    nl = len(w.lambda_rel)
+    f32 = dict(device="cuda", dtype=torch.float32)
+    E = torch.empty((N, C), **f32)
+    T = torch.empty((L, N, d), device="cuda", dtype=act)
+    tsq = torch.empty((L,), device="cuda", dtype=torch.float64)
+    xsq = torch.empty((L,), device="cuda", dtype=torch.float64)
+    alpha = torch.empty((L,), **f32)
+    gram = torch.empty((L, d, d), **f32)
+    cross = torch.empty((L, d, d), **f32)
+    B = torch.empty((nl, L, d, k), **f32)
+    info = torch.empty((nl, L), device="cuda", dtype=torch.int32)
+    C_out = torch.empty((L, d, k), **f32)
+    lc.loca_error(_dev(f["z"]), _dev(f["label_cols"], torch.int32), _dev(f["y"], torch.int32), E)
+    lc.loca_targets(E, _dev(f["P"]), _dev(f["Q"]), T, tsq=tsq)
+    lc.loca_gram_cross(_dev(X, act), T, torch.ones((L,), **f32), gram, cross, zero_first=True)
+    lc.loca_step_from_gram(gram, tsq, w.eta, xsq, alpha)
+    lc.loca_ridge_solve(gram, cross, _dev(f["A"]), w.lambda_rel, B, info, xsq_total=xsq,
+                        B_prev=None if Bp is None else _dev(Bp), C_out=C_out, cross_scale=alpha)
+    torch.cuda.synchronize()
+    assert lc.loca_device_status() == 0 and int(info.abs().sum()) == 0
+    return dict(xsq=_np(xsq), alpha=_np(alpha), B=_np(B), C=_np(C_out), cross=_np(cross), gram=_np(gram), tsq=_np(tsq))
+
+
+@pytest.mark.parametrize("prev", [False, True])
+def test_single_batch_chain_bf16(lc, prev):
+    """The one-mini-batch chain (step from tr(Gram), alpha applied in the solve) against the
+    oracle's pass: B and C within 2e-3, the unscaled cross product is T^T X (bf16 feed), and
+    alpha / xsq agree with the separate sum-of-squares step."""
+    w = S.scaled(S.WORKLOADS["qwen2.5-0.5b"], L=3, d=392, N=1500, C=3, V=3, r=8, k=8)
+    f = S.host_inputs(w)
+    Bp = S.host_B_prev(w) if prev else None
+    out = _single_batch_chain(lc, w, f, f["X"], Bp)
+    ref = O.loca_pass(f["z"], f["label_cols"], f["y"], f["X"].astype(np.float64), f["P"], f["Q"], f["A"], w.eta,
+                      w.lambda_rel, B_prev=Bp, t_feed="bf16")
+    assert np.allclose(out["xsq"], ref["xsq_total"], rtol=1e-5)
+    alpha_ref = -w.eta * np.sqrt(ref["xsq_total"] / ref["tsq"])
+    assert np.allclose(out["alpha"], alpha_ref, rtol=1e-5)
+    assert _rel(out["cross"] * out["alpha"][:, None, None], ref["cross"]) < 2e-3
+    assert _rel(out["C"], ref["C"]) < 2e-3
+    rb = max(_rel(out["B"][j, l], ref["B"][j, l]) for j in range(len(w.lambda_rel)) for l in range(w.L))
+    assert rb < 2e-3, rb
+    # the separate step on the same inputs gives the same alpha
+    X = _dev(f["X"], torch.bfloat16)
+    xsq2 = torch.empty((w.L,), device="cuda", dtype=torch.float64)
+    alpha2 = torch.empty((w.L,), device="cuda")
+    lc.loca_batch_step(X, _dev(out["tsq"], torch.float64), w.eta, xsq2, alpha2, True)
+    torch.cuda.synchronize()
+    assert np.allclose(out["alpha"], _np(alpha2), rtol=1e-5)
+
+
+def test_single_batch_chain_f32_tiny(lc):
+    """The same chain on the fp32 tiny workload: B within 1e-5 of the oracle (the trace is read
+    from the fp32-stored Gram diagonal, ~1e-7 relative)."""
+    w = S.WORKLOADS["tiny"]
+    f = S.host_inputs(w)
+    out = _single_batch_chain(lc, w, f, f["X"])
+    ref = O.loca_pass(f["z"], f["label_cols"], f["y"], f["X"].astype(np.float64), f["P"], f["Q"], f["A"], w.eta,
+                      w.lambda_rel)
+    assert np.allclose(out["xsq"], ref["xsq_total"], rtol=1e-6)
+    assert _rel(out["B"], ref["B"]) < 1e-5
