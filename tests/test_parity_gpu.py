@@ -476,3 +476,32 @@ def test_single_batch_chain_f32_tiny(lc):
                       w.lambda_rel)
     assert np.allclose(out["xsq"], ref["xsq_total"], rtol=1e-6)
     assert _rel(out["B"], ref["B"]) < 1e-5
+
+
+def test_step_from_gram_with_zero_targets(lc):
+    """tsq = 0 (zero feedback, T = 0): the step is 0 (Eq. 10's convention), the trace still gives
+    ||X||^2, and the solve with that cross_scale leaves C = B_prev G."""
+    L, N, d, k = 2, 512, 128, 8
+    X, _ = _synthetic_stats_inputs(L, N, d, "bf16", seed=10)
+    Xd = _dev(X, torch.bfloat16)
+    gram = torch.empty((L, d, d), device="cuda")
+    cross = torch.empty_like(gram)
+    lc.loca_gram_cross(Xd, torch.zeros_like(Xd), torch.ones((L,), device="cuda"), gram, cross, zero_first=True)
+    tsq = torch.zeros((L,), dtype=torch.float64, device="cuda")
+    xsq = torch.empty((L,), dtype=torch.float64, device="cuda")
+    alpha = torch.full((L,), 7.0, device="cuda")
+    lc.loca_step_from_gram(gram, tsq, 0.01, xsq, alpha)
+    A = _dev(np.linalg.qr(np.random.default_rng(3).standard_normal((d, k)))[0][None].repeat(L, 0))
+    Bp = _dev(0.01 * np.random.default_rng(4).standard_normal((L, d, k)))
+    B = torch.empty((1, L, d, k), device="cuda")
+    info = torch.empty((1, L), dtype=torch.int32, device="cuda")
+    G_out = torch.empty((L, k, k), device="cuda")
+    C_out = torch.empty((L, d, k), device="cuda")
+    lc.loca_ridge_solve(gram, cross, A, [1e-3], B, info, xsq_total=xsq, B_prev=Bp, G_out=G_out, C_out=C_out,
+                        cross_scale=alpha)
+    torch.cuda.synchronize()
+    assert torch.count_nonzero(alpha) == 0
+    x64 = X.astype(np.float64)
+    assert np.allclose(_np(xsq), (x64 ** 2).sum(axis=(1, 2)), rtol=1e-5)
+    C_ref = np.einsum("ldk,lkj->ldj", _np(Bp).astype(np.float64), _np(G_out).astype(np.float64))
+    assert _rel(_np(C_out), C_ref) < 1e-5
