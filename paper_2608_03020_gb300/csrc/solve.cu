@@ -2,11 +2,12 @@
 //
 // k_project_rows  GA_l = Gram_l A_l, CA_l = Cross_l A_l (d x k each), as PR_SPLIT partial
 //                 products over quarters of the column range (GA = sum_z GA_z, summed in a fixed
-//                 order by k_chol_solve).  One thread per row of the stacked [Gram_l; Cross_l] and
-//                 column quarter; each thread streams its stretch of the row with 32-byte loads
-//                 while the block shares A_l through shared memory (broadcast reads).  The split
-//                 gives 4x as many, 4x shorter CTAs, so the last wave is small.  Bound: the HBM
-//                 read of Gram and Cross (8 d^2 bytes per block), k fp32 FMAs per element read.
+//                 order by k_chol_solve).  A CTA takes 256 rows of the stacked [Gram_l; Cross_l]
+//                 and one column quarter; 32-column slabs of its rows are staged in shared memory
+//                 by row-contiguous 16-byte loads (a warp request covers 4 rows, so L1 sees 4
+//                 lines per request, not 32), then each thread forms a register block of
+//                 RPT rows x SPT columns of the product with A's slab (broadcast reads).  Bound: the
+//                 HBM read of Gram and Cross (8 d^2 bytes per block).
 // k_chol_solve    one thread block per (ridge candidate j, block l):
 //                 G_l = A_l^T GA_l (k x k), lambda from the trace, Cholesky of G_l + lambda I in
 //                 fp64 in shared memory, then every row i of C_l = B_prev,l G_l + s_l CA_l
@@ -21,70 +22,104 @@ namespace loca {
 namespace {
 
 constexpr int PR_THREADS = 256;
-constexpr int PR_JC = 128;  // columns of A staged per step
-constexpr int PR_SPLIT = 4;  // column ranges per row (partial products)
+constexpr int PR_ROWS = 256;   // rows per CTA
+constexpr int PR_JC = 32;      // columns per staged slab
+constexpr int PR_LD = PR_JC + 4;
+constexpr int PR_SPLIT = 4;    // column ranges per row (partial products)
 
 template <int KM>
-__global__ void __launch_bounds__(PR_THREADS) k_project_rows(const float* __restrict__ gram,
+__global__ void __launch_bounds__(PR_THREADS, KM <= 16 ? 3 : 1) k_project_rows(const float* __restrict__ gram,
                                                             const float* __restrict__ cross,
                                                             const float* __restrict__ A, int64_t d,
                                                             int k, float* __restrict__ GA,
                                                             float* __restrict__ CA) {
-  __shared__ float As[PR_JC][KM];
-  const int l = blockIdx.y, z = blockIdx.z;
+  constexpr int SPT = KM < 8 ? KM : 8;         // product columns per thread
+  constexpr int G = KM / SPT;                  // column groups
+  constexpr int RPT = PR_ROWS * G / PR_THREADS;  // rows per thread
+  constexpr int RS = PR_ROWS / RPT;            // row stride between a thread's rows
+  extern __shared__ __align__(16) float pr_smem[];
+  float* Ms = pr_smem;                          // PR_ROWS x PR_LD
+  float* As = pr_smem + PR_ROWS * PR_LD;        // PR_JC x KM
+  const int l = blockIdx.y, z = blockIdx.z, tid = threadIdx.x;
   const int64_t zlen = ((d + PR_SPLIT * PR_JC - 1) / (PR_SPLIT * PR_JC)) * PR_JC;
   const int64_t jb = int64_t(z) * zlen;
   const int64_t je = (jb + zlen < d) ? jb + zlen : d;
-  const int64_t row = int64_t(blockIdx.x) * PR_THREADS + threadIdx.x;  // in [0, 2d)
-  const bool active = row < 2 * d;
-  const bool is_gram = row < d;
-  const int64_t i = is_gram ? row : row - d;
-  const float* M = (is_gram ? gram : cross) + int64_t(l) * d * d + (active ? i * d : 0);
+  const int64_t row0 = int64_t(blockIdx.x) * PR_ROWS;  // in the stacked [Gram; Cross], 2d rows
   const float* Al = A + int64_t(l) * d * k;
   const bool vec = (d % 4 == 0);
-  float acc[KM];
+  const int g = tid % G, rs = tid / G;
+  float acc[RPT][SPT];
 #pragma unroll
-  for (int s = 0; s < KM; ++s) acc[s] = 0.f;
-  for (int64_t j0 = jb; j0 < je; j0 += PR_JC) {
-    __syncthreads();
-    for (int e = threadIdx.x; e < PR_JC * KM; e += PR_THREADS) {
-      const int jj = e / KM, s = e % KM;
-      As[jj][s] = (j0 + jj < je && s < k) ? Al[(j0 + jj) * k + s] : 0.f;
-    }
-    __syncthreads();
-    if (!active) continue;
-    const int64_t jn = (je - j0) < PR_JC ? (je - j0) : PR_JC;
-    if (vec && jn == PR_JC) {
-      // 64 columns at a time: all sixteen 16-byte loads of the row stretch are issued before
-      // the multiplications, so each lane keeps 256 bytes in flight
-#pragma unroll 1
-      for (int jh = 0; jh < PR_JC; jh += 64) {
-        float4 m4[16];
+  for (int i = 0; i < RPT; ++i)
 #pragma unroll
-        for (int v = 0; v < 16; ++v) m4[v] = __ldg(reinterpret_cast<const float4*>(M + j0 + jh + 4 * v));
+    for (int s = 0; s < SPT; ++s) acc[i][s] = 0.f;
+  // each thread moves PR_LOADS 16-byte pieces of a slab: all are loaded into registers before any
+  // is stored, and the next slab's loads are in flight while the current one is multiplied
+  constexpr int PR_LOADS = PR_ROWS * (PR_JC / 4) / PR_THREADS;
+  float4 pre[PR_LOADS];
+  auto gload = [&](int64_t j0) {
+    const int jn = int((je - j0) < PR_JC ? (je - j0) : PR_JC);
 #pragma unroll
-        for (int v = 0; v < 16; ++v) {
-          const float m[4] = {m4[v].x, m4[v].y, m4[v].z, m4[v].w};
-#pragma unroll
-          for (int u = 0; u < 4; ++u)
-#pragma unroll
-            for (int s = 0; s < KM; ++s) acc[s] = fmaf(m[u], As[jh + 4 * v + u][s], acc[s]);
+    for (int it = 0; it < PR_LOADS; ++it) {
+      const int e = tid + it * PR_THREADS;
+      const int rr = e / (PR_JC / 4), c4 = (e % (PR_JC / 4)) * 4;
+      const int64_t row = row0 + rr;
+      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (row < 2 * d) {
+        const float* M = (row < d ? gram + int64_t(l) * d * d + row * d
+                                  : cross + int64_t(l) * d * d + (row - d) * d) + j0 + c4;
+        if (vec && c4 + 4 <= jn) {
+          v = __ldg(reinterpret_cast<const float4*>(M));
+        } else {
+          if (c4 + 0 < jn) v.x = M[0];
+          if (c4 + 1 < jn) v.y = M[1];
+          if (c4 + 2 < jn) v.z = M[2];
+          if (c4 + 3 < jn) v.w = M[3];
         }
       }
-    } else {
-      for (int jj = 0; jj < jn; ++jj) {
-        const float m = M[j0 + jj];
+      pre[it] = v;
+    }
+  };
+  if (jb < je) gload(jb);
+  for (int64_t j0 = jb; j0 < je; j0 += PR_JC) {
+    const int jn = int((je - j0) < PR_JC ? (je - j0) : PR_JC);
+    __syncthreads();  // the previous slab's products are done with Ms and As
 #pragma unroll
-        for (int s = 0; s < KM; ++s) acc[s] = fmaf(m, As[jj][s], acc[s]);
+    for (int it = 0; it < PR_LOADS; ++it) {
+      const int e = tid + it * PR_THREADS;
+      *reinterpret_cast<float4*>(&Ms[(e / (PR_JC / 4)) * PR_LD + (e % (PR_JC / 4)) * 4]) = pre[it];
+    }
+    for (int e = tid; e < PR_JC * KM; e += PR_THREADS) {
+      const int jj = e / KM, s = e % KM;
+      As[e] = (jj < jn && s < k) ? Al[(j0 + jj) * k + s] : 0.f;
+    }
+    __syncthreads();
+    if (j0 + PR_JC < je) gload(j0 + PR_JC);
+#pragma unroll 4
+    for (int jj = 0; jj < PR_JC; ++jj) {
+      float av[SPT];
+#pragma unroll
+      for (int s = 0; s < SPT; ++s) av[s] = As[jj * KM + g * SPT + s];
+#pragma unroll
+      for (int i = 0; i < RPT; ++i) {
+        const float m = Ms[(rs + RS * i) * PR_LD + jj];
+#pragma unroll
+        for (int s = 0; s < SPT; ++s) acc[i][s] = fmaf(m, av[s], acc[i][s]);
       }
     }
   }
-  if (!active) return;
   const int64_t part = int64_t(z) * gridDim.y * d * k;
-  float* out = (is_gram ? GA : CA) + part + (int64_t(l) * d + i) * k;
 #pragma unroll
-  for (int s = 0; s < KM; ++s)
-    if (s < k) out[s] = acc[s];
+  for (int i = 0; i < RPT; ++i) {
+    const int64_t row = row0 + rs + RS * i;
+    if (row >= 2 * d) continue;
+    const bool is_gram = row < d;
+    const int64_t ri = is_gram ? row : row - d;
+    float* out = (is_gram ? GA : CA) + part + (int64_t(l) * d + ri) * k;
+#pragma unroll
+    for (int s = 0; s < SPT; ++s)
+      if (g * SPT + s < k) out[g * SPT + s] = acc[i][s];
+  }
 }
 
 constexpr int CS_THREADS = 256;
@@ -176,12 +211,16 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
   for (int64_t i = threadIdx.x; i < d; i += CS_THREADS) {
     float c[KM];
 #pragma unroll
-    for (int s = 0; s < KM; ++s) {
-      float csum = 0.f;
-      if (s < k)
-        for (int z = 0; z < PR_SPLIT; ++z) csum += CAl[z * zs + i * k + s];
-      c[s] = cs * csum;
+    for (int s = 0; s < KM; ++s) c[s] = 0.f;
+#pragma unroll 1
+    for (int z = 0; z < PR_SPLIT; ++z) {
+      const float* cz = CAl + z * zs + i * k;
+#pragma unroll
+      for (int s = 0; s < KM; ++s)
+        if (s < k) c[s] += cz[s];
     }
+#pragma unroll
+    for (int s = 0; s < KM; ++s) c[s] *= cs;
     if (Bp != nullptr) {
       float b[KM];
 #pragma unroll
@@ -215,8 +254,11 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
 template <int KM>
 cudaError_t project_t(const float* gram, const float* cross, const float* A, int L, int64_t d,
                       int k, float* GA, float* CA, cudaStream_t s) {
-  const dim3 grid = dim3(unsigned((2 * d + PR_THREADS - 1) / PR_THREADS), unsigned(L), unsigned(PR_SPLIT));
-  k_project_rows<KM><<<grid, PR_THREADS, 0, s>>>(gram, cross, A, d, k, GA, CA);
+  const dim3 grid = dim3(unsigned((2 * d + PR_ROWS - 1) / PR_ROWS), unsigned(L), unsigned(PR_SPLIT));
+  const size_t smem = sizeof(float) * (size_t(PR_ROWS) * PR_LD + size_t(PR_JC) * KM);
+  cudaError_t e = cudaFuncSetAttribute(k_project_rows<KM>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  if (e != cudaSuccess) return e;
+  k_project_rows<KM><<<grid, PR_THREADS, smem, s>>>(gram, cross, A, d, k, GA, CA);
   return cudaGetLastError();
 }
 
