@@ -315,6 +315,7 @@ def test_host_empty_is_pinned_zeroed_and_freed(lc):
     (8, 200, 3, True, True),
     (16, 328, 2, True, False),
     (32, 96, 2, False, True),
+    (32, 520, 2, True, True),
     (1, 16, 1, True, True),
 ])
 def test_ridge_solve_parity(lc, k, d, L, with_prev, relative):
