@@ -208,6 +208,76 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
   float* Bj = B + (int64_t(j) * L + l) * d * k;
   const float* Bp = B_prev ? B_prev + int64_t(l) * d * k : nullptr;
   const float cs = cross_scale != nullptr ? cross_scale[l] : 1.f;
+  if constexpr (KM == 32) {
+    // one warp per row, lane s holding entry s: 32 values per thread do not fit in registers
+    // next to the unrolled substitutions, so they move between lanes by shuffles instead
+    __shared__ float Lp[KM][KM + 1];  // Lf with a padded row: column reads without bank conflicts
+    for (int e = threadIdx.x; e < KM * KM; e += CS_THREADS) Lp[e / KM][e % KM] = Lf[e / KM][e % KM];
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    const bool on = lane < k;
+    constexpr int RW = 4;  // rows per warp at a time: four independent shuffle chains
+    for (int64_t i0 = int64_t(threadIdx.x >> 5) * RW; i0 < d; i0 += (CS_THREADS / 32) * RW) {
+      float c[RW];
+#pragma unroll
+      for (int r = 0; r < RW; ++r) {
+        const int64_t i = i0 + r;
+        float v = 0.f;
+        if (on && i < d)
+          for (int z = 0; z < PR_SPLIT; ++z) v += CAl[z * zs + i * k + lane];
+        c[r] = v * cs;
+      }
+      if (Bp != nullptr) {
+        float bl[RW];
+#pragma unroll
+        for (int r = 0; r < RW; ++r) bl[r] = (on && i0 + r < d) ? Bp[(i0 + r) * k + lane] : 0.f;
+#pragma unroll
+        for (int t = 0; t < KM; ++t) {
+          const float g = Gf[t][lane];
+#pragma unroll
+          for (int r = 0; r < RW; ++r) c[r] = fmaf(__shfl_sync(0xffffffffu, bl[r], t), g, c[r]);
+        }
+#pragma unroll
+        for (int r = 0; r < RW; ++r)
+          if (!on) c[r] = 0.f;
+      }
+      if (C_out != nullptr && j == 0 && on)
+#pragma unroll
+        for (int r = 0; r < RW; ++r)
+          if (i0 + r < d) C_out[(int64_t(l) * d + i0 + r) * k + lane] = c[r];
+      if (inf != 0) {
+#pragma unroll
+        for (int r = 0; r < RW; ++r)
+          if (on && i0 + r < d) Bj[(i0 + r) * k + lane] = 0.f;
+        continue;
+      }
+      // c <- c (L L^T)^-1: forward L y = c^T, then L^T x = y
+#pragma unroll
+      for (int t = 0; t < KM; ++t) {
+        const float lt = Lp[lane][t], it = Linv[t];
+#pragma unroll
+        for (int r = 0; r < RW; ++r) {
+          if (lane == t) c[r] *= it;
+          const float yt = __shfl_sync(0xffffffffu, c[r], t);
+          if (lane > t) c[r] = fmaf(-lt, yt, c[r]);
+        }
+      }
+#pragma unroll
+      for (int t = KM - 1; t >= 0; --t) {
+        const float lt = Lp[t][lane], it = Linv[t];
+#pragma unroll
+        for (int r = 0; r < RW; ++r) {
+          if (lane == t) c[r] *= it;
+          const float xt = __shfl_sync(0xffffffffu, c[r], t);
+          if (lane < t) c[r] = fmaf(-lt, xt, c[r]);
+        }
+      }
+#pragma unroll
+      for (int r = 0; r < RW; ++r)
+        if (on && i0 + r < d) Bj[(i0 + r) * k + lane] = c[r];
+    }
+    return;
+  }
   for (int64_t i = threadIdx.x; i < d; i += CS_THREADS) {
     float c[KM];
 #pragma unroll
