@@ -56,9 +56,17 @@ __global__ void __launch_bounds__(PR_THREADS, KM <= 16 ? 3 : 1) k_project_rows(c
   // each thread moves PR_LOADS 16-byte pieces of a slab: all are loaded into registers before any
   // is stored, and the next slab's loads are in flight while the current one is multiplied
   constexpr int PR_LOADS = PR_ROWS * (PR_JC / 4) / PR_THREADS;
+  constexpr int PR_ALOADS = (PR_JC * KM + PR_THREADS - 1) / PR_THREADS;
   float4 pre[PR_LOADS];
+  float apre[PR_ALOADS];
   auto gload = [&](int64_t j0) {
     const int jn = int((je - j0) < PR_JC ? (je - j0) : PR_JC);
+#pragma unroll
+    for (int it = 0; it < PR_ALOADS; ++it) {
+      const int e = tid + it * PR_THREADS;
+      const int jj = e / KM, s = e % KM;
+      apre[it] = (e < PR_JC * KM && jj < jn && s < k) ? __ldg(Al + (j0 + jj) * k + s) : 0.f;
+    }
 #pragma unroll
     for (int it = 0; it < PR_LOADS; ++it) {
       const int e = tid + it * PR_THREADS;
@@ -82,16 +90,16 @@ __global__ void __launch_bounds__(PR_THREADS, KM <= 16 ? 3 : 1) k_project_rows(c
   };
   if (jb < je) gload(jb);
   for (int64_t j0 = jb; j0 < je; j0 += PR_JC) {
-    const int jn = int((je - j0) < PR_JC ? (je - j0) : PR_JC);
     __syncthreads();  // the previous slab's products are done with Ms and As
 #pragma unroll
     for (int it = 0; it < PR_LOADS; ++it) {
       const int e = tid + it * PR_THREADS;
       *reinterpret_cast<float4*>(&Ms[(e / (PR_JC / 4)) * PR_LD + (e % (PR_JC / 4)) * 4]) = pre[it];
     }
-    for (int e = tid; e < PR_JC * KM; e += PR_THREADS) {
-      const int jj = e / KM, s = e % KM;
-      As[e] = (jj < jn && s < k) ? Al[(j0 + jj) * k + s] : 0.f;
+#pragma unroll
+    for (int it = 0; it < PR_ALOADS; ++it) {
+      const int e = tid + it * PR_THREADS;
+      if (e < PR_JC * KM) As[e] = apre[it];
     }
     __syncthreads();
     if (j0 + PR_JC < je) gload(j0 + PR_JC);
