@@ -32,6 +32,9 @@
 // L2 no longer holds what the others read, and the load latency, not the tensor core, sets the
 // pace (about 1.25x slower at 7B size); the points within items keep the clusters' token windows
 // within ~L2 of each other (HBM re-reads 4.0x -> 2.6x of X and T, 3-4% faster under the power cap).
+// Rounds are aligned to blocks: the items are ordered so that a round holds the items of one block
+// only, each block filling whole rounds, and the few items left of every block follow at the end;
+// a round then streams one block's tiles instead of parts of two.
 // Every mbarrier wait is bounded: on expiry the status word gets LOCA_ERR_TIMEOUT, a launch-local
 // flag makes every other wait give up, the even CTA drains the loads and MMAs in flight, and
 // both CTAs meet at the final cluster barrier before TMEM is freed.
@@ -72,6 +75,7 @@ struct Geo {
   int L, d, N;
   int nM, nN;       // 256-row tiles and 256-column tiles
   int per_block;    // work items per block l
+  int full;         // items of each block that fill whole rounds of their own (0: plain order)
 };
 
 // Gram row tiles of column tile nt that contain an element with row <= column.
@@ -92,10 +96,24 @@ struct Item {
   int mt[2];    // 256-row tile index
 };
 
+// Round-aligned order: a round is the items cid + round * (clusters).  The first `full` items of
+// block l (a multiple of the cluster count) fill rounds of block l alone, so a round streams the
+// tiles of one block; the per_block - full items left of every block come after all blocks.
 __device__ __forceinline__ Item decode(const Geo& g, int it) {
   Item r;
-  r.l = it / g.per_block;
-  int rem = it - r.l * g.per_block;
+  int rem;
+  if (g.full > 0 && it < g.L * g.full) {
+    r.l = it / g.full;
+    rem = it - r.l * g.full;
+  } else if (g.full > 0) {
+    const int q = g.per_block - g.full;  // > 0 here: it < L * per_block
+    const int j = it - g.L * g.full;
+    r.l = j / q;
+    rem = g.full + (j - r.l * q);
+  } else {
+    r.l = it / g.per_block;
+    rem = it - r.l * g.per_block;
+  }
   int nt = 0;
   for (;; ++nt) {
     const int c = items_of_col(g, nt);
@@ -441,6 +459,7 @@ cudaError_t launch_gram_cross_tc(const void* X, const void* T, int L, int64_t N,
   g.nM = int((d + BMP - 1) / BMP);
   g.nN = int((d + BN - 1) / BN);
   g.per_block = 0;
+  g.full = 0;
   for (int nt = 0; nt < g.nN; ++nt) g.per_block += items_of_col(g, nt);
   const int total = g.per_block * L;
   cudaError_t e = cudaFuncSetAttribute(k_gram_cross_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -451,6 +470,7 @@ cudaError_t launch_gram_cross_tc(const void* X, const void* T, int L, int64_t N,
   int clusters = clusters_cached;
   if (clusters > total) clusters = total;
   if (clusters < 1) clusters = 1;
+  g.full = (g.per_block / clusters) * clusters;
   // abort flag and round counter (two int32 of the launch-local flag area)
   e = cudaMemsetAsync(abort_flag, 0, 2 * sizeof(int32_t), s);
   if (e != cudaSuccess) return e;
