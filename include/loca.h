@@ -194,12 +194,15 @@ int loca_accumulate_streamed(const void* X_host, void* staging, const void* T, i
  * the cosine between the stacked feedback predictions and the stacked exact hidden-state
  * gradients at the probe positions (0 when either is zero).  Random feedback gives ~0; the
  * paper reports 0.3-0.5 after calibration.
- *   E_probe  Np x m float (m <= 64);  G_probe  L x Np x d float;  P  L x m x r, Q  L x r x d float
- *   (r <= 32);  alpha  L double (output).  Workspace: loca_alignment_workspace_size.
+ *   E_probe  Np x m float (m <= 16384);  G_probe  L x Np x d float;  P  L x m x r,
+ *   Q  L x r x d float (r <= 32);  alpha  L double (output).
+ *   Workspace: loca_alignment_workspace_size (partial sums; for m > 64, the paper's d-wide
+ *   error space, also U_l = E_probe P_l, L x Np x r float, formed first).
  *   T is formed in registers and never written; sums in fp32 per thread over 1024 tokens,
  *   fp64 across, in a fixed order (deterministic).
  */
-int loca_alignment_workspace_size(int64_t Np, int64_t d, int32_t L, size_t* bytes /* host */);
+int loca_alignment_workspace_size(int64_t Np, int32_t m, int64_t d, int32_t L, int32_t r,
+                                  size_t* bytes /* host */);
 int loca_alignment(const float* E_probe, const float* G_probe, int64_t Np, int32_t m, int64_t d,
                    int32_t L, const float* P, const float* Q, int32_t r, double* alpha,
                    void* workspace, size_t workspace_bytes, void* stream);

@@ -450,10 +450,11 @@ int loca_accumulate_streamed(const void* X_host, void* staging, const void* T, i
   return LOCA_OK;
 }
 
-int loca_alignment_workspace_size(int64_t Np, int64_t d, int32_t L, size_t* bytes) {
+int loca_alignment_workspace_size(int64_t Np, int32_t m, int64_t d, int32_t L, int32_t r, size_t* bytes) {
   if (!bytes) return fail(LOCA_ERR_INVALID_ARG, "bytes is NULL");
-  if (Np < 0 || d < 1 || L < 1) return fail(LOCA_ERR_SHAPE, "need Np >= 0, d >= 1, L >= 1");
-  *bytes = align_workspace_bytes(Np, d, L);
+  if (Np < 0 || m < 1 || d < 1 || L < 1 || r < 1)
+    return fail(LOCA_ERR_SHAPE, "need Np >= 0, m, d, L, r >= 1");
+  *bytes = align_workspace_bytes(Np, m, d, L, r);
   return LOCA_OK;
 }
 
@@ -470,7 +471,7 @@ int loca_alignment(const float* E_probe, const float* G_probe, int64_t Np, int32
   if ((E_probe && !aligned(E_probe, 4)) || (G_probe && !aligned(G_probe, 4)) || !aligned(P, 4) || !aligned(Q, 4) ||
       !aligned(alpha, 8))
     return fail(LOCA_ERR_ALIGNMENT, "pointers must be aligned to their element size");
-  const int rc = check_ws(workspace, workspace_bytes, align_workspace_bytes(Np, d, L));
+  const int rc = check_ws(workspace, workspace_bytes, align_workspace_bytes(Np, m, d, L, r));
   if (rc != LOCA_OK) return rc;
   cudaError_t e = launch_alignment(E_probe, G_probe, Np, m, d, L, P, Q, r, alpha, workspace,
                                    static_cast<cudaStream_t>(stream));

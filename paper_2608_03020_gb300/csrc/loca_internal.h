@@ -72,7 +72,7 @@ unsigned long long wait_limit_ns();
 // ---- alignment diagnostic (align.cu)
 int align_max_m();
 int align_max_r();
-size_t align_workspace_bytes(int64_t Np, int64_t d, int L);
+size_t align_workspace_bytes(int64_t Np, int m, int64_t d, int L, int r);
 cudaError_t launch_alignment(const float* E, const float* G, int64_t Np, int m, int64_t d, int L, const float* P,
                              const float* Q, int r, double* alpha, void* workspace, cudaStream_t s);
 

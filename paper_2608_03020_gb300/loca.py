@@ -47,7 +47,7 @@ SIGNATURES = [
      [_P, _P, ctypes.c_int, _I32, _I64, _I64, _P, _F, ctypes.c_int, _P, _P, _P, _P]),
     ("loca_accumulate_streamed", ctypes.c_int,
      [_P, _P, _P, ctypes.c_int, _I32, _I64, _I64, _I32, _P, _F, ctypes.c_int, _P, _P, _P, _P, _SZ, _P]),
-    ("loca_alignment_workspace_size", ctypes.c_int, [_I64, _I64, _I32, ctypes.POINTER(_SZ)]),
+    ("loca_alignment_workspace_size", ctypes.c_int, [_I64, _I32, _I64, _I32, _I32, ctypes.POINTER(_SZ)]),
     ("loca_alignment", ctypes.c_int, [_P, _P, _I64, _I32, _I64, _I32, _P, _P, _I32, _P, _P, _SZ, _P]),
     ("loca_kspace_workspace_size", ctypes.c_int, [_I32, _I64, _I64, _I32, _I32, _I32, ctypes.POINTER(_SZ)]),
     ("loca_kspace_accumulate", ctypes.c_int,
@@ -328,7 +328,7 @@ def loca_alignment(E_probe, G_probe, P, Q, alpha, workspace=None, stream=None):
             or alpha.numel() != L):
         raise ValueError("shape mismatch among E_probe, G_probe, P, Q, alpha")
     out = ctypes.c_size_t(0)
-    _check(lib().loca_alignment_workspace_size(Np, d, L, ctypes.byref(out)), "loca_alignment_workspace_size")
+    _check(lib().loca_alignment_workspace_size(Np, m, d, L, r, ctypes.byref(out)), "loca_alignment_workspace_size")
     ws = _workspace(out.value, G_probe.device, workspace)
     rc = lib().loca_alignment(_ptr(E_probe), _ptr(G_probe), Np, m, d, L, _ptr(P), _ptr(Q), r, _ptr(alpha), _ptr(ws),
                               out.value, _stream(stream))

@@ -148,10 +148,12 @@ def test_calib_reports_beta_below_rounding(lc):
         assert torch.count_nonzero(P) == 0 and torch.count_nonzero(Q) == 0
 
 
-@pytest.mark.parametrize("Np,m,d,L,r", [(3000, 4, 328, 3, 4), (1500, 16, 1024, 2, 16), (700, 64, 96, 1, 32)])
+@pytest.mark.parametrize("Np,m,d,L,r", [(3000, 4, 328, 3, 4), (1500, 16, 1024, 2, 16), (700, 64, 96, 1, 32),
+                                         (700, 65, 96, 1, 32), (1500, 200, 256, 2, 8), (2048, 1024, 512, 2, 16)])
 def test_alignment_matches_oracle(lc, Np, m, d, L, r):
     """Supplement, one-shot calibration: the in-probe cosine of each block against the oracle's.
-    fp32 products summed in fp32 over 1024 tokens per thread, fp64 across: relative 1e-5."""
+    fp32 products summed in fp32 over 1024 tokens per thread, fp64 across: relative 1e-5.  Error
+    widths above 64 (the paper's d-wide e) go through U_l = E P_l formed first."""
     rng = np.random.default_rng(Np + d)
     E = rng.standard_normal((Np, m)).astype(np.float32)
     P = rng.standard_normal((L, m, r)).astype(np.float32)
