@@ -87,11 +87,13 @@ def hbm_peak():
 
 
 class ClockSampler:
-    """nvidia-smi samples (200 ms) of SM clock and throttle reasons during the timed region."""
+    """nvidia-smi samples (200 ms) of SM and memory clocks, power and throttle reasons during the
+    timed region (read only)."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap,"
+              "clocks.mem,clocks.max.mem")
 
     def __init__(self, uuid):
         self.uuid = uuid
@@ -123,7 +125,7 @@ class ClockSampler:
     def summary(self):
         if self.proc is None or self.path is None:
             return None
-        rows = []
+        rows, extra = [], []
         for line in open(self.path):
             parts = [p.strip() for p in line.split(",")]
             if len(parts) < 9:
@@ -132,13 +134,21 @@ class ClockSampler:
                 rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
             except ValueError:
                 continue
+            try:
+                extra.append((float(parts[3]), float(parts[9]), float(parts[10])))
+            except (ValueError, IndexError):
+                pass
         os.unlink(self.path)
         if not rows:
             return None
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         reasons = sorted({names[i] for _, _, flags in rows for i, v in enumerate(flags) if v.lower() == "active"})
-        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
-                "reasons": reasons, "samples": len(rows)}
+        out = {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+               "reasons": reasons, "samples": len(rows)}
+        if extra:
+            out.update({"power_w": statistics.median(e[0] for e in extra),
+                        "mem_mhz": statistics.median(e[1] for e in extra), "mem_max_mhz": max(e[2] for e in extra)})
+        return out
 
 
 def dist_setup(args):
