@@ -46,8 +46,8 @@ FALLBACK_SUSTAINED_TFLOPS = 1700.0  # profiling recipe's sustained figure, used 
 # dram bytes (read + write) per launch of k_gram_cross_tc from a one-pass ncu capture of this
 # workload (profiles/gram_cross_tc_qwen2.5-7b.md), valid only for the kernel source whose sha256
 # prefix is given and for the captured (L, N, d); otherwise traffic is reported as null
-GRAM_TC_TRAFFIC = {"sha256": "1fabb85b0d95522b", "L": 28, "N": 131072, "d": 3584,
-                   "read": 106725806080, "write": 3014179584,
+GRAM_TC_TRAFFIC = {"sha256": "e55b0d4848cbeaee", "L": 28, "N": 131072, "d": 3584,
+                   "read": 103600324352, "write": 3014398208,
                    "source": "profiles/gram_cross_tc_qwen2.5-7b.md"}
 
 

@@ -57,7 +57,7 @@ constexpr int BN = 256;                             // accumulator columns (chan
 constexpr int BNC = 128;                            // B columns loaded per CTA
 constexpr int BK = 64;                              // tokens per pipeline stage
 constexpr int STAGES = 4;
-constexpr int kSyncEvery = 128;                     // k-blocks between lockstep sync points
+constexpr int kSyncEvery = 64;                     // k-blocks between lockstep sync points
 constexpr int SUB_BYTES = 64 * BK * 2;              // one 64-channel x 64-token swizzled tile (8 KB)
 constexpr int A_BYTES = BMC * BK * 2;               // 16 KB
 constexpr int B_BYTES = BNC * BK * 2;               // 16 KB
