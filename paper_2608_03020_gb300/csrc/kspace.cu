@@ -82,7 +82,13 @@ __global__ void __launch_bounds__(PREP_THREADS) k_kspace_prep(const float* __res
 }
 
 // ------------------------------------------------------------------ X A on the tensor cores
-constexpr int XA_THREADS = 256;  // producer, MMA, 4 TMEM / statistics warps, 2 sum-of-squares warps
+// warps: producer, MMA, 4 TMEM / statistics warps, then the sum-of-squares warps, which share the
+// 128 token rows of each stage and own one of the CTA's four partial slots of ||x||^2 each.  Four
+// of them (one row per lane) keep up with the TMA ring at kp = 16; at kp = 32 the statistics warps'
+// registers leave room for only two in one CTA per SM without spills.
+__host__ __device__ constexpr int xa_sq_warps(int kp) { return kp <= 16 ? 4 : 2; }
+__host__ __device__ constexpr int xa_threads(int kp) { return 32 * (6 + xa_sq_warps(kp)); }
+static_assert(xa_sq_warps(16) <= 4 && xa_sq_warps(32) <= 4, "four partial slots per CTA");
 constexpr int XA_TM = 128;          // tokens per tile (TMEM lanes)
 constexpr int XA_BK = 64;           // channels per stage (one 128-byte swizzle row)
 constexpr int XA_STAGES = 8;
@@ -100,12 +106,14 @@ __host__ __device__ constexpr int part_stride(int kp, int C) { return ntri(kp) +
 constexpr int XA_SMEM = XA_STAGES * XA_STAGE + 1024 + 256 + XA_EPI_SMEM;
 
 template <int KP>
-__global__ void __launch_bounds__(XA_THREADS, 1)
+__global__ void __launch_bounds__(xa_threads(KP), 1)
     k_kspace_xa(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW, int L,
                 int64_t N, int64_t d, int ntiles, const float* __restrict__ E, int C,
                 double* __restrict__ part, int32_t* status, int32_t* abort_flag, unsigned long long limit_ns) {
   constexpr int NCOL = 2 * KP;
   constexpr uint32_t WBYTES = uint32_t(NCOL) * 128u;
+  constexpr int SQW = xa_sq_warps(KP);
+  constexpr int RPW = XA_TM / SQW;  // token rows of a stage per sum-of-squares warp
   constexpr uint32_t ID = tc::idesc(1, 1, 0, 0, XA_TM, NCOL);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -125,7 +133,7 @@ __global__ void __launch_bounds__(XA_THREADS, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < XA_STAGES; ++s) {
       mbar_init(full_bar(s), 1);
-      mbar_init(empty_bar(s), 3);  // the MMA commit and lane 0 of the two sum-of-squares warps
+      mbar_init(empty_bar(s), 1 + SQW);  // the MMA commit and lane 0 of each sum-of-squares warp
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(acc_full(b), 1);
@@ -210,7 +218,7 @@ __global__ void __launch_bounds__(XA_THREADS, 1)
     }
     __syncwarp();
   } else if (warp >= 6) {
-    // sum-of-squares warps 6, 7: tokens (warp - 6) * 64 + lane and + 32 of every stage; they alone
+    // sum-of-squares warps 6..5+SQW: tokens w2 * RPW + h * 32 + lane of every stage; they alone
     // (with the MMA commit) release the stages, so the statistics below never hold up the ring
     const int w2 = warp - 6;
     const int PS = part_stride(KP, C);
@@ -242,8 +250,8 @@ __global__ void __launch_bounds__(XA_THREADS, 1)
         // all banks); zero-filled out-of-range tokens and channels add nothing
         float pa[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // independent chains
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int row = w2 * 64 + h * 32 + lane;
+        for (int h = 0; h < RPW / 32; ++h) {
+          const int row = w2 * RPW + h * 32 + lane;
           const uint32_t ra = sbase + uint32_t(stage) * XA_STAGE + uint32_t(row) * 128u;
 #pragma unroll
           for (int c = 0; c < 8; ++c) {
@@ -447,7 +455,7 @@ __global__ void __launch_bounds__(FI_THREADS) k_kspace_final(const double* __res
   __syncthreads();
   const int nslot = grid * 4;
   // one warp; lanes over slots in order, then a fixed butterfly.  The ||x||^2 entry is written
-  // by the two sum-of-squares warps only (slots 0 and 1 of each CTA).
+  // by the sum-of-squares warps, one slot each (slots 0..xa_sq_warps(kp)-1 of each CTA).
   auto sum_entry = [&](int e, int nq) {
     const double* pe = part + (int64_t(l) * ps + e) * nslot;
     double v = 0.0;
@@ -459,7 +467,7 @@ __global__ void __launch_bounds__(FI_THREADS) k_kspace_final(const double* __res
   };
   const int nt = ntri(kp);
   if (warp == 0) {
-    const double v = sum_entry(nt + C * kp, 2);
+    const double v = sum_entry(nt + C * kp, xa_sq_warps(kp));
     if (lane == 0) s_xsq = v;
   }
   // ||T_l||^2 = sum_{c, c'} (P M P^T)[c][c'] (E^T E)[c][c']
@@ -662,13 +670,13 @@ cudaError_t launch_kspace_accumulate(const void* X, int L, int64_t N, int64_t d,
   if (kp == 16) {
     e = cudaFuncSetAttribute(k_kspace_xa<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, XA_SMEM);
     if (e != cudaSuccess) return e;
-    k_kspace_xa<16><<<grid, XA_THREADS, XA_SMEM, s>>>(tmX, tmW, L, N, d, ntiles, E, C, part, status, abort_flag,
-                                                      limit);
+    k_kspace_xa<16><<<grid, xa_threads(16), XA_SMEM, s>>>(tmX, tmW, L, N, d, ntiles, E, C, part, status,
+                                                            abort_flag, limit);
   } else {
     e = cudaFuncSetAttribute(k_kspace_xa<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, XA_SMEM);
     if (e != cudaSuccess) return e;
-    k_kspace_xa<32><<<grid, XA_THREADS, XA_SMEM, s>>>(tmX, tmW, L, N, d, ntiles, E, C, part, status, abort_flag,
-                                                      limit);
+    k_kspace_xa<32><<<grid, xa_threads(32), XA_SMEM, s>>>(tmX, tmW, L, N, d, ntiles, E, C, part, status,
+                                                            abort_flag, limit);
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
