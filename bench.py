@@ -49,6 +49,20 @@ FALLBACK_SUSTAINED_TFLOPS = 1700.0  # profiling recipe's sustained figure, used 
 GRAM_TC_TRAFFIC = {"sha256": "e55b0d4848cbeaee", "L": 28, "N": 131072, "d": 3584,
                    "read": 103600324352, "write": 3014398208,
                    "source": "profiles/gram_cross_tc_qwen2.5-7b.md"}
+# the same for one loca_kspace_accumulate call (k_kspace_prep, k_kspace_xa, k_kspace_ete,
+# k_kspace_final) at k = 16 (profiles/kspace_xa_qwen2.5-7b.md)
+KSPACE_TRAFFIC = {"sha256": "8d43fae519b52027", "L": 28, "N": 131072, "d": 3584, "k": 16,
+                  "read": 26422970624, "write": 27690496,
+                  "source": "profiles/kspace_xa_qwen2.5-7b.md"}
+
+
+def recorded_traffic(rec, source_file, **shape):
+    """DRAM bytes per launch from a capture record, or None once the kernel source or the shape
+    (every key of ``shape``, which the record must hold) differs from the captured one."""
+    src = open(os.path.join(ROOT, "paper_2608_03020_gb300", "csrc", source_file), "rb").read()
+    if rec["sha256"] != hashlib.sha256(src).hexdigest()[:16] or any(rec[n] != v for n, v in shape.items()):
+        return None
+    return float(rec["read"] + rec["write"])
 
 
 def parse():
@@ -351,11 +365,7 @@ def main():
     peak, peak_kind = peaks()
     flops = L * (2.0 * N * d * d + N * d * (d + 1.0))
     achieved = flops / (stages["gram_cross"] / 1e3) / 1e12
-    src = open(os.path.join(ROOT, "paper_2608_03020_gb300", "csrc", "gram_tc.cu"), "rb").read()
-    sha = hashlib.sha256(src).hexdigest()[:16]
-    traffic = None
-    if GRAM_TC_TRAFFIC["sha256"] == sha and (GRAM_TC_TRAFFIC["L"], GRAM_TC_TRAFFIC["N"], GRAM_TC_TRAFFIC["d"]) == (L, N, d):
-        traffic = float(GRAM_TC_TRAFFIC["read"] + GRAM_TC_TRAFFIC["write"])
+    traffic = recorded_traffic(GRAM_TC_TRAFFIC, "gram_tc.cu", L=L, N=N, d=d)
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "traffic": traffic, "kernel": "k_gram_cross_tc",
                 "peak_kind": f"bf16 dense sustained, {peak_kind}", "flops_per_launch": flops}
@@ -409,7 +419,8 @@ def main():
                   "roofline": {"bound": "hbm", "achieved": xbytes / (kst["accumulate"] / 1e3) / 1e9,
                                "peak": hbm_peak(), "unit": "GB/s",
                                "frac": xbytes / (kst["accumulate"] / 1e3) / 1e9 / hbm_peak(),
-                               "traffic": None, "kernel": "loca_kspace_accumulate (prep, X A on tcgen05, stats, final)",
+                               "traffic": recorded_traffic(KSPACE_TRAFFIC, "kspace.cu", L=L, N=N, d=d, k=k),
+                               "kernel": "loca_kspace_accumulate (prep, X A on tcgen05, stats, final)",
                                "bytes_per_launch": xbytes}}
 
     # the head error where it is HBM-bound: the Qwen2.5-14B row of the workloads (N = 131072 tokens,
