@@ -51,8 +51,8 @@ GRAM_TC_TRAFFIC = {"sha256": "e55b0d4848cbeaee", "L": 28, "N": 131072, "d": 3584
                    "source": "profiles/gram_cross_tc_qwen2.5-7b.md"}
 # the same for one loca_kspace_accumulate call (k_kspace_prep, k_kspace_xa, k_kspace_ete,
 # k_kspace_final) at k = 16 (profiles/kspace_xa_qwen2.5-7b.md)
-KSPACE_TRAFFIC = {"sha256": "8d43fae519b52027", "L": 28, "N": 131072, "d": 3584, "k": 16,
-                  "read": 26422970624, "write": 27690496,
+KSPACE_TRAFFIC = {"sha256": "11441129ac44e2da", "L": 28, "N": 131072, "d": 3584, "k": 16,
+                  "read": 26419919872, "write": 27811584,
                   "source": "profiles/kspace_xa_qwen2.5-7b.md"}
 
 

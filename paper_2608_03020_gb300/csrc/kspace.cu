@@ -82,11 +82,10 @@ __global__ void __launch_bounds__(PREP_THREADS) k_kspace_prep(const float* __res
 }
 
 // ------------------------------------------------------------------ X A on the tensor cores
-// warps: producer, MMA, 4 TMEM / statistics warps, then the sum-of-squares warps, which share the
-// 128 token rows of each stage and own one of the CTA's four partial slots of ||x||^2 each.  Four
-// of them (one row per lane) keep up with the TMA ring at kp = 16; at kp = 32 the statistics warps'
-// registers leave room for only two in one CTA per SM without spills.
-__host__ __device__ constexpr int xa_sq_warps(int kp) { return kp <= 16 ? 4 : 2; }
+// warps: producer, MMA, 4 TMEM / statistics warps, then four sum-of-squares warps, which share the
+// 128 token rows of each stage (one row per lane, so that they keep up with the TMA ring) and own
+// one of the CTA's four partial slots of ||x||^2 each.  320 threads leave 168 registers a thread.
+__host__ __device__ constexpr int xa_sq_warps(int) { return 4; }
 __host__ __device__ constexpr int xa_threads(int kp) { return 32 * (6 + xa_sq_warps(kp)); }
 static_assert(xa_sq_warps(16) <= 4 && xa_sq_warps(32) <= 4, "four partial slots per CTA");
 constexpr int XA_TM = 128;          // tokens per tile (TMEM lanes)
@@ -285,10 +284,15 @@ __global__ void __launch_bounds__(xa_threads(KP), 1)
     const int PS = part_stride(KP, C);
     float* ps = epi + (warp - 2) * 32 * (33 + ESTR);
     float* es = ps + 32 * 33;
-    // upper-triangle entries owned by this lane: eidx = lane + 32 i -> (a, b), a <= b
-    int pair[NG];
+    // upper-triangle entries owned by this lane: eidx = lane + 32 i -> (a, b), a <= b, row-major
+    // over the triangle.  At kp = 16 the pairs are held in registers; at kp = 32 they are
+    // recomputed per tile (closed form: the largest a with a kp - a (a - 1) / 2 <= eidx, from an
+    // fp32 square root of exact integers, then corrected by one either way), which keeps the
+    // statistics warps within 168 registers without spills.
+    constexpr int NPR = KP <= 16 ? NG : 1;
+    int pair[NPR];
 #pragma unroll
-    for (int i2 = 0; i2 < NG; ++i2) {
+    for (int i2 = 0; i2 < NPR; ++i2) {
       int rem = lane + 32 * i2, a = 0;
       while (a < KP && rem >= KP - a) {
         rem -= KP - a;
@@ -296,6 +300,20 @@ __global__ void __launch_bounds__(xa_threads(KP), 1)
       }
       pair[i2] = (a << 8) | (a + rem);
     }
+    auto tri_pair = [&](int i2, int& a, int& b) {
+      if constexpr (KP <= 16) {
+        a = pair[i2] >> 8;
+        b = pair[i2] & 0xff;
+      } else {
+        const int e = lane + 32 * i2;  // < ntri(KP)
+        const float w = float(2 * KP + 1);
+        a = int((w - sqrtf(w * w - 8.f * float(e))) * 0.5f);
+        if (a < 0) a = 0;
+        if (a * KP - a * (a - 1) / 2 > e) --a;
+        if ((a + 1) * KP - (a + 1) * a / 2 <= e) ++a;
+        b = e - (a * KP - a * (a - 1) / 2) + a;
+      }
+    };
     constexpr int NSM = (kMaxCk * KP + 31) / 32;
     const int NS = C * KP;
     // this lane's sums for the current block (fp32 within one CTA's run of tiles of a block; the
@@ -353,7 +371,8 @@ __global__ void __launch_bounds__(xa_threads(KP), 1)
 #pragma unroll
       for (int i2 = 0; i2 < NG; ++i2) {
         if (lane + 32 * i2 < NTRI) {
-          const int a = pair[i2] >> 8, b = pair[i2] & 0xff;
+          int a, b;
+          tri_pair(i2, a, b);
           float acc = 0.f;
 #pragma unroll 8
           for (int t = 0; t < 32; ++t) acc = fmaf(ps[t * PSTR + a], ps[t * PSTR + b], acc);
