@@ -58,7 +58,7 @@ typedef enum loca_status {
   LOCA_ERR_CUDA = 5,               /* a CUDA runtime call or launch failed */
   LOCA_ERR_TIMEOUT = 6,            /* a device wait gave up (reported by loca_device_status) */
   LOCA_ERR_WORKSPACE = 7,          /* workspace missing or smaller than required */
-  LOCA_ERR_UNSUPPORTED = 8,        /* valid request outside what this build supports */
+  LOCA_ERR_UNSUPPORTED = 8,        /* valid request outside what this library supports */
   LOCA_ERR_NUMERIC = 9             /* device: a system that should be positive definite was not
                                       in floating point (reported by loca_device_status) */
 } loca_status;
