@@ -97,7 +97,11 @@ constexpr uint32_t XA_TMEM_COLS = 128;
 constexpr int XA_MAX_GRID = 256;   // partial slots per block are sized for at most this many CTAs
 constexpr int kMaxCk = 16;         // C limit of the k-space path
 constexpr int kMaxRk = 32;         // r limit
-constexpr int XA_EPI_SMEM = 4 * 32 * ((32 + 1) + (kMaxCk + 1)) * 4;  // per-warp p and e staging
+// per-warp p and e staging: token-major rows at kp = 16 (32 x (33 + 17) floats), channel-major
+// rows of 36 floats at kp = 32 ((32 + 16) x 36 floats)
+constexpr int XA_EPI_WARP =
+    (32 + kMaxCk) * 36 > 32 * (33 + kMaxCk + 1) ? (32 + kMaxCk) * 36 : 32 * (33 + kMaxCk + 1);
+constexpr int XA_EPI_SMEM = 4 * XA_EPI_WARP * 4;
 
 // partial slot: upper triangle of p p^T (kp (kp + 1) / 2), e p^T (C x kp), ||x||^2
 __host__ __device__ constexpr int ntri(int kp) { return kp * (kp + 1) / 2; }
@@ -278,55 +282,77 @@ __global__ void __launch_bounds__(xa_threads(KP), 1)
     // epilogue warps 2..5: TMEM lane quarter q; token row = q * 32 + lane of each tile
     const int q = warp & 3;
     const int row = q * 32 + lane;
-    constexpr int PSTR = KP + 1, ESTR = kMaxCk + 1;
     constexpr int NTRI = ntri(KP);
-    constexpr int NG = (NTRI + 31) / 32;
     const int PS = part_stride(KP, C);
-    float* ps = epi + (warp - 2) * 32 * (33 + ESTR);
-    float* es = ps + 32 * 33;
-    // upper-triangle entries owned by this lane: eidx = lane + 32 i -> (a, b), a <= b, row-major
-    // over the triangle.  At kp = 16 the pairs are held in registers; at kp = 32 they are
-    // recomputed per tile (closed form: the largest a with a kp - a (a - 1) / 2 <= eidx, from an
-    // fp32 square root of exact integers, then corrected by one either way), which keeps the
-    // statistics warps within 168 registers without spills.
-    constexpr int NPR = KP <= 16 ? NG : 1;
-    int pair[NPR];
-#pragma unroll
-    for (int i2 = 0; i2 < NPR; ++i2) {
-      int rem = lane + 32 * i2, a = 0;
-      while (a < KP && rem >= KP - a) {
-        rem -= KP - a;
-        ++a;
-      }
-      pair[i2] = (a << 8) | (a + rem);
-    }
-    auto tri_pair = [&](int i2, int& a, int& b) {
-      if constexpr (KP <= 16) {
-        a = pair[i2] >> 8;
-        b = pair[i2] & 0xff;
-      } else {
-        const int e = lane + 32 * i2;  // < ntri(KP)
-        const float w = float(2 * KP + 1);
-        a = int((w - sqrtf(w * w - 8.f * float(e))) * 0.5f);
-        if (a < 0) a = 0;
-        if (a * KP - a * (a - 1) / 2 > e) --a;
-        if ((a + 1) * KP - (a + 1) * a / 2 <= e) ++a;
-        b = e - (a * KP - a * (a - 1) / 2) + a;
-      }
-    };
     constexpr int NSM = (kMaxCk * KP + 31) / 32;
     const int NS = C * KP;
+    // p p^T: at kp = 16 a lane owns single upper-triangle entries eidx = lane + 32 i; at kp = 32
+    // it owns 2 x 2 blocks (rows 2I, 2I+1; columns 2J, 2J+1; I <= J) of the 16 x 16 block
+    // triangle, bidx = lane + 32 i, whose p rows it reads four tokens at a time.  Either way each
+    // entry is the same fp32 FMA chain over the tile's tokens in order.
+    constexpr bool kBlk = KP > 16;
+    constexpr int KQ = kBlk ? KP / 2 : KP;   // side of the triangle a lane's items tile
+    constexpr int NQ = ntri(KQ);
+    constexpr int NG = (NQ + 31) / 32;
+    constexpr int NACC = kBlk ? 4 * NG : NG;
+    // item lane + 32 i -> (a, b), row-major over the triangle: (a << 8) | b at kp = 16; at kp = 32
+    // (a, b < 16) packed as (a << 4) | b into byte i % 4 of word i / 4
+    constexpr int NPW = kBlk ? (NG + 3) / 4 : NG;
+    uint32_t pair[NPW];
+#pragma unroll
+    for (int i2 = 0; i2 < NPW; ++i2) pair[i2] = 0u;
+#pragma unroll
+    for (int i2 = 0; i2 < NG; ++i2) {
+      int rem = lane + 32 * i2, a = 0;
+      while (a < KQ && rem >= KQ - a) {
+        rem -= KQ - a;
+        ++a;
+      }
+      if constexpr (kBlk)
+        pair[i2 / 4] |= uint32_t(((a << 4) | ((a + rem) & 15)) & 0xff) << (8 * (i2 % 4));
+      else
+        pair[i2] = uint32_t((a << 8) | (a + rem));
+    }
+    auto blk_pair = [&](int i2, int& bi, int& bj) {
+      const uint32_t x = (pair[i2 / 4] >> (8 * (i2 % 4))) & 0xffu;
+      bi = int(x >> 4);
+      bj = int(x & 15u);
+    };
+    // staging.  kp = 16: token-major rows (ps[t][s], es[t][c]).  kp = 32: channel-major rows of
+    // 36 floats (pT[.][t], eT[c][t]; 16-byte aligned for four-token loads), p row s stored at
+    // (s / 2) + 16 (s % 2) so that the column rows 2J of eight lanes fall in distinct banks.
+    constexpr int PSTR = KP + 1, ESTR = kMaxCk + 1;
+    constexpr int TST = 36;
+    float* ps = epi + (warp - 2) * (kBlk ? (32 + kMaxCk) * TST : 32 * (33 + ESTR));
+    float* es = kBlk ? ps + 32 * TST : ps + 32 * 33;
+    auto prow = [](int s2) { return (s2 >> 1) + (s2 & 1) * (KP / 2); };
+    auto entry = [](int a, int b) { return a * KP - a * (a - 1) / 2 + (b - a); };
     // this lane's sums for the current block (fp32 within one CTA's run of tiles of a block; the
     // runs are written once, as fp64, when the block changes, and reduced in a fixed order later)
-    float accg[NG], accs[NSM];
+    float accg[NACC], accs[NSM];
     int cur_l = -1;
     const int64_t nslot = int64_t(gridDim.x) * 4;
     auto flush = [&](int lf) {
       // entry-major: entry e of block lf at part[(lf * PS + e) * nslot + this slot]
       double* slot = part + int64_t(lf) * PS * nslot + int64_t(blockIdx.x) * 4 + q;
+      if constexpr (kBlk) {
 #pragma unroll
-      for (int i2 = 0; i2 < NG; ++i2)
-        if (lane + 32 * i2 < NTRI) slot[int64_t(lane + 32 * i2) * nslot] = double(accg[i2]);
+        for (int i2 = 0; i2 < NG; ++i2) {
+          if (lane + 32 * i2 < NQ) {
+            int bi, bj;
+            blk_pair(i2, bi, bj);
+            const int a0 = 2 * bi, b0 = 2 * bj;
+            slot[int64_t(entry(a0, b0)) * nslot] = double(accg[4 * i2]);
+            slot[int64_t(entry(a0, b0 + 1)) * nslot] = double(accg[4 * i2 + 1]);
+            if (a0 != b0) slot[int64_t(entry(a0 + 1, b0)) * nslot] = double(accg[4 * i2 + 2]);
+            slot[int64_t(entry(a0 + 1, b0 + 1)) * nslot] = double(accg[4 * i2 + 3]);
+          }
+        }
+      } else {
+#pragma unroll
+        for (int i2 = 0; i2 < NG; ++i2)
+          if (lane + 32 * i2 < NTRI) slot[int64_t(lane + 32 * i2) * nslot] = double(accg[i2]);
+      }
 #pragma unroll
       for (int i2 = 0; i2 < NSM; ++i2)
         if (lane + 32 * i2 < NS) slot[int64_t(NTRI + lane + 32 * i2) * nslot] = double(accs[i2]);
@@ -340,7 +366,7 @@ __global__ void __launch_bounds__(xa_threads(KP), 1)
         if (cur_l >= 0) flush(cur_l);
         cur_l = l;
 #pragma unroll
-        for (int i2 = 0; i2 < NG; ++i2) accg[i2] = 0.f;
+        for (int i2 = 0; i2 < NACC; ++i2) accg[i2] = 0.f;
 #pragma unroll
         for (int i2 = 0; i2 < NSM; ++i2) accs[i2] = 0.f;
       }
@@ -348,46 +374,122 @@ __global__ void __launch_bounds__(xa_threads(KP), 1)
       const bool a_ok = mbar_wait(acc_full(buf), (tcount >> 1) & 1u, wc);
       if (!__all_sync(0xffffffffu, a_ok)) break;
       fence_after();
-      float v[NCOL];
       const uint32_t ta = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(buf * NCOL);
-      if constexpr (NCOL == 32) {
+      // stage this warp's 32 tokens: p (kp) and e (C); tokens beyond N contribute zeros.  p is the
+      // sum of the hi and lo accumulator columns; at kp = 32 the two halves are read one after the
+      // other (hi staged, then lo added to it: the same fp32 sum)
+      if constexpr (kBlk) {
+        const int64_t n = int64_t(t0) + row;
+        const bool nv = n < N;
+        float v[32];
         tmem_ld32(ta, v);
+#pragma unroll
+        for (int s2 = 0; s2 < KP; ++s2) ps[prow(s2) * TST + lane] = v[s2];
+        tmem_ld32(ta + uint32_t(KP), v);
+        fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(acc_empty(buf));
+#pragma unroll
+        for (int s2 = 0; s2 < KP; ++s2) {
+          float* d = ps + prow(s2) * TST + lane;
+          *d = *d + v[s2];
+        }
+#pragma unroll
+        for (int c = 0; c < kMaxCk; ++c)
+          if (c < C) es[c * TST + lane] = nv ? E[n * C + c] : 0.f;
       } else {
-        tmem_ld32x2(ta, v);
+        float v[NCOL];
+        if constexpr (NCOL == 32) {
+          tmem_ld32(ta, v);
+        } else {
+          tmem_ld32x2(ta, v);
+        }
+        fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(acc_empty(buf));
+        const int64_t n = int64_t(t0) + row;
+        const bool nv = n < N;
+#pragma unroll
+        for (int s2 = 0; s2 < KP; ++s2) ps[lane * PSTR + s2] = v[s2] + v[KP + s2];
+#pragma unroll
+        for (int c = 0; c < kMaxCk; ++c)
+          if (c < C) es[lane * ESTR + c] = nv ? E[n * C + c] : 0.f;
       }
-      fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(acc_empty(buf));
-      // stage this warp's 32 tokens: p (kp) and e (C); tokens beyond N contribute zeros
-      const int64_t n = int64_t(t0) + row;
-      const bool nv = n < N;
-#pragma unroll
-      for (int s2 = 0; s2 < KP; ++s2) ps[lane * PSTR + s2] = v[s2] + v[KP + s2];
-#pragma unroll
-      for (int c = 0; c < kMaxCk; ++c)
-        if (c < C) es[lane * ESTR + c] = nv ? E[n * C + c] : 0.f;
       __syncwarp();
       // the tile's sums over this warp's 32 tokens, for the entries this lane owns
+      if constexpr (kBlk) {
 #pragma unroll
-      for (int i2 = 0; i2 < NG; ++i2) {
-        if (lane + 32 * i2 < NTRI) {
-          int a, b;
-          tri_pair(i2, a, b);
-          float acc = 0.f;
-#pragma unroll 8
-          for (int t = 0; t < 32; ++t) acc = fmaf(ps[t * PSTR + a], ps[t * PSTR + b], acc);
-          accg[i2] += acc;
+        for (int i2 = 0; i2 < NG; ++i2) {
+          if (lane + 32 * i2 < NQ) {
+            int bi, bj;
+            blk_pair(i2, bi, bj);
+            const float* ra0 = ps + prow(2 * bi) * TST;
+            const float* ra1 = ps + prow(2 * bi + 1) * TST;
+            const float* rb0 = ps + prow(2 * bj) * TST;
+            const float* rb1 = ps + prow(2 * bj + 1) * TST;
+            float s00 = 0.f, s01 = 0.f, s10 = 0.f, s11 = 0.f;
+#pragma unroll 2
+            for (int t = 0; t < 32; t += 4) {
+              const float4 x0 = *reinterpret_cast<const float4*>(ra0 + t);
+              const float4 x1 = *reinterpret_cast<const float4*>(ra1 + t);
+              const float4 y0 = *reinterpret_cast<const float4*>(rb0 + t);
+              const float4 y1 = *reinterpret_cast<const float4*>(rb1 + t);
+              s00 = fmaf(x0.x, y0.x, s00); s01 = fmaf(x0.x, y1.x, s01);
+              s10 = fmaf(x1.x, y0.x, s10); s11 = fmaf(x1.x, y1.x, s11);
+              s00 = fmaf(x0.y, y0.y, s00); s01 = fmaf(x0.y, y1.y, s01);
+              s10 = fmaf(x1.y, y0.y, s10); s11 = fmaf(x1.y, y1.y, s11);
+              s00 = fmaf(x0.z, y0.z, s00); s01 = fmaf(x0.z, y1.z, s01);
+              s10 = fmaf(x1.z, y0.z, s10); s11 = fmaf(x1.z, y1.z, s11);
+              s00 = fmaf(x0.w, y0.w, s00); s01 = fmaf(x0.w, y1.w, s01);
+              s10 = fmaf(x1.w, y0.w, s10); s11 = fmaf(x1.w, y1.w, s11);
+            }
+            accg[4 * i2] += s00;
+            accg[4 * i2 + 1] += s01;
+            accg[4 * i2 + 2] += s10;
+            accg[4 * i2 + 3] += s11;
+          }
         }
-      }
+        // e p^T: this lane's channel s = lane of every label column c (eidx = c kp + lane)
+        const float* rp = ps + prow(lane) * TST;
+        static_assert(!kBlk || NSM == kMaxCk, "one e p^T entry per label column and lane");
 #pragma unroll
-      for (int i2 = 0; i2 < NSM; ++i2) {
-        const int eidx = lane + 32 * i2;
-        if (eidx < NS) {
-          const int c = eidx / KP, s2 = eidx - c * KP;
-          float acc = 0.f;
+        for (int c = 0; c < kMaxCk; ++c) {
+          if (c < C) {
+            const float* re = es + c * TST;
+            float sc = 0.f;
+#pragma unroll 1
+            for (int t = 0; t < 32; t += 4) {
+              const float4 pv = *reinterpret_cast<const float4*>(rp + t);
+              const float4 ev = *reinterpret_cast<const float4*>(re + t);
+              sc = fmaf(ev.x, pv.x, sc);
+              sc = fmaf(ev.y, pv.y, sc);
+              sc = fmaf(ev.z, pv.z, sc);
+              sc = fmaf(ev.w, pv.w, sc);
+            }
+            accs[c] += sc;
+          }
+        }
+      } else {
+#pragma unroll
+        for (int i2 = 0; i2 < NG; ++i2) {
+          if (lane + 32 * i2 < NTRI) {
+            const int a = int(pair[i2] >> 8), b = int(pair[i2] & 0xffu);
+            float acc = 0.f;
 #pragma unroll 8
-          for (int t = 0; t < 32; ++t) acc = fmaf(es[t * ESTR + c], ps[t * PSTR + s2], acc);
-          accs[i2] += acc;
+            for (int t = 0; t < 32; ++t) acc = fmaf(ps[t * PSTR + a], ps[t * PSTR + b], acc);
+            accg[i2] += acc;
+          }
+        }
+#pragma unroll
+        for (int i2 = 0; i2 < NSM; ++i2) {
+          const int eidx = lane + 32 * i2;
+          if (eidx < NS) {
+            const int c = eidx / KP, s2 = eidx - c * KP;
+            float acc = 0.f;
+#pragma unroll 8
+            for (int t = 0; t < 32; ++t) acc = fmaf(es[t * ESTR + c], ps[t * PSTR + s2], acc);
+            accs[i2] += acc;
+          }
         }
       }
       __syncwarp();  // the staging rows are rewritten by the next tile
