@@ -37,6 +37,7 @@ __all__ = [
     "scaled_step",
     "accumulate_stats",
     "project_stats",
+    "kspace_stats",
     "ridge_lambdas",
     "cholesky",
     "ridge_solve",
@@ -198,6 +199,39 @@ def project_stats(gram, cross, A, B_prev=None):
         Bp = np.asarray(B_prev, dtype=np.float64)
         C = C + np.stack([Bp[l] @ G[l] for l in range(L)])
     return G, C
+
+
+def kspace_stats(X_batches, T_batches, A, eta, B_prev=None):
+    """The paper's own projected statistics, accumulated token by token over the
+    mini-batches (Eq. 9; S7 additivity; S8 one step per block and mini-batch):
+
+    ``p_n = A_l^T x_n`` (the adapter features, Eq. 1), ``rho_n = B^(t) p_n - eta_bar q_n``
+    (Eq. 6, ``q_n`` the target row), ``G_l = sum_n p_n p_n^T`` (``k x k``) and
+    ``C_l = sum_n rho_n p_n^T`` (``d x k``), with ``eta_bar`` from :func:`scaled_step` on the
+    token's mini-batch.  Written token-major: ``P_feat = X_l A_l`` (one row per token),
+    ``R = P_feat B^T - eta_bar T_l`` (rows ``rho_n^T``), ``G_l += P_feat^T P_feat``,
+    ``C_l += R^T P_feat``.  The targets enter unrounded (this route never stores them).
+    ``B_prev=None`` means ``B^(t) = 0``.  Returns ``(G, C, xsq_total)``.
+    """
+    A = np.asarray(A, dtype=np.float64)
+    L, d, k = A.shape
+    G = np.zeros((L, k, k))
+    C = np.zeros((L, d, k))
+    xsq_total = np.zeros(L)
+    Bp = None if B_prev is None else np.asarray(B_prev, dtype=np.float64)
+    for Xm, Tm in zip(X_batches, T_batches):
+        for l in range(L):
+            Xl = np.asarray(Xm[l], dtype=np.float64)
+            Tl = np.asarray(Tm[l], dtype=np.float64)
+            step = scaled_step(eta, Xl, Tl)
+            feat = Xl @ A[l]
+            R = -step * Tl
+            if Bp is not None:
+                R = R + feat @ Bp[l].T
+            G[l] += feat.T @ feat
+            C[l] += R.T @ feat
+            xsq_total[l] += float(np.sum(Xl * Xl))
+    return G, C, xsq_total
 
 
 def ridge_lambdas(lambda_rel, xsq_total, d):

@@ -284,6 +284,35 @@ def test_streaming_and_projection_match_per_token_definitions():
     # one-shot Gram equals the streamed Gram (additivity)
     g1, _, _ = O.accumulate_stats([X], [np.concatenate(Tb, axis=1)], 0.01)
     assert _rel(g1, gram) < 1e-14
+    # the paper's own k x k / d x k statistics, accumulated without a d x d matrix
+    Gk, Ck, xk = O.kspace_stats(Xb, Tb, A, 0.01, B_prev=Bp)
+    assert _rel(Gk, G_ref) < 1e-13 and _rel(Ck, C_ref) < 1e-13
+    assert np.allclose(xk, xsq, rtol=1e-14)
+
+
+def test_kspace_stats_brute_force_and_special_cases():
+    """kspace_stats against per-token loops without B_prev (rho = -eta_bar q), the zero-target
+    case (no step, C = B_prev G), Prop. S8 (T -> aT leaves C unchanged) and a feature map that
+    is the identity (G is then the Gram of X)."""
+    rng = np.random.default_rng(12)
+    L, N, d, k, C, r = 2, 17, 5, 2, 3, 2
+    X = rng.standard_normal((L, N, d))
+    E = rng.standard_normal((N, C))
+    P = rng.standard_normal((L, C, r))
+    Q = rng.standard_normal((L, r, d))
+    A = rng.standard_normal((L, d, k))
+    T, _ = O.feedback_targets(E, P, Q)
+    G, Cs, _ = O.kspace_stats([X], [T], A, 0.03)
+    G_ref, C_ref = _per_token_stats(X, [T], np.zeros(N, dtype=int), 0.03, A, None)
+    assert _rel(G, G_ref) < 1e-13 and _rel(Cs, C_ref) < 1e-13
+    Bp = rng.standard_normal((L, d, k))
+    G0, C0, _ = O.kspace_stats([X], [np.zeros_like(T)], A, 0.03, B_prev=Bp)
+    assert np.allclose(C0, np.einsum("ldk,lkj->ldj", Bp, G0), rtol=1e-13, atol=1e-12)
+    _, C2, _ = O.kspace_stats([X], [4.0 * T], A, 0.03)
+    assert _rel(C2, Cs) < 1e-13
+    eye = np.stack([np.eye(d)] * L)
+    Gi, _, _ = O.kspace_stats([X], [T], eye, 0.03)
+    assert np.allclose(Gi, np.einsum("lnd,lne->lde", X, X), rtol=1e-13, atol=1e-12)
 
 
 # ---------------------------------------------------------------- O5 solve
