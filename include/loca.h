@@ -75,9 +75,10 @@ int loca_version(void);
  * when one runs out the kernel records LOCA_ERR_TIMEOUT in the device status word, makes the
  * other waits of its launch give up, lets the copies and MMAs already in flight land, frees its
  * tensor memory and returns, so the context stays usable.  This sets, for the whole process,
- * how long such a wait may take in the single-CTA kernels (loca_targets, loca_kspace_accumulate)
+ * how long such a wait may take in the tensor-core kernels (loca_targets, loca_kspace_accumulate
+ * and the CTA-pair Gram / cross kernel of loca_gram_cross, loca_accumulate and their variants)
  * before it gives up: ns = 0 restores the default of 4 s; a tiny value makes a call time out on
- * purpose, to test that path.  (The CTA-pair Gram / cross kernel always uses 4 s.)
+ * purpose, to test that path.
  */
 int loca_set_wait_limit(uint64_t ns);
 

@@ -18,11 +18,21 @@
 //                CTA one thread issues the MMAs.  Its loop is kept short (descriptors built once,
 //                advanced by integer adds; bounded wait entered only if an inline try_wait fails)
 //                so that issue keeps pace with the tensor core.
-//   warps 2-5    epilogue (both CTAs): tcgen05.ld, scale, store.
+//   warps 2-5    epilogue (both CTAs): tcgen05.ld, scale, stage 32 x 32 boxes in shared memory
+//                (128-byte swizzle) and hand them to the TMA unit: a bulk store for the first
+//                segment of a zero_first launch, a bulk reduce-add into the fp32 output otherwise.
 // Work item = one 256-column tile of X (B) and up to two 256-row accumulators sharing it (Gram
 // tiles that touch the upper triangle and all cross tiles of that column, paired in order).
-// Gram elements (i, j), i <= j, are stored directly and mirrored to (j, i): every output element
-// has one writer (deterministic, no atomics).  MMA commits multicast to both CTAs' barriers.
+// Segments: an item's token axis is cut into segments of kSegTokens tokens; the accumulators start
+// from zero in every segment and each segment's sums are added into the fp32 output.  The tensor
+// cores' fp32 accumulation loses a fraction of an ulp of the running sum at every MMA step, always
+// toward zero; bounding the steps per accumulator bounds that bias (the output's own additions
+// round to nearest).  The MMA issuer waits for the epilogue only until the TMEM reads are done:
+// the stores and additions are the TMA unit's.  Each output element has one issuing thread, which
+// waits for its previous segment's additions to complete before issuing the next, so the order
+// of additions is fixed (deterministic, no atomics).  Gram tiles are written whole; the elements
+// below the diagonal are then overwritten with their mirror images by k_gram_mirror, so the Gram
+// matrix is exactly symmetric.
 // Lockstep: all clusters stream the same token window of X_l and T_l at the same time, so an
 // operand line read from HBM is then served from L2 to the other tiles that need it.  The even
 // CTA's producer passes a sync point at the start of every work item and every kSyncEvery
@@ -36,8 +46,13 @@
 // only, each block filling whole rounds, and the few items left of every block follow at the end;
 // a round then streams one block's tiles instead of parts of two.
 // Every mbarrier wait is bounded: on expiry the status word gets LOCA_ERR_TIMEOUT, a launch-local
-// flag makes every other wait give up, the even CTA drains the loads and MMAs in flight, and
-// both CTAs meet at the final cluster barrier before TMEM is freed.
+// flag makes every other wait give up, and the roles stop, each CTA's producer at its own point.
+// At the end both CTAs meet at a cluster barrier (the odd CTA has posted how many pipeline
+// iterations it issued); then the even CTA reconciles its full barriers with what each CTA issued
+// (arming what only the odd CTA issued, settling with mbarrier.complete_tx the bytes the odd CTA
+// never issued) and waits for every copy to land; the MMAs in flight are waited for and the
+// epilogue's bulk copies have completed; only then do both CTAs pass the final cluster barrier
+// and free TMEM.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -64,8 +79,15 @@ constexpr int B_BYTES = BNC * BK * 2;               // 16 KB
 constexpr int STAGE_BYTES = 2 * A_BYTES + B_BYTES;  // 48 KB
 constexpr int TMEM_COLS = 512;
 constexpr int NUM_THREADS = 192;
+constexpr int kSegTokens = 16384;                   // tokens per accumulation segment
+constexpr int EPI_BOX_BYTES = 32 * 32 * 4;          // one 32-row x 32-column fp32 output box
+constexpr int EPI_BUFS = 2;                         // staging boxes per epilogue warp
+constexpr int EPI_BYTES = 4 * EPI_BUFS * EPI_BOX_BYTES;  // 32 KB
+// barriers: full[S], empty[S], acc_full, acc_empty, drain
 constexpr int NUM_BARS = 2 * STAGES + 3;
-constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /* align slack */ + 256 /* barriers */;
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EPI_BYTES + 1024 /* align slack */ + 256 /* barriers */;
+static_assert(SMEM_BYTES <= 232448, "shared memory per CTA");
+static_assert(kSegTokens % (BK * kSyncEvery) == 0, "segments end on lockstep sync points");
 
 // Instruction descriptor (kind::f16): D fp32, A bf16, B bf16, A and B MN-major, M = 256, N = 256.
 constexpr uint32_t IDESC_PAIR = tc::idesc(1, 1, 1, 1, BMP, BN);
@@ -136,16 +158,17 @@ __device__ __forceinline__ Item decode(const Geo& g, int it) {
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     k_gram_cross_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmT,
                     const __grid_constant__ CUtensorMap tmXa, const __grid_constant__ CUtensorMap tmTa,
-                    const __grid_constant__ CUtensorMap tmXb, int blocked, Geo g, int total_items,
-                    const float* __restrict__ alpha, int zero_first, float* __restrict__ gram,
-                    float* __restrict__ cross, int32_t* status, int32_t* abort_flag,
+                    const __grid_constant__ CUtensorMap tmXb, const __grid_constant__ CUtensorMap tmG,
+                    const __grid_constant__ CUtensorMap tmC, int blocked, Geo g, int total_items, int seg_kb,
+                    const float* __restrict__ alpha, int zero_first, int32_t* status, int32_t* abort_flag,
                     uint32_t* round_ctr, unsigned long long limit_ns, unsigned long long sync_ns) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
-  // full[S] (loads of both CTAs, used in the even CTA), empty[S], acc_full, acc_empty, drain
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + NUM_BARS + 1);
+  uint8_t* epi = smem + STAGES * STAGE_BYTES;  // 1024-aligned: the boxes use the 128-byte swizzle
+  uint64_t* bars = reinterpret_cast<uint64_t*>(epi + EPI_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + NUM_BARS);
+  uint32_t* odd_issued = tmem_slot + 1;  // even CTA: pipeline iterations the odd CTA issued
   const uint32_t smem_base = smem_u32(smem);
   const uint32_t bar_base = smem_u32(bars);
   auto full_bar = [&](int s) { return bar_base + 8u * s; };
@@ -170,6 +193,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     mbar_init(acc_full, 1);
     mbar_init(acc_empty, 8);  // lane 0 of the 4 epilogue warps of each CTA
     mbar_init(drain_bar, 1);
+    *odd_issued = 0;
     mbar_init_fence();
     if (blocked) {
       prefetch_tensormap(&tmXa);
@@ -179,6 +203,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       prefetch_tensormap(&tmX);
       prefetch_tensormap(&tmT);
     }
+    prefetch_tensormap(&tmG);
+    prefetch_tensormap(&tmC);
   }
   if (warp == 1) tmem_alloc_pair(smem_u32(tmem_slot), TMEM_COLS);
   fence_before();
@@ -186,13 +212,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
   fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const int nkb = (g.N + BK - 1) / BK;
+  const int nseg = (nkb + seg_kb - 1) / seg_kb;
+
+  uint32_t iters_done = 0;  // producer: pipeline iterations this CTA issued
 
   if (warp == 0) {
     if (lane == 0) {
       // ---------------- TMA producer (both CTAs): this CTA's rows of A and columns of B
       int stage = 0;
       uint32_t phase = 0;
-      uint32_t pending = 0, pending_par = 0;  // even CTA: armed stages and their phase parity
+      uint32_t iter = 0;  // pipeline iterations issued by this CTA
       bool ok = true;
       bool sync = leader;  // dropped for the rest of the launch if a wait runs out
       // sync points: each item counts one every kSyncEvery k-blocks and one at its end (P per item)
@@ -214,7 +243,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
         const uint32_t active = uint32_t(left < ncl ? left : ncl);
         if (sync && round > 0) wait_for(before);  // every cluster finished issuing its last item
         const Item w = decode(g, it);
-        const uint32_t bytes_both = 2u * (uint32_t(w.nslots) * A_BYTES + B_BYTES);
+        const uint32_t bytes_one = uint32_t(w.nslots) * A_BYTES + B_BYTES;
         for (int kb = 0; kb < nkb; ++kb) {
           if (leader && kb > 0 && kb % kSyncEvery == 0) {
             atomicAdd(round_ctr, 1u);
@@ -225,12 +254,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
             ok = false;
             break;
           }
+          if (leader) mbar_arrive_expect_tx(full_bar(stage), 2u * bytes_one);
           const uint32_t fb = mapa_shared(full_bar(stage), 0);
-          if (leader) {
-            mbar_arrive_expect_tx(full_bar(stage), bytes_both);
-            pending |= 1u << stage;
-            pending_par = (pending_par & ~(1u << stage)) | (phase << stage);
-          }
           const uint32_t st = smem_base + uint32_t(stage) * STAGE_BYTES;
           const uint32_t bdst = st + 2u * A_BYTES;
           const int tok = kb * BK;
@@ -251,16 +276,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
             tma_load_3d_pair(bdst, &tmX, fb, col0, tok, w.l);
             tma_load_3d_pair(bdst + SUB_BYTES, &tmX, fb, col0 + 64, tok, w.l);
           }
+          ++iter;
           if (++stage == STAGES) { stage = 0; phase ^= 1u; }
         }
         if (ok && leader) atomicAdd(round_ctr, 1u);
         before += active * uint32_t(P);
       }
-      if (!ok && leader) {
-        // the armed stages count the bytes of both CTAs: let them land before either CTA exits
-        for (int s = 0; s < STAGES; ++s)
-          if (pending & (1u << s)) mbar_drain(full_bar(s), (pending_par >> s) & 1u, limit_ns);
-      }
+      // the odd CTA posts how many iterations it issued (read by the even CTA after the barrier)
+      if (!leader) st_shared_cluster_u32(mapa_shared(smem_u32(odd_issued), 0), iter);
+      iters_done = iter;
     }
     __syncwarp();
   } else if (warp == 1) {
@@ -277,13 +301,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       for (int it = cid; it < total_items && ok; it += ncl) {
         const Item w = decode(g, it);
         const bool two = w.nslots == 2;
-        if (!mbar_try_wait_cluster(acc_empty, acc_phase ^ 1u) &&
-            !mbar_wait_cluster(acc_empty, acc_phase ^ 1u, wc)) {
-          ok = false;
-          break;
-        }
-        fence_after();
         for (int kb = 0; kb < nkb; ++kb) {
+          const int in_seg = kb % seg_kb;
+          if (in_seg == 0) {  // a new segment: wait until the epilogue has read the accumulators
+            if (!mbar_try_wait_cluster(acc_empty, acc_phase ^ 1u) &&
+                !mbar_wait_cluster(acc_empty, acc_phase ^ 1u, wc)) {
+              ok = false;
+              break;
+            }
+            fence_after();
+          }
           if (!mbar_try_wait_cluster(full_bar(stage), phase) &&
               !mbar_wait_cluster(full_bar(stage), phase, wc)) {
             ok = false;
@@ -294,99 +321,149 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
           const uint64_t ad = a_desc0 + so, bd = b_desc0 + so;
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk) {
-            const uint32_t acc = (kb | kk) != 0 ? 1u : 0u;
+            const uint32_t acc = (in_seg | kk) != 0 ? 1u : 0u;
             mma_f16_pair(d0, ad + kk * kKStep, bd + kk * kKStep, IDESC_PAIR, acc);
             if (two) mma_f16_pair(d1, ad + kSlotStep + kk * kKStep, bd + kk * kKStep, IDESC_PAIR, acc);
           }
           issued = true;
           mma_commit_pair_mc(empty_bar(stage), 0x3);  // frees the stage in both CTAs
           if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+          if (in_seg == seg_kb - 1 || kb == nkb - 1) {
+            mma_commit_pair_mc(acc_full, 0x3);  // this segment's sums complete in both CTAs
+            acc_phase ^= 1u;
+          }
         }
-        if (!ok) break;
-        mma_commit_pair_mc(acc_full, 0x3);  // accumulators of both CTAs complete
-        acc_phase ^= 1u;
       }
-      if (!ok && issued) {
+      if (issued) {  // every MMA of this launch has completed before TMEM can be freed
         mma_commit_pair(drain_bar);
-        mbar_drain(drain_bar, 0, limit_ns);
+        mbar_drain(drain_bar, 0, kDrainLimitNs);
       }
     }
     __syncwarp();
   } else {
     // ---------------- epilogue: warps 2..5, TMEM lane quarter = warp % 4
     const int q = warp & 3;
-    const int row_in_tile = q * 32 + lane;
+    uint8_t* box0 = epi + (warp - 2) * (EPI_BUFS * EPI_BOX_BYTES);
+    const uint32_t box0_s = smem_u32(box0);
     const uint32_t acc_empty_leader = leader ? acc_empty : mapa_shared(acc_empty, 0);
     uint32_t acc_phase = 0;
-    for (int it = cid; it < total_items; it += ncl) {
+    uint32_t nbox = 0;  // boxes this warp has handed to the TMA unit
+    bool go = true;
+    for (int it = cid; it < total_items && go; it += ncl) {
       const Item w = decode(g, it);
-      const bool ok = mbar_wait_cluster(acc_full, acc_phase, wc);
-      if (!__all_sync(0xffffffffu, ok)) break;  // warp-uniform decision, warp reconverged
-      fence_after();
       const float al = alpha[w.l];
-      for (int s = 0; s < w.nslots; ++s) {
-        const bool is_gram = w.kind[s] == 0;
-        float* out = (is_gram ? gram : cross) + int64_t(w.l) * g.d * g.d;
-        const int i = w.mt[s] * BMP + int(rank) * BMC + row_in_tile;
-        const float sc = is_gram ? 1.f : al;
+      for (int seg = 0; seg < nseg; ++seg) {
+        const bool ok = mbar_wait_cluster(acc_full, acc_phase, wc);
+        if (!__all_sync(0xffffffffu, ok)) {  // warp-uniform decision, warp reconverged
+          go = false;
+          break;
+        }
+        fence_after();
+        // the previous segment's additions to these boxes are complete: fixed order of additions
+        if (lane == 0) bulk_wait_group0();
+        __syncwarp();
+        const bool store = zero_first && seg == 0;
+        for (int s = 0; s < w.nslots; ++s) {
+          const bool is_gram = w.kind[s] == 0;
+          const CUtensorMap* omap = is_gram ? &tmG : &tmC;
+          const float sc = is_gram ? 1.f : al;
+          const int i0 = w.mt[s] * BMP + int(rank) * BMC + q * 32;
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
-          float v[32];
-          tmem_ld32(tmem_base + (uint32_t(q * 32) << 16) + uint32_t(s * BN + c * 32), v);
-          const int j0 = w.nt * BN + c * 32;
-          if (i >= g.d || j0 >= g.d) continue;
-          float* orow = out + int64_t(i) * g.d;
-          const bool whole = (j0 + 32 <= g.d) && (!is_gram || i <= j0);
-          if (whole) {
-            float4* p = reinterpret_cast<float4*>(orow + j0);
-#pragma unroll
-            for (int u = 0; u < 8; ++u) {
-              float4 x = make_float4(sc * v[4 * u], sc * v[4 * u + 1], sc * v[4 * u + 2],
-                                     sc * v[4 * u + 3]);
-              if (!zero_first) {
-                const float4 o = p[u];
-                x.x += o.x; x.y += o.y; x.z += o.z; x.w += o.w;
-              }
-              p[u] = x;
-            }
-          } else {
-#pragma unroll
-            for (int u = 0; u < 32; ++u) {
-              const int j = j0 + u;
-              if (j >= g.d) break;
-              if (is_gram && i > j) continue;
-              const float x = sc * v[u];
-              orow[j] = zero_first ? x : orow[j] + x;
-            }
-          }
-          if (is_gram) {
-            // mirror (i, j), i < j, to (j, i): for fixed j the warp writes 32 consecutive i
-#pragma unroll 4
-            for (int u = 0; u < 32; ++u) {
-              const int j = j0 + u;
-              if (j >= g.d) break;
-              if (i < j) {
-                float* p = out + int64_t(j) * g.d + i;
-                *p = zero_first ? v[u] : *p + v[u];
+          for (int c = 0; c < BN / 32; ++c) {
+            float v[32];
+            tmem_ld32(tmem_base + (uint32_t(q * 32) << 16) + uint32_t(s * BN + c * 32), v);
+            if (s == w.nslots - 1 && c == BN / 32 - 1) {
+              // all of this warp's accumulator reads are done: the MMA may start the next segment
+              fence_before();
+              __syncwarp();
+              if (lane == 0) {
+                if (leader) mbar_arrive(acc_empty);
+                else mbar_arrive_remote(acc_empty_leader);
               }
             }
+            const int j0 = w.nt * BN + c * 32;
+            if (i0 >= g.d || j0 >= g.d) continue;  // warp-uniform; partial boxes are clipped by the TMA unit
+            const uint32_t buf = nbox & (EPI_BUFS - 1);
+            if (lane == 0) bulk_wait_group_read1();  // this buffer's previous box has been read
+            __syncwarp();
+            // row `lane` of the box: 8 chunks of 16 bytes, chunk u at position u ^ (lane & 7)
+            float4* row = reinterpret_cast<float4*>(box0 + buf * EPI_BOX_BYTES + lane * 128);
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+              row[u ^ (lane & 7)] = make_float4(sc * v[4 * u], sc * v[4 * u + 1], sc * v[4 * u + 2],
+                                                sc * v[4 * u + 3]);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              const uint32_t src = box0_s + buf * EPI_BOX_BYTES;
+              if (store) tma_store_3d(omap, src, j0, i0, w.l);
+              else tma_reduce_add_3d(omap, src, j0, i0, w.l);
+              bulk_commit_group();
+            }
+            ++nbox;
           }
         }
+        acc_phase ^= 1u;
       }
-      fence_before();
-      __syncwarp();
-      if (lane == 0) {
-        if (leader) mbar_arrive(acc_empty);
-        else mbar_arrive_remote(acc_empty_leader);
-      }
-      acc_phase ^= 1u;
     }
+    if (lane == 0) bulk_wait_group0();  // every box written before the CTA can leave
+    __syncwarp();
   }
 
+  fence_before();
+  cluster_sync();  // every role has stopped; the odd CTA's issue count is visible
+  fence_after();
+  if (warp == 0 && lane == 0 && leader) {
+    // Copies still in flight when a role gave up.  Iteration t of the pipeline uses stage
+    // t % STAGES; the even CTA arms it (the bytes of both CTAs) and issues its half, the odd CTA
+    // issues its half after its own wait for the stage.  The two CTAs issued n_even and n_odd
+    // iterations, |n_even - n_odd| <= STAGES, and every iteration before the last STAGES of
+    // max(n_even, n_odd) has landed (a later use of its stage waited for it).  Of those last ones,
+    // an iteration the odd CTA never issued gets its bytes settled, an iteration only the odd CTA
+    // issued gets armed with its bytes, and every one is waited for.  After a normal run both
+    // counts are equal, every phase has completed and these waits return at once.
+    const uint32_t n_even = iters_done;
+    const uint32_t n_odd = *reinterpret_cast<volatile uint32_t*>(odd_issued);
+    const uint32_t hi = n_even > n_odd ? n_even : n_odd;
+    const uint32_t lo = hi > uint32_t(STAGES) ? hi - uint32_t(STAGES) : 0u;
+    for (uint32_t t = lo; t < hi; ++t) {
+      const int s = int(t % STAGES);
+      const Item w = decode(g, cid + int(t / uint32_t(nkb)) * ncl);
+      const uint32_t odd_bytes = uint32_t(w.nslots) * A_BYTES + B_BYTES;
+      if (t >= n_odd && t < n_even) mbar_complete_tx(full_bar(s), odd_bytes);
+      else if (t >= n_even && t < n_odd) mbar_arrive_expect_tx(full_bar(s), odd_bytes);
+      mbar_drain(full_bar(s), (t / STAGES) & 1u, kDrainLimitNs);
+    }
+  }
   fence_before();
   cluster_sync();  // no CTA leaves while its peer may still use its barriers, smem or TMEM
   fence_after();
   if (warp == 1) tmem_dealloc_pair(tmem_base, TMEM_COLS);
+}
+
+// Lower triangle of every Gram_l from its upper triangle: element (i, j), i > j, becomes (j, i).
+// One 32 x 32 tile (bi, bj), bi >= bj, per CTA (256 threads), through a padded shared tile.
+__global__ void __launch_bounds__(256) k_gram_mirror(float* __restrict__ gram, int d, int nt) {
+  __shared__ float tile[32][33];
+  const int l = blockIdx.y;
+  // triangular index t = bi (bi + 1) / 2 + bj, 0 <= bj <= bi < nt
+  const int t = blockIdx.x;
+  int bi = int((sqrtf(8.f * float(t) + 1.f) - 1.f) * 0.5f);
+  while ((bi + 1) * (bi + 2) / 2 <= t) ++bi;
+  while (bi * (bi + 1) / 2 > t) --bi;
+  const int bj = t - bi * (bi + 1) / 2;
+  (void)nt;
+  float* G = gram + int64_t(l) * d * d;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  for (int r = ty; r < 32; r += 8) {  // source rows j of the upper tile (bj, bi)
+    const int i = bj * 32 + r, j = bi * 32 + tx;
+    if (i < d && j < d) tile[r][tx] = G[int64_t(i) * d + j];
+  }
+  __syncthreads();
+  for (int r = ty; r < 32; r += 8) {
+    const int i = bi * 32 + r, j = bj * 32 + tx;
+    if (i < d && j < d && i > j) G[int64_t(i) * d + j] = tile[tx][r];
+  }
 }
 
 // ------------------------------------------------------------------ host side
@@ -417,6 +494,20 @@ bool make_map_blocked(CUtensorMap* m, const void* base, int L, int64_t N, int64_
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 3-D view (column, row, block) of the fp32 d x d outputs; boxes of 32 x 32 elements, 128-byte
+// swizzle (the epilogue's staging layout).  Rows are d * 4 bytes (d % 8 == 0 on this path).
+bool make_out_map(CUtensorMap* m, float* base, int L, int64_t d) {
+  auto fn = tensor_map_encoder();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {cuuint64_t(d), cuuint64_t(d), cuuint64_t(L)};
+  cuuint64_t strides[2] = {cuuint64_t(d) * 4, cuuint64_t(d) * cuuint64_t(d) * 4};
+  cuuint32_t box[3] = {32, 32, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, static_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Clusters of 2 that can be resident at once (every SM pairs on GB300: 76 clusters on 152 SMs).
 int resident_clusters() {
   int clusters = sm_count() / 2;
@@ -443,11 +534,13 @@ int resident_clusters() {
 cudaError_t launch_gram_cross_tc(const void* X, const void* T, int L, int64_t N, int64_t d,
                                  const float* alpha, int zero_first, float* gram, float* cross,
                                  int32_t* status, int32_t* abort_flag, cudaStream_t s) {
-  CUtensorMap mx, mt, mxa, mta, mxb;
+  CUtensorMap mx, mt, mxa, mta, mxb, mg, mc;
   memset(&mxa, 0, sizeof(mxa));
   memset(&mta, 0, sizeof(mta));
   memset(&mxb, 0, sizeof(mxb));
-  if (!make_map(&mx, X, L, N, d) || !make_map(&mt, T, L, N, d)) return cudaErrorInvalidValue;
+  if (!make_map(&mx, X, L, N, d) || !make_map(&mt, T, L, N, d) || !make_out_map(&mg, gram, L, d) ||
+      !make_out_map(&mc, cross, L, d))
+    return cudaErrorInvalidValue;
   int blocked = 0;
   if (d % 64 == 0 && make_map_blocked(&mxa, X, L, N, d, BMC / 64) &&
       make_map_blocked(&mta, T, L, N, d, BMC / 64) && make_map_blocked(&mxb, X, L, N, d, BNC / 64))
@@ -478,8 +571,12 @@ cudaError_t launch_gram_cross_tc(const void* X, const void* T, int L, int64_t N,
   const int64_t nkb = (N + BK - 1) / BK;
   const unsigned long long sync_ns = 50000ull + 2000ull * (unsigned long long)nkb;
   k_gram_cross_tc<<<2 * clusters, NUM_THREADS, SMEM_BYTES, s>>>(
-      mx, mt, mxa, mta, mxb, blocked, g, total, alpha, zero_first, gram, cross, status, abort_flag,
-      reinterpret_cast<uint32_t*>(abort_flag + 1), 4000000000ull /* 4 s per wait */, sync_ns);
+      mx, mt, mxa, mta, mxb, mg, mc, blocked, g, total, kSegTokens / BK, alpha, zero_first, status, abort_flag,
+      reinterpret_cast<uint32_t*>(abort_flag + 1), wait_limit_ns(), sync_ns);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const int nt = int((d + 31) / 32);
+  k_gram_mirror<<<dim3(unsigned(nt * (nt + 1) / 2), unsigned(L)), 256, 0, s>>>(gram, int(d), nt);
   return cudaGetLastError();
 }
 

@@ -65,8 +65,8 @@ cudaError_t launch_gram_cross_tc(const void* X, const void* T, int L, int64_t N,
                                  const float* alpha, int zero_first, float* gram, float* cross,
                                  int32_t* status, int32_t* abort_flag, cudaStream_t s);
 
-// Limit of the bounded device waits of the single-CTA tensor-core kernels (targets, k-space
-// statistics): 4 s unless loca_set_wait_limit changed it.
+// Limit of the bounded device waits of the tensor-core kernels (targets, k-space statistics,
+// Gram / cross): 4 s unless loca_set_wait_limit changed it.
 unsigned long long wait_limit_ns();
 
 // ---- alignment diagnostic (align.cu)

@@ -131,7 +131,7 @@ static __device__ __noinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t par
   const uint64_t t0 = globaltimer();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait_cluster(bar, parity)) return true;
-    if ((it & 255u) == 0) {
+    if ((it & 7u) == 0) {
       if (*w.abort_flag != 0) return false;
       if (globaltimer() - t0 > w.limit_ns) {
         atomicExch(w.status, int32_t(LOCA_ERR_TIMEOUT));
@@ -368,6 +368,23 @@ __device__ __forceinline__ void tma_store_4d(const CUtensorMap* map, uint32_t sr
 // Wait until all but the most recent committed bulk group of this thread have read their source.
 __device__ __forceinline__ void bulk_wait_group_read1() {
   asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+// TMA reduction of one box from shared memory into global memory: element-wise add (the data
+// type is the tensor map's), bulk-group completion.
+__device__ __forceinline__ void tma_reduce_add_3d(const CUtensorMap* map, uint32_t src, int c0, int c1, int c2) {
+  asm volatile("cp.reduce.async.bulk.tensor.3d.global.shared::cta.add.tile.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(src), "r"(c0), "r"(c1), "r"(c2)
+               : "memory");
+}
+// Count `bytes` of expected transfer as complete on a barrier of this CTA without a transfer
+// (settles the bytes of copies that were armed but never issued).
+__device__ __forceinline__ void mbar_complete_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.complete_tx.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+// 32-bit store to shared memory of another CTA of the cluster (address from mapa_shared).
+__device__ __forceinline__ void st_shared_cluster_u32(uint32_t cluster_addr, uint32_t v) {
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(cluster_addr), "r"(v) : "memory");
 }
 
 }  // namespace tc

@@ -158,7 +158,7 @@ def loca_device_status(stream=None) -> int:
 
 
 def loca_set_wait_limit(ns: int):
-    """Test hook: how long a device wait of the single-CTA tensor-core kernels may take before it
+    """Test hook: how long a device wait of the tensor-core kernels may take before it
     gives up with LOCA_ERR_TIMEOUT (0 restores the default of 4 s)."""
     _check(lib().loca_set_wait_limit(int(ns)), "loca_set_wait_limit")
 

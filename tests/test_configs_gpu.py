@@ -148,6 +148,9 @@ def _check_stats(tag, gram_g, cross_g, B_g, ref, nl):
     rb = [_rel(_np(B_g[j]), ref["B"][j, 0]) for j in range(nl)]
     print(f"{tag}: rel err gram {rg:.2e} cross {rc:.2e} B {' '.join(f'{v:.2e}' for v in rb)}")
     assert rg <= 2e-3 and rc <= 2e-3 and max(rb) <= 2e-3
+    # the same drift bound as the trace: the segmented accumulation keeps the statistics well
+    # inside the bf16 tolerance at every workload size
+    assert rg <= 2e-4 and rc <= 2e-4
 
 
 # ----------------------------------------------------------------------------- single batch
@@ -238,7 +241,9 @@ def test_single_batch_workload(lc, name, C, kspace):
         rx_sep = (float(o["xsq2"][l]) - x_ref) / x_ref
         print(f"{name} block {l}: ||X||^2 rel err, Gram trace {rx_trace:+.2e}, separate sum {rx_sep:+.2e}")
         assert abs(rx_sep) <= 2e-6
-        assert abs(rx_trace) <= 1e-3
+        # the tensor cores' fp32 accumulation drifts toward zero by a fraction of an ulp per MMA step;
+        # restarting the accumulators every 16384 tokens bounds that drift to ~1e-4 of the sums
+        assert abs(rx_trace) <= 1e-4
         assert abs(-float(o["alpha2"][l]) - ref["steps"][0]) <= 1e-5 * ref["steps"][0]
         cross_g = o["cross"][l] * o["alpha"][l]
         _check_stats(f"{name} block {l}", o["gram"][l], cross_g, o["B"][:, l], ref, nl)

@@ -159,6 +159,7 @@ def _synthetic_stats_inputs(L, N, d, dtype, seed):
     ("bf16", 3, 8, (1, 5)),
     ("bf16", 2, 896, (4096,)),
     ("bf16", 1, 1536, (640, 640)),
+    ("bf16", 2, 640, (40000, 17000)),  # several accumulation segments, ragged; then accumulate
 ])
 def test_accumulate_parity(lc, dtype, L, d, batches):
     """Eqs. 6, 9, 10; S7, S8.  fp32 inputs: fp64 accumulation, one fp32 rounding -> 1e-5 holds
@@ -191,6 +192,35 @@ def test_accumulate_parity(lc, dtype, L, d, batches):
     if dtype == "bf16":
         # bf16 inputs are exact; the only error is fp32 accumulation: far inside 2e-3
         assert rg <= 1e-4 and rc <= 1e-4
+
+
+def test_gram_accumulation_bias_is_bounded_over_long_batches(lc):
+    """Eq. 9 and S7 ask for exact sums.  The tensor cores accumulate in fp32 and lose a fraction of
+    an ulp of the running sum toward zero at every MMA step (K = 16 tokens), so an accumulator fed
+    N tokens drifts by about N/16 such losses relative to its value: 6.5e-4 at 131072 tokens.  The
+    kernel restarts its accumulators every 16384 tokens and adds the segments into the fp32 output
+    with round-to-nearest additions, so the drift no longer grows with N.  At 2^20 tokens in one
+    call: Gram, cross product and the Gram trace (= ||X||^2) within 1e-4 of the fp64 sums."""
+    L, N, d = 1, 1 << 20, 512
+    X, T = _synthetic_stats_inputs(L, N, d, "bf16", seed=77)
+    Xd, Td = _dev(X, torch.bfloat16), _dev(T, torch.bfloat16)
+    gram = torch.empty((L, d, d), dtype=torch.float32, device="cuda")
+    cross = torch.empty_like(gram)
+    tsq = _dev(np.array([np.sum(T[l] ** 2) for l in range(L)]), torch.float64)
+    xsq = torch.empty((L,), dtype=torch.float64, device="cuda")
+    alpha = torch.empty((L,), dtype=torch.float32, device="cuda")
+    lc.loca_gram_cross(Xd, Td, torch.ones((L,), dtype=torch.float32, device="cuda"), gram, cross, zero_first=True)
+    lc.loca_step_from_gram(gram, tsq, 0.01, xsq, alpha)
+    torch.cuda.synchronize()
+    assert lc.loca_device_status() == 0
+    del Xd, Td
+    g_ref = X[0].T @ X[0]
+    c_ref = T[0].T @ X[0]
+    rg, rc = _rel(_np(gram[0]), g_ref), _rel(_np(cross[0]), c_ref)
+    tr = float(np.trace(g_ref))
+    rx = (float(xsq[0]) - tr) / tr
+    print(f"N = 2^20: rel err gram {rg:.2e} cross {rc:.2e} trace {rx:+.2e}")
+    assert rg <= 1e-4 and rc <= 1e-4 and abs(rx) <= 1e-4
 
 
 def test_accumulate_deterministic(lc):

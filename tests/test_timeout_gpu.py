@@ -1,7 +1,8 @@
 """The failure path of the bounded device waits, exercised without faulting or hanging the GPU.
 
 A wait limit of 1 microsecond (the loca_set_wait_limit test hook) makes the first wait of the
-tensor-core kernels that does not succeed at once give up: the kernel must record
+tensor-core kernels (targets, k-space statistics, the CTA-pair Gram / cross kernel) that does not
+succeed at once give up: the kernel must record
 LOCA_ERR_TIMEOUT in the device status word, let its copies and MMAs in flight land, free its
 tensor memory and return.  The CUDA context must stay usable: with the default limit restored,
 the same call then gives results bit-identical to a call made before the failure, and the status
@@ -49,6 +50,15 @@ def _targets_call(lc, E, P, Q, L, N, d):
     return T, tsq
 
 
+def _gram_call(lc, X, T):
+    L, N, d = X.shape
+    gram = torch.empty((L, d, d), device="cuda")
+    cross = torch.empty((L, d, d), device="cuda")
+    lc.loca_gram_cross(X, T, torch.full((L,), -0.5, device="cuda"), gram, cross, zero_first=True)
+    torch.cuda.synchronize()
+    return gram, cross
+
+
 def test_wait_timeout_is_reported_and_the_context_recovers(lc):
     g = torch.Generator(device="cuda")
     g.manual_seed(5)
@@ -60,19 +70,27 @@ def test_wait_timeout_is_reported_and_the_context_recovers(lc):
     Q = torch.randn((L, r, d), device="cuda", generator=g) * 0.25
     lc.loca_set_wait_limit(0)
     assert lc.loca_device_status() == 0
+    T = torch.randn((L, N, d), device="cuda", generator=g).to(torch.bfloat16)
     ref_k = _kspace_call(lc, X, A, E, P, Q)
     ref_t = _targets_call(lc, E, P, Q, L, N, d)
+    ref_g = _gram_call(lc, X, T)
     assert lc.loca_device_status() == 0
-    for call in ("kspace", "targets"):
+    for call in ("kspace", "targets", "gram"):
         lc.loca_set_wait_limit(1000)  # 1 us: a wait that does not succeed at once gives up
         if call == "kspace":
             _kspace_call(lc, X, A, E, P, Q)
-        else:
+        elif call == "targets":
             _targets_call(lc, E, P, Q, L, N, d)
+        else:
+            # the CTA-pair kernel: its roles stop at different points, the odd CTA's half of an
+            # armed stage may never be issued, and every copy, MMA and bulk store still lands
+            # before either CTA of a pair leaves
+            _gram_call(lc, X, T)
         assert lc.loca_device_status() == LOCA_ERR_TIMEOUT, call
         lc.loca_set_wait_limit(0)
         again_k = _kspace_call(lc, X, A, E, P, Q)
         again_t = _targets_call(lc, E, P, Q, L, N, d)
+        again_g = _gram_call(lc, X, T)
         assert lc.loca_device_status() == 0, call
-        for a, b in zip(ref_k + ref_t, again_k + again_t):
+        for a, b in zip(ref_k + ref_t + ref_g, again_k + again_t + again_g):
             assert torch.equal(a, b), call
