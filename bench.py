@@ -43,26 +43,31 @@ METRIC = "LoCA fit tokens/s/block at Qwen2.5-7B shape, 1 GB300; % bf16 tensor-co
 UNIT = "tokens/s/block"
 FALLBACK_SUSTAINED_TFLOPS = 1700.0  # profiling recipe's sustained figure, used if no measured file
 
-# dram bytes (read + write) per launch of k_gram_cross_tc from a one-pass ncu capture of this
-# workload (profiles/gram_cross_tc_qwen2.5-7b.md), valid only for the kernel source whose sha256
-# prefix is given and for the captured (L, N, d); otherwise traffic is reported as null
-GRAM_TC_TRAFFIC = {"sha256": "e55b0d4848cbeaee", "L": 28, "N": 131072, "d": 3584,
-                   "read": 103600324352, "write": 3014398208,
-                   "source": "profiles/gram_cross_tc_qwen2.5-7b.md"}
-# the same for one loca_kspace_accumulate call (k_kspace_prep, k_kspace_xa, k_kspace_ete,
-# k_kspace_final) at k = 16 (profiles/kspace_xa_qwen2.5-7b.md)
-KSPACE_TRAFFIC = {"sha256": "11441129ac44e2da", "L": 28, "N": 131072, "d": 3584, "k": 16,
-                  "read": 26419919872, "write": 27811584,
-                  "source": "profiles/kspace_xa_qwen2.5-7b.md"}
+# DRAM bytes (read + write) per launch from an ncu capture of a small case of the same kernel
+# (L_capture blocks at the workload's own N and d: a few GB on the device), valid only for the
+# kernel source whose sha256 prefix is given.  Work items and rounds repeat block by block, so
+# the traffic of a launch over L blocks is the capture's times L / L_capture; any other N, d or
+# k, or another source, reports null.
+GRAM_TC_TRAFFIC = {"sha256": "90572b4fced76acd", "L_capture": 2, "N": 131072, "d": 3584,
+                   "read": 8479111000, "write": 1260654000,
+                   "kernel": "k_gram_cross_tc"}
+# k_kspace_xa (the k-space statistics kernel, which reads X) at k = 16
+KSPACE_TRAFFIC = {"sha256": "0000195dca10d804", "L_capture": 2, "N": 131072, "d": 3584, "k": 16,
+                  "read": 1885318656, "write": 2222848,
+                  "kernel": "k_kspace_xa"}
+# k_targets_tc (writes T) at r = 16, bf16 output
+TARGETS_TRAFFIC = {"sha256": "c16a9c990782675b", "L_capture": 2, "N": 131072, "d": 3584, "r": 16,
+                   "read": 13240832, "write": 1819753728,
+                   "kernel": "k_targets_tc"}
 
 
-def recorded_traffic(rec, source_file, **shape):
-    """DRAM bytes per launch from a capture record, or None once the kernel source or the shape
-    (every key of ``shape``, which the record must hold) differs from the captured one."""
+def recorded_traffic(rec, source_file, L, **shape):
+    """DRAM bytes per launch over L blocks from a small-case capture record, or None once the
+    kernel source or the shape (every key of ``shape``, which the record must hold) differs."""
     src = open(os.path.join(ROOT, "paper_2608_03020_gb300", "csrc", source_file), "rb").read()
     if rec["sha256"] != hashlib.sha256(src).hexdigest()[:16] or any(rec[n] != v for n, v in shape.items()):
         return None
-    return float(rec["read"] + rec["write"])
+    return float(rec["read"] + rec["write"]) * L / rec["L_capture"]
 
 
 def parse():
@@ -80,6 +85,7 @@ def parse():
     ap.add_argument("--no-calib", action="store_true", help="skip the one-shot d-wide feedback-fit measurement")
     ap.add_argument("--e2e-group", type=int, default=2, help="blocks per host-to-device copy in the e2e leg")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true", help="skip the other workloads' own-shape measurements")
     return ap.parse_args()
 
 
@@ -253,6 +259,188 @@ def run_reference(args, w):
     print(json.dumps(line))
 
 
+# ----------------------------------------------------------------------------- host description
+
+def host_cpu():
+    """Host CPU as lscpu reports it (model, logical CPUs) and the oracle's BLAS thread count."""
+    out = {"cores": os.cpu_count()}
+    try:
+        txt = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=20).stdout
+        for line in txt.splitlines():
+            k, _, v = line.partition(":")
+            k, v = k.strip(), v.strip()
+            if k in ("Architecture", "Model name", "CPU(s)", "Thread(s) per core", "Core(s) per socket", "Socket(s)"):
+                out[k.lower().replace("(s)", "s").replace(" ", "_")] = v
+    except Exception as e:  # lscpu missing: report what Python sees
+        out["lscpu"] = f"unavailable: {e}"
+    return out
+
+
+def tiny_oracle_times():
+    """The fp64 oracle's full pass on the tiny workload (every block and token), with BLAS on all
+    host cores (this process) and single-threaded (a fresh interpreter with one BLAS thread)."""
+    code = ("import time, sys; sys.path.insert(0, %r); from synth import inputs as S; from oracle import loca_oracle as O; "
+            "w = S.WORKLOADS['tiny']; f = S.host_inputs(w); "
+            "run = lambda: O.loca_pass(f['z'], f['label_cols'], f['y'], f['X'], f['P'], f['Q'], f['A'], w.eta, w.lambda_rel); "
+            "run(); t = time.perf_counter(); [run() for _ in range(5)]; print((time.perf_counter() - t) / 5)") % ROOT
+    res = {}
+    for name, threads in (("all_cores_s", None), ("single_thread_s", "1")):
+        env = dict(os.environ)
+        if threads:
+            for v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+                env[v] = threads
+        try:
+            r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=300)
+            res[name] = float(r.stdout.strip().splitlines()[-1])
+        except Exception as e:
+            res[name] = f"failed: {e}"
+    return res
+
+
+# ----------------------------------------------------------------------------- other workloads
+
+def write_peak(buf, stream, reps=3):
+    """Write-only HBM rate of this GPU in this run: torch's fill of ``buf`` (larger than L2)."""
+    import torch
+
+    buf.zero_()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(reps):
+        buf.zero_()
+    b.record(stream)
+    torch.cuda.synchronize()
+    return reps * buf.numel() * buf.element_size() / (a.elapsed_time(b) / 1e3) / 1e9
+
+
+def hbm_object(nbytes, ms, kernel, hbm, wpeak=None):
+    gbs = nbytes / (ms / 1e3) / 1e9
+    o = {"bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s", "frac": gbs / hbm, "kernel": kernel,
+         "bytes_per_launch": float(nbytes), "ms": ms}
+    if wpeak:
+        o["write_peak_gbs"] = wpeak
+        o["frac_of_write_peak"] = gbs / wpeak
+    return o
+
+
+def measure_workload(lc, name, dev, stream, steps, warmup, peak, hbm, wpeak):
+    """One step of workload `name` at its own shape, timed like the headline: error -> targets ->
+    statistics -> solve (single mini-batch: the cross product at alpha = 1, the step from the Gram
+    trace, alpha in the solve; several mini-batches: targets and loca_accumulate per batch)."""
+    import torch
+
+    from synth import inputs as S
+
+    w = S.WORKLOADS[name]
+    inp = S.device_inputs(w, seed=0, device=dev)
+    X, z, y, cols, P, Q, A = (inp[k] for k in ("X", "z", "y", "label_cols", "P", "Q", "A"))
+    L, N, d, C, r, k = w.L, w.N, w.d, w.C, w.r, w.k
+    mb, nb = w.micro_batches, w.tokens_per_batch
+    nl = len(w.lambda_rel)
+    act = X.dtype
+    if mb > 1:  # contiguous per-batch inputs (L x nb x d each)
+        X = X.view(L, mb, nb, d).permute(1, 0, 2, 3).contiguous()
+        inp["X"] = None
+    f32 = dict(dtype=torch.float32, device=dev)
+    E = torch.empty((N, C), **f32)
+    ce = torch.empty((N,), **f32)
+    T = torch.empty((L, nb, d), dtype=act, device=dev)
+    tsq = torch.empty((L,), dtype=torch.float64, device=dev)
+    xsq = torch.empty((L,), dtype=torch.float64, device=dev)
+    alpha = torch.empty((L,), **f32)
+    ones = torch.ones((L,), **f32)
+    gram = torch.empty((L, d, d), **f32)
+    cross = torch.empty((L, d, d), **f32)
+    B = torch.empty((nl, L, d, k), **f32)
+    info = torch.empty((nl, L), dtype=torch.int32, device=dev)
+    ws_t = torch.empty(lc.targets_workspace_size(nb, L, d), dtype=torch.uint8, device=dev)
+    ws_a = torch.empty(lc.accumulate_workspace_size(L, nb, d, act), dtype=torch.uint8, device=dev)
+    ws_g = torch.empty(lc.gram_cross_workspace_size(), dtype=torch.uint8, device=dev)
+    ws_s = torch.empty(lc.ridge_solve_workspace_size(L, d, k), dtype=torch.uint8, device=dev)
+    names = ["error", "targets", "statistics", "step", "ridge_solve"]
+
+    def step(ev=None):
+        t = {n: 0.0 for n in names}
+        marks = []
+
+        def mark(n):
+            if ev is not None:
+                e = torch.cuda.Event(enable_timing=True)
+                e.record(stream)
+                marks.append((n, e))
+
+        mark("start")
+        lc.loca_error(z, cols, y, E, ce=ce, stream=stream)
+        mark("error")
+        if mb == 1:
+            lc.loca_targets(E, P, Q, T, tsq=tsq, workspace=ws_t, stream=stream)
+            mark("targets")
+            lc.loca_gram_cross(X, T, ones, gram, cross, zero_first=True, workspace=ws_g, stream=stream)
+            mark("statistics")
+            lc.loca_step_from_gram(gram, tsq, w.eta, xsq, alpha, stream=stream)
+            mark("step")
+            lc.loca_ridge_solve(gram, cross, A, w.lambda_rel, B, info, xsq_total=xsq, cross_scale=alpha,
+                                workspace=ws_s, stream=stream)
+        else:
+            for m in range(mb):
+                lc.loca_targets(E[m * nb:(m + 1) * nb], P, Q, T, tsq=tsq, workspace=ws_t, stream=stream)
+                mark("targets")
+                lc.loca_accumulate(X[m], T, tsq, w.eta, gram, cross, xsq, zero_first=(m == 0), workspace=ws_a,
+                                   stream=stream)
+                mark("statistics")
+            mark("step")
+            lc.loca_ridge_solve(gram, cross, A, w.lambda_rel, B, info, xsq_total=xsq, workspace=ws_s, stream=stream)
+        mark("ridge_solve")
+        if ev is not None:
+            ev.append((marks, t))
+
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize()
+    evs = []
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(steps):
+        step(evs)
+    b.record(stream)
+    torch.cuda.synchronize()
+    if lc.loca_device_status() != 0 or int(info.abs().sum().item()) != 0:
+        raise SystemExit(f"{name}: a device error or a non-PD system")
+    ms = a.elapsed_time(b) / steps
+    stages = {n: 0.0 for n in names}
+    for marks, _ in evs:
+        for (_, e0), (n1, e1) in zip(marks, marks[1:]):
+            stages[n1] += e0.elapsed_time(e1) / steps
+    out = {"L": L, "d": d, "N": N, "C": C, "V": w.V, "r": r, "k": k, "micro_batches": mb,
+           "dtype": "bf16" if act == torch.bfloat16 else "f32",
+           "value": N * L / (ms / 1e3), "unit": UNIT, "ms_per_step": ms, "stages_ms": stages,
+           "solve_ms": stages["ridge_solve"], "steps": steps, "warmup": warmup}
+    if act == torch.bfloat16:
+        flops = L * (2.0 * N * d * d + N * d * (d + 1.0))
+        ach = flops / (stages["statistics"] / 1e3) / 1e12
+        out["gram_roofline"] = {"bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
+                                "frac": ach / peak, "kernel": "k_gram_cross_tc (+ k_gram_mirror)"
+                                + (", k_sumsq / k_step per batch" if mb > 1 else ""),
+                                "flops_per_step": flops}
+    else:
+        out["gram_path"] = "fp32 inputs: k_gram_cross_f32 (CUDA cores, fp64 accumulation)"
+    zb = N * V_bytes(z)
+    out["error_roofline"] = hbm_object(zb + N * C * 4, stages["error"], "k_head_error", hbm)
+    out["error_roofline"]["graded"] = w.V > 64 * w.C  # launch-bound when the row holds only the labels
+    out["targets_roofline"] = hbm_object(L * N * d * T.element_size(), stages["targets"], "k_targets_tc", hbm,
+                                         wpeak)
+    out["ridge_solve_roofline"] = hbm_object(2 * L * d * d * 4, stages["ridge_solve"],
+                                             "k_project_rows + k_chol_solve (reads of Gram and cross)", hbm)
+    del inp, X, z, T, gram, cross, E, ce, B
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    return out
+
+
+def V_bytes(z):
+    return z.shape[1] * z.element_size()
+
+
 # ----------------------------------------------------------------------------- GPU arm
 
 def main():
@@ -267,6 +455,14 @@ def main():
         if rank == 0:
             run_reference(args, w)
         return
+
+    world0 = int(os.environ.get("WORLD_SIZE", "1"))
+    rank0 = int(os.environ.get("RANK", "0"))
+    host_info, tiny_times = None, None
+    if rank0 == 0 and world0 == 1 and not args.no_cpu_baseline:
+        # host-side only, before this process touches the GPU
+        host_info = host_cpu()
+        tiny_times = tiny_oracle_times()
 
     import numpy as np
     import torch
@@ -300,7 +496,7 @@ def main():
     ws_g = torch.empty(lc.gram_cross_workspace_size(), dtype=torch.uint8, device=dev)
     ws_s = torch.empty(lc.ridge_solve_workspace_size(L, d, k), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
-    launches_per_step = 1 + 2 + 1 + 1 + 2  # error; targets+reduce; gram/cross; step; project+solve
+    launches_per_step = 1 + 2 + 2 + 1 + 2  # error; targets+reduce; gram/cross+mirror; step; project+solve
 
     def step(ev=None):
         if ev is not None:
@@ -330,6 +526,9 @@ def main():
     status = lc.loca_device_status()
     if status != 0:
         raise SystemExit(f"device status {status} after warm-up")
+    # this GPU's write-only HBM rate in this run (a fill of T's 26 GB), the ceiling of the targets
+    # kernel, whose traffic is the write of T
+    wpeak = write_peak(T, stream)
 
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
     uuid = None
@@ -365,10 +564,15 @@ def main():
     peak, peak_kind = peaks()
     flops = L * (2.0 * N * d * d + N * d * (d + 1.0))
     achieved = flops / (stages["gram_cross"] / 1e3) / 1e12
-    traffic = recorded_traffic(GRAM_TC_TRAFFIC, "gram_tc.cu", L=L, N=N, d=d)
+    traffic = recorded_traffic(GRAM_TC_TRAFFIC, "gram_tc.cu", L, N=N, d=d)
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "traffic": traffic, "kernel": "k_gram_cross_tc",
                 "peak_kind": f"bf16 dense sustained, {peak_kind}", "flops_per_launch": flops}
+    hbm = hbm_peak()
+    targets_roofline = hbm_object(L * N * d * T.element_size(), stages["targets"], "k_targets_tc", hbm, wpeak)
+    targets_roofline["traffic"] = recorded_traffic(TARGETS_TRAFFIC, "targets.cu", L, N=N, d=d, r=r)
+    solve_roofline = hbm_object(2 * L * d * d * 4, stages["ridge_solve"],
+                                "k_project_rows + k_chol_solve (reads of Gram and cross)", hbm)
 
     # the paper's own k-space statistics on the same inputs (no T, no d x d statistics):
     # error -> k-space accumulate (X A_l on the tensor cores, one HBM read of X) -> k-space solve
@@ -419,7 +623,8 @@ def main():
                   "roofline": {"bound": "hbm", "achieved": xbytes / (kst["accumulate"] / 1e3) / 1e9,
                                "peak": hbm_peak(), "unit": "GB/s",
                                "frac": xbytes / (kst["accumulate"] / 1e3) / 1e9 / hbm_peak(),
-                               "traffic": recorded_traffic(KSPACE_TRAFFIC, "kspace.cu", L=L, N=N, d=d, k=k),
+                               "traffic": recorded_traffic(KSPACE_TRAFFIC, "kspace.cu", L, N=N, d=d, k=k),
+                               "traffic_kernel": "k_kspace_xa",
                                "kernel": "loca_kspace_accumulate (prep, X A on tcgen05, stats, final)",
                                "bytes_per_launch": xbytes}}
 
@@ -564,6 +769,20 @@ def main():
             raise SystemExit("the end-to-end steps reported a device error or a non-PD system")
         del hX, hz, staging
 
+    x_gb = X.numel() * X.element_size() / 1e9
+    # every other workload at its own shape (the headline's buffers released first)
+    configs = None
+    if not args.no_configs and world == 1:
+        del X, z, T, gram, cross, inp, ws_t, ws_g, ws_s, B, E, ce
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+        configs = {}
+        for name in ("tiny", "qwen2.5-0.5b", "qwen2.5-1.5b", "smollm2-1.7b", "qwen2.5-14b"):
+            if name == w.name:
+                continue
+            configs[name] = measure_workload(lc, name, dev, stream, max(1, min(args.steps, 5)), args.warmup, peak,
+                                             hbm, wpeak)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         # bounded sample: one block, a token prefix sized from a 2048-token pilot run to take about
@@ -577,7 +796,8 @@ def main():
         sec = oracle_sample(w, tokens, host)
         cpu = {"value": tokens / sec, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
                "sample": f"one block (of {L}), first {tokens} of {N} tokens, full d={d}, C={C}, r={r}, k={k}; "
-                         f"numpy fp64, {sec:.1f} s"}
+                         f"numpy fp64, {sec:.1f} s",
+               "host": host_info, "tiny_workload_full_pass": tiny_times}
 
     if rank == 0:
         line = {
@@ -586,10 +806,14 @@ def main():
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": w.name, "L": L, "d": d, "N": N, "C": C, "r": r, "k": k,
                        "lambda_rel": list(w.lambda_rel), "eta": w.eta, "parallelism": f"replicas{world}",
-                       "l2": "inputs larger than L2 (X is %.1f GB)" % (X.numel() * X.element_size() / 1e9)},
+                       "l2": "inputs larger than L2 (X is %.1f GB)" % x_gb},
             "stages_ms": stages,
             "solve_ms": stages["ridge_solve"],
             "roofline": roofline,
+            "targets_roofline": targets_roofline,
+            "ridge_solve_roofline": solve_roofline,
+            "write_peak_gbs": wpeak,
+            "configs": configs,
             "gpu_launches": launches_per_step * args.steps,
             "e2e": e2e,
             "kspace": kspace,

@@ -55,7 +55,7 @@ def _inputs(L, N, d, k, C, r, seed):
     (3, 4097, 896, 32, 16, 32, 1, True),   # k = 32 (two TMEM loads), C and r at their limits
     (1, 300, 64, 4, 1, 1, 1, False),       # smallest shapes (k padded to 16)
     (2, 2500, 512, 16, 4, 16, 2, True),    # two mini-batches: zero_first, then accumulate
-    (2, 1500, 200, 20, 3, 12, 1, True),    # k = 20 padded to 32 (pairs recomputed per tile), ragged d, N
+    (2, 1500, 200, 20, 3, 12, 1, True),    # k = 20 padded to 32 (2 x 2 register-blocked statistics), ragged d, N
 ])
 def test_kspace_matches_dense_oracle(lc, L, N, d, k, C, r, batches, with_prev):
     eta = 0.02
