@@ -86,6 +86,7 @@ def parse():
     ap.add_argument("--e2e-group", type=int, default=2, help="blocks per host-to-device copy in the e2e leg")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-configs", action="store_true", help="skip the other workloads' own-shape measurements")
+    ap.add_argument("--no-fused", action="store_true", help="skip the fused-targets pass")
     return ap.parse_args()
 
 
@@ -628,6 +629,62 @@ def main():
                                "kernel": "loca_kspace_accumulate (prep, X A on tcgen05, stats, final)",
                                "bytes_per_launch": xbytes}}
 
+    # the same pass with the targets generated inside the statistics kernel (T never written):
+    # error -> ||T||^2 in closed form -> fused Gram / cross at alpha = 1 -> step -> solve
+    fused = None
+    if not args.no_fused and X.dtype == torch.bfloat16:
+        tsq_f = torch.empty((L,), dtype=torch.float64, device=dev)
+        ws_q = torch.empty(lc.targets_sq_workspace_size(N, C), dtype=torch.uint8, device=dev)
+        ws_f = torch.empty(lc.gram_cross_fused_workspace_size(L, N, r), dtype=torch.uint8, device=dev)
+
+        def fstep(ev=None):
+            if ev is not None:
+                ev[0].record(stream)
+            lc.loca_error(z, cols, y, E, ce=ce, stream=stream)
+            if ev is not None:
+                ev[1].record(stream)
+            lc.loca_targets_sq(E, P, Q, tsq_f, workspace=ws_q, stream=stream)
+            if ev is not None:
+                ev[2].record(stream)
+            lc.loca_gram_cross_fused(X, E, P, Q, ones, gram, cross, zero_first=True, workspace=ws_f, stream=stream)
+            if ev is not None:
+                ev[3].record(stream)
+            lc.loca_step_from_gram(gram, tsq_f, w.eta, xsq, alpha, stream=stream)
+            if ev is not None:
+                ev[4].record(stream)
+            lc.loca_ridge_solve(gram, cross, A, w.lambda_rel, B, info, xsq_total=xsq, cross_scale=alpha,
+                                workspace=ws_s, stream=stream)
+            if ev is not None:
+                ev[5].record(stream)
+
+        for _ in range(args.warmup):
+            fstep()
+        torch.cuda.synchronize()
+        fev = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
+        barrier(world)
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for i in range(args.steps):
+            fstep(fev[i])
+        b.record(stream)
+        torch.cuda.synchronize()
+        ms_f = max_over_ranks(world, a.elapsed_time(b)) / args.steps
+        if lc.loca_device_status() != 0 or int(info.abs().sum().item()) != 0:
+            raise SystemExit("the fused-targets steps reported a device error or a non-PD system")
+        fst = {n: statistics.mean(e[i].elapsed_time(e[i + 1]) for e in fev)
+               for i, n in enumerate(["error", "targets_sq", "gram_cross_fused", "step", "ridge_solve"])}
+        ach_f = flops / (fst["gram_cross_fused"] / 1e3) / 1e12
+        fused = {"value": world * N * L / (ms_f / 1e3), "unit": UNIT, "ms_per_step": ms_f, "stages_ms": fst,
+                 "vs_split": {"targets_plus_gram_ms": stages["targets"] + stages["gram_cross"],
+                              "targets_sq_plus_fused_ms": fst["targets_sq"] + fst["gram_cross_fused"]},
+                 "roofline": {"bound": "tensor", "achieved": ach_f, "peak": peak, "unit": "TFLOP/s",
+                              "frac": ach_f / peak, "kernel": "k_gram_cross_tc<fused> (+ k_gram_mirror)",
+                              "flops_per_launch": flops, "note": "useful flops of the statistics only; the "
+                              "generation of T adds 6 N d r flops per block on the tensor cores"}}
+        del ws_q, ws_f
+
     # the head error where it is HBM-bound: the Qwen2.5-14B row of the workloads (N = 131072 tokens,
     # V = 151936 bf16 logits, C = 4 label columns; 39.8 GB of logits, drawn as in synth)
     vocab = None
@@ -817,6 +874,7 @@ def main():
             "gpu_launches": launches_per_step * args.steps,
             "e2e": e2e,
             "kspace": kspace,
+            "fused_targets": fused,
             "head_error_vocab": vocab,
             "calibration": calib,
             "cpu_baseline": cpu,

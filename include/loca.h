@@ -284,6 +284,37 @@ int loca_gram_cross(const void* X, const void* T, int dtype, int32_t L, int64_t 
                     size_t workspace_bytes, void* stream);
 
 /*
+ * Fused targets: the Gram / cross statistics with each block's targets generated inside the
+ * tensor-core kernel instead of read from memory (S3: Q_l := F_l E; S11: F e applied through
+ * the factors).  Together with loca_targets_sq they replace loca_targets + loca_gram_cross; T is
+ * never written, so the statistics read only X from HBM.
+ *
+ * loca_targets_sq (S3, S11; the ||Q_l||^2 of the step in Eq. 10):
+ *   tsq[l] = ||E P_l Q_l||_F^2 = < P_l (Q_l Q_l^T) P_l^T , E^T E >, without forming T.
+ *   E N x C, P L x C x r, Q L x r x d (fp32, row-major, device); tsq L doubles (device, out).
+ *   1 <= C <= 64, 1 <= r <= 32.  fp32 products summed in fp64; deterministic.
+ *   Workspace: loca_targets_sq_workspace_size(N, C) bytes (partial sums of E^T E).
+ * loca_gram_cross_fused (Eq. 9; S7): gram_l (+)= X_l^T X_l, cross_l (+)= alpha[l] T_l^T X_l with
+ *   T_l = (E P_l) Q_l formed tile by tile on the tensor cores (bf16 hi / lo parts of U = E P_l and
+ *   of Q_l, three products, ~2^-17 per element) and rounded once to bf16 before it meets X, as
+ *   loca_gram_cross does with a T from loca_targets.  X: L x N x d bf16 only (dtype LOCA_BF16),
+ *   E, P, Q as loca_targets_sq, 1 <= r <= 32, C <= 64.  Workspace:
+ *   loca_gram_cross_fused_workspace_size(L, N, r) bytes (launch-local flags and U_l = E P_l as
+ *   bf16 hi / lo parts, 4 L N rp bytes with rp = 16 for r <= 16, else 32).  Other arguments,
+ *   layouts and determinism as loca_gram_cross.
+ *   Cost: the cross tiles take one accumulator each (the T generation needs the other TMEM
+ *   half), so this kernel does more passes over X than loca_gram_cross; it saves the write of
+ *   T and its reads.
+ */
+int loca_targets_sq_workspace_size(int64_t N, int32_t C, size_t* bytes /* host */);
+int loca_targets_sq(const float* E, int64_t N, int32_t C, const float* P, const float* Q, int32_t L, int32_t r,
+                    int64_t d, double* tsq, void* workspace, size_t workspace_bytes, void* stream);
+int loca_gram_cross_fused_workspace_size(int32_t L, int64_t N, int32_t r, size_t* bytes /* host */);
+int loca_gram_cross_fused(const void* X, int dtype, int32_t L, int64_t N, int64_t d, const float* E, int32_t C,
+                          const float* P, const float* Q, int32_t r, const float* alpha, int zero_first,
+                          float* gram, float* cross, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
  * loca_accumulate_noalloc — loca_accumulate for callers that cannot provide device scratch
  * memory.  The paper has no counterpart: it concerns only how this library obtains scratch.
  *
@@ -298,8 +329,10 @@ int loca_gram_cross(const void* X, const void* T, int dtype, int32_t L, int64_t 
  *
  * Limits and use:
  *  - L <= 64 blocks; a larger L is rejected with LOCA_ERR_SHAPE (use loca_accumulate).
- *  - The first call on each device looks up the array's device address (cudaGetSymbolAddress,
- *    with that device current) and caches it; make that first call before any stream capture.
+ *  - Every call looks up the array's device address in the current context
+ *    (cudaGetSymbolAddress, with the caller's device current; the lookup allocates nothing and
+ *    stays valid after a cudaDeviceReset).  The first lookup on a device may load the library's
+ *    device code there: make the first call on each device before any stream capture.
  *  - Every call reuses the same array.  Calls whose work may overlap on the GPU (different
  *    streams, or threads without ordering between them) race on it: serialise them.
  *  - Calls no cudaMalloc, cudaFree or other allocating routine.

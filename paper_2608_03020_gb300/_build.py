@@ -18,7 +18,8 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libloca.so")
 SOURCES = ["loca_abi.cu", "error.cu", "targets.cu", "stats.cu", "gram_tc.cu", "solve.cu", "calib.cu",
-           "noalloc.cu", "host_mem.cu", "kspace.cu", "align.cu", "calib_rsvd.cu"]
+           "noalloc.cu", "host_mem.cu", "kspace.cu", "align.cu", "calib_rsvd.cu",
+           "targets_sq.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVFLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
                   "-I" + os.path.join(ROOT, "include")]

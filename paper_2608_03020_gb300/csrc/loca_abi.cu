@@ -261,7 +261,7 @@ int loca_targets(const float* E, int64_t N, int32_t C, const float* P, const flo
 
 }  // extern "C"
 
-namespace {
+namespace loca {
 
 int validate_stats_inputs(const void* X, const void* T, int dtype, int32_t L, int64_t N, int64_t d,
                           bool need_T) {
@@ -277,6 +277,19 @@ int validate_stats_inputs(const void* X, const void* T, int dtype, int32_t L, in
   } else {
     if (N > 0 && (!aligned(X, 4) || (need_T && !aligned(T, 4)))) return fail(LOCA_ERR_ALIGNMENT, "X and T need 4-byte alignment");
   }
+  return LOCA_OK;
+}
+
+int validate_accumulate(const void* X, const void* T, int dtype, int32_t L, int64_t N, int64_t d,
+                        const double* tsq, float eta, const float* gram, const float* cross,
+                        const double* xsq_total) {
+  const int rc = validate_stats_inputs(X, T, dtype, L, N, d, true);
+  if (rc != LOCA_OK) return rc;
+  if (!(eta >= 0.f)) return fail(LOCA_ERR_INVALID_ARG, "eta must be >= 0");
+  if (!tsq || !gram || !cross || !xsq_total)
+    return fail(LOCA_ERR_INVALID_ARG, "tsq, gram, cross and xsq_total are required");
+  if (!aligned(gram, 16) || !aligned(cross, 16) || !aligned(tsq, 8) || !aligned(xsq_total, 8))
+    return fail(LOCA_ERR_ALIGNMENT, "gram and cross need 16-byte, tsq and xsq_total 8-byte alignment");
   return LOCA_OK;
 }
 
@@ -311,6 +324,10 @@ int run_gram_cross(const void* X, const void* T, int dtype, int32_t L, int64_t N
   if (e != cudaSuccess) return cuda_fail(e, "Gram/cross launch");
   return LOCA_OK;
 }
+
+}  // namespace loca
+
+namespace {
 
 size_t batch_step_ws(int32_t L) { return align256(sizeof(double) * size_t(L) * size_t(sumsq_num_partials())); }
 constexpr size_t kGramCrossWs = 256;
@@ -363,6 +380,64 @@ int loca_gram_cross(const void* X, const void* T, int dtype, int32_t L, int64_t 
                         reinterpret_cast<int32_t*>(workspace), static_cast<cudaStream_t>(stream));
 }
 
+int loca_targets_sq_workspace_size(int64_t N, int32_t C, size_t* bytes) {
+  if (!bytes) return fail(LOCA_ERR_INVALID_ARG, "bytes is NULL");
+  if (N < 0 || C < 1 || C > tsq_max_C()) return fail(LOCA_ERR_SHAPE, "need N >= 0 and 1 <= C <= %d", tsq_max_C());
+  *bytes = tsq_workspace_bytes(N, C);
+  return LOCA_OK;
+}
+
+int loca_targets_sq(const float* E, int64_t N, int32_t C, const float* P, const float* Q, int32_t L, int32_t r,
+                    int64_t d, double* tsq, void* workspace, size_t workspace_bytes, void* stream) {
+  g_msg[0] = 0;
+  if (N < 0 || L < 1 || L > 65535 || d < 1) return fail(LOCA_ERR_SHAPE, "need N >= 0, 1 <= L <= 65535, d >= 1");
+  if (C < 1 || C > tsq_max_C()) return fail(LOCA_ERR_SHAPE, "need 1 <= C <= %d, got C=%d", tsq_max_C(), C);
+  if (r < 1 || r > tsq_max_r()) return fail(LOCA_ERR_SHAPE, "need 1 <= r <= %d, got %d", tsq_max_r(), r);
+  if ((N > 0 && !E) || !P || !Q || !tsq) return fail(LOCA_ERR_INVALID_ARG, "E, P, Q and tsq are required");
+  if (!aligned(E, 4) || !aligned(P, 4) || !aligned(Q, 4) || !aligned(tsq, 8))
+    return fail(LOCA_ERR_ALIGNMENT, "E, P, Q need 4-byte and tsq 8-byte alignment");
+  const int rc = check_ws(workspace, workspace_bytes, tsq_workspace_bytes(N, C));
+  if (rc != LOCA_OK) return rc;
+  const cudaError_t e = launch_targets_sq(E, N, C, P, Q, L, r, d, tsq, workspace, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "loca_targets_sq launch");
+  return LOCA_OK;
+}
+
+int loca_gram_cross_fused_workspace_size(int32_t L, int64_t N, int32_t r, size_t* bytes) {
+  if (!bytes) return fail(LOCA_ERR_INVALID_ARG, "bytes is NULL");
+  if (L < 1 || N < 0 || r < 1 || r > gram_fused_max_r())
+    return fail(LOCA_ERR_SHAPE, "need L >= 1, N >= 0 and 1 <= r <= %d", gram_fused_max_r());
+  *bytes = gram_fused_workspace_bytes(L, N, r);
+  return LOCA_OK;
+}
+
+int loca_gram_cross_fused(const void* X, int dtype, int32_t L, int64_t N, int64_t d, const float* E, int32_t C,
+                          const float* P, const float* Q, int32_t r, const float* alpha, int zero_first,
+                          float* gram, float* cross, void* workspace, size_t workspace_bytes, void* stream) {
+  g_msg[0] = 0;
+  if (dtype != LOCA_BF16)
+    return fail(LOCA_ERR_UNSUPPORTED_DTYPE, "loca_gram_cross_fused takes bf16 X (LOCA_BF16) only");
+  int rc = validate_stats_inputs(X, X, dtype, L, N, d, false);
+  if (rc != LOCA_OK) return rc;
+  if (C < 1 || C > tsq_max_C()) return fail(LOCA_ERR_SHAPE, "need 1 <= C <= %d, got C=%d", tsq_max_C(), C);
+  if (r < 1 || r > gram_fused_max_r()) return fail(LOCA_ERR_SHAPE, "need 1 <= r <= %d, got %d", gram_fused_max_r(), r);
+  if ((N > 0 && !E) || !P || !Q || !alpha || !gram || !cross)
+    return fail(LOCA_ERR_INVALID_ARG, "E, P, Q, alpha, gram and cross are required");
+  if (!aligned(gram, 16) || !aligned(cross, 16) || !aligned(alpha, 4) || !aligned(E, 4) || !aligned(P, 4) ||
+      !aligned(Q, 4))
+    return fail(LOCA_ERR_ALIGNMENT, "gram and cross need 16-byte, alpha, E, P, Q 4-byte alignment");
+  rc = check_ws(workspace, workspace_bytes, gram_fused_workspace_bytes(L, N, r));
+  if (rc != LOCA_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (N == 0) return run_gram_cross(X, X, dtype, L, N, d, alpha, zero_first, gram, cross, nullptr, s);
+  int32_t* status = device_status_word();
+  if (!status) return fail(LOCA_ERR_CUDA, "cannot resolve the device status word");
+  const cudaError_t e = launch_gram_cross_fused_tc(X, E, C, P, Q, r, L, N, d, alpha, zero_first, gram, cross, status,
+                                                   workspace, s);
+  if (e != cudaSuccess) return cuda_fail(e, "loca_gram_cross_fused launch");
+  return LOCA_OK;
+}
+
 int loca_accumulate_workspace_size(int32_t L, int64_t N, int64_t d, int dtype, size_t* bytes) {
   (void)N;
   (void)d;
@@ -377,13 +452,8 @@ int loca_accumulate(const void* X, const void* T, int dtype, int32_t L, int64_t 
                     const double* tsq, float eta, int zero_first, float* gram, float* cross,
                     double* xsq_total, void* workspace, size_t workspace_bytes, void* stream) {
   g_msg[0] = 0;
-  int rc = validate_stats_inputs(X, T, dtype, L, N, d, true);
+  int rc = validate_accumulate(X, T, dtype, L, N, d, tsq, eta, gram, cross, xsq_total);
   if (rc != LOCA_OK) return rc;
-  if (!(eta >= 0.f)) return fail(LOCA_ERR_INVALID_ARG, "eta must be >= 0");
-  if (!tsq || !gram || !cross || !xsq_total)
-    return fail(LOCA_ERR_INVALID_ARG, "tsq, gram, cross and xsq_total are required");
-  if (!aligned(gram, 16) || !aligned(cross, 16) || !aligned(tsq, 8) || !aligned(xsq_total, 8))
-    return fail(LOCA_ERR_ALIGNMENT, "gram and cross need 16-byte, tsq and xsq_total 8-byte alignment");
   const AccumWs lay = accum_ws(L);
   rc = check_ws(workspace, workspace_bytes, lay.total);
   if (rc != LOCA_OK) return rc;

@@ -65,6 +65,35 @@ cudaError_t launch_gram_cross_tc(const void* X, const void* T, int L, int64_t N,
                                  const float* alpha, int zero_first, float* gram, float* cross,
                                  int32_t* status, int32_t* abort_flag, cudaStream_t s);
 
+// Gram / cross with the targets generated in the kernel from E, P, Q (bf16 X only); r <= 32.
+// Workspace: launch-local flags (256 bytes), then U_l = E P_l as bf16 hi / lo parts.
+int gram_fused_max_r();
+size_t gram_fused_workspace_bytes(int L, int64_t N, int r);
+cudaError_t launch_gram_cross_fused_tc(const void* X, const float* E, int C, const float* P, const float* Q,
+                                       int r, int L, int64_t N, int64_t d, const float* alpha, int zero_first,
+                                       float* gram, float* cross, int32_t* status, void* workspace,
+                                       cudaStream_t s);
+// ||T_l||^2 in closed form (targets_sq.cu); workspace: tsq_workspace_bytes(N, C).
+int tsq_max_C();
+int tsq_max_r();
+size_t tsq_workspace_bytes(int64_t N, int C);
+cudaError_t launch_targets_sq(const float* E, int64_t N, int C, const float* P, const float* Q, int L, int r,
+                              int64_t d, double* tsq, void* workspace, cudaStream_t s);
+
+// Host-side checks and launches shared by the statistics entry points (loca_abi.cu): they set the
+// message of loca_last_error_string() and return a loca_status.
+int validate_stats_inputs(const void* X, const void* T, int dtype, int32_t L, int64_t N, int64_t d,
+                          bool need_T);
+int validate_accumulate(const void* X, const void* T, int dtype, int32_t L, int64_t N, int64_t d,
+                        const double* tsq, float eta, const float* gram, const float* cross,
+                        const double* xsq_total);
+int run_batch_step(const void* X, int dtype, int32_t L, int64_t N, int64_t d, const double* tsq,
+                   float eta, int zero_first, double* xsq_total, float* alpha, double* partials,
+                   cudaStream_t s);
+int run_gram_cross(const void* X, const void* T, int dtype, int32_t L, int64_t N, int64_t d,
+                   const float* alpha, int zero_first, float* gram, float* cross, int32_t* abort_flag,
+                   cudaStream_t s);
+
 // Limit of the bounded device waits of the tensor-core kernels (targets, k-space statistics,
 // Gram / cross): 4 s unless loca_set_wait_limit changed it.
 unsigned long long wait_limit_ns();

@@ -53,20 +53,22 @@ struct WaitCtl {
 
 // Bounded wait for the phase of parity `parity` of barrier `bar`.  Returns false when the wait
 // gave up (time limit reached, or another waiter of this launch gave up).  A try_wait that fails
-// may itself have suspended the thread for a while, so the limit is checked every 8 of them.
+// may itself have suspended the thread for a while, so the clock (a register read) is checked
+// every 8 of them; the launch's abort flag lives in global memory, and a thread stalled on that
+// load cannot see its barrier complete, so it is read only every 128.
 static __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const WaitCtl& w) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 7u) == 0) {
-      if (*w.abort_flag != 0) return false;
       if (globaltimer() - t0 > w.limit_ns) {
         atomicExch(w.status, int32_t(LOCA_ERR_TIMEOUT));
         *w.abort_flag = 1;
         __threadfence();
         return false;
       }
+      if ((it & 127u) == 0 && *w.abort_flag != 0) return false;
     }
   }
 }
@@ -132,13 +134,13 @@ static __device__ __noinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t par
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait_cluster(bar, parity)) return true;
     if ((it & 7u) == 0) {
-      if (*w.abort_flag != 0) return false;
       if (globaltimer() - t0 > w.limit_ns) {
         atomicExch(w.status, int32_t(LOCA_ERR_TIMEOUT));
         *w.abort_flag = 1;
         __threadfence();
         return false;
       }
+      if ((it & 127u) == 0 && *w.abort_flag != 0) return false;
     }
   }
 }

@@ -62,6 +62,11 @@ SIGNATURES = [
     ("loca_gram_cross_workspace_size", ctypes.c_int, [ctypes.POINTER(_SZ)]),
     ("loca_gram_cross", ctypes.c_int,
      [_P, _P, ctypes.c_int, _I32, _I64, _I64, _P, ctypes.c_int, _P, _P, _P, _SZ, _P]),
+    ("loca_targets_sq_workspace_size", ctypes.c_int, [_I64, _I32, ctypes.POINTER(_SZ)]),
+    ("loca_targets_sq", ctypes.c_int, [_P, _I64, _I32, _P, _P, _I32, _I32, _I64, _P, _P, _SZ, _P]),
+    ("loca_gram_cross_fused_workspace_size", ctypes.c_int, [_I32, _I64, _I32, ctypes.POINTER(_SZ)]),
+    ("loca_gram_cross_fused", ctypes.c_int,
+     [_P, ctypes.c_int, _I32, _I64, _I64, _P, _I32, _P, _P, _I32, _P, ctypes.c_int, _P, _P, _P, _SZ, _P]),
     ("loca_ridge_solve_workspace_size", ctypes.c_int, [_I32, _I64, _I32, ctypes.POINTER(_SZ)]),
     ("loca_ridge_solve", ctypes.c_int,
      [_P, _P, _P, _P, _P, _P, ctypes.POINTER(_F), _I32, _I32, _I64, _I32, _P, _P, _P, _P, _P, _SZ, _P]),
@@ -436,6 +441,57 @@ def loca_gram_cross(X, T, alpha, gram, cross, zero_first, workspace=None, stream
     rc = lib().loca_gram_cross(_ptr(X), _ptr(T), _code(X.dtype), L, N, d, _ptr(alpha), int(bool(zero_first)),
                                _ptr(gram), _ptr(cross), _ptr(ws), nbytes, _stream(stream))
     _check(rc, "loca_gram_cross")
+
+
+def targets_sq_workspace_size(N, C) -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib().loca_targets_sq_workspace_size(N, C, ctypes.byref(out)), "loca_targets_sq_workspace_size")
+    return out.value
+
+
+def loca_targets_sq(E, P, Q, tsq, workspace=None, stream=None):
+    """``tsq[l] = ||E P_l Q_l||_F^2`` (float64, L) without forming the targets."""
+    _dev(E, "E", torch.float32, 2)
+    _dev(P, "P", torch.float32, 3)
+    _dev(Q, "Q", torch.float32, 3)
+    _dev(tsq, "tsq", torch.float64, 1)
+    N, C = E.shape
+    L, C2, r = P.shape
+    L2, r2, d = Q.shape
+    if C2 != C or L2 != L or r2 != r or tuple(tsq.shape) != (L,):
+        raise ValueError("shape mismatch among E (N x C), P (L x C x r), Q (L x r x d), tsq (L)")
+    nbytes = targets_sq_workspace_size(N, C)
+    ws = _workspace(nbytes, E.device, workspace)
+    rc = lib().loca_targets_sq(_ptr(E), N, C, _ptr(P), _ptr(Q), L, r, d, _ptr(tsq), _ptr(ws), nbytes, _stream(stream))
+    _check(rc, "loca_targets_sq")
+
+
+def gram_cross_fused_workspace_size(L, N, r) -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib().loca_gram_cross_fused_workspace_size(L, N, r, ctypes.byref(out)),
+           "loca_gram_cross_fused_workspace_size")
+    return out.value
+
+
+def loca_gram_cross_fused(X, E, P, Q, alpha, gram, cross, zero_first, workspace=None, stream=None):
+    """loca_gram_cross with each block's targets ``T_l = (E P_l) Q_l`` generated inside the kernel."""
+    _dev(X, "X", torch.bfloat16, 3)
+    _dev(E, "E", torch.float32, 2)
+    _dev(P, "P", torch.float32, 3)
+    _dev(Q, "Q", torch.float32, 3)
+    _dev(alpha, "alpha", torch.float32, 1)
+    _dev(gram, "gram", torch.float32, 3)
+    _dev(cross, "cross", torch.float32, 3)
+    L, N, d = X.shape
+    C, r = P.shape[1], P.shape[2]
+    if (tuple(E.shape) != (N, C) or tuple(P.shape) != (L, C, r) or tuple(Q.shape) != (L, r, d)
+            or tuple(gram.shape) != (L, d, d) or tuple(cross.shape) != (L, d, d)):
+        raise ValueError("shape mismatch among X, E, P, Q, gram, cross")
+    nbytes = gram_cross_fused_workspace_size(L, N, r)
+    ws = _workspace(nbytes, X.device, workspace)
+    rc = lib().loca_gram_cross_fused(_ptr(X), LOCA_BF16, L, N, d, _ptr(E), C, _ptr(P), _ptr(Q), r, _ptr(alpha),
+                                     int(bool(zero_first)), _ptr(gram), _ptr(cross), _ptr(ws), nbytes, _stream(stream))
+    _check(rc, "loca_gram_cross_fused")
 
 
 def ridge_solve_workspace_size(L, d, k) -> int:

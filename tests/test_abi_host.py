@@ -128,6 +128,30 @@ def test_validation_codes(L):
     rc2, n2 = _ws(L.loca_kspace_workspace_size, 28, 1024, 3584, 16, 4, 16)
     # W_l (2 x 16 x d bf16 per block) plus partial slots; only the tiny E^T E partials grow with N
     assert rc == 0 and rc2 == 0 and n2 <= n < n2 + (1 << 21) and n >= 28 * 32 * 3584 * 2
+    # fused targets: bf16 X only, r and C limits, misaligned gram, missing E; ||T||^2 limits
+    f = ctypes.c_float
+    assert L.loca_gram_cross_fused(fake, 0, 2, 64, 64, fake, 4, fake, fake, 16, fake, 1, fake, fake, fake,
+                                   1 << 20, None) == 4
+    assert L.loca_gram_cross_fused(fake, 1, 2, 64, 64, fake, 4, fake, fake, 33, fake, 1, fake, fake, fake,
+                                   1 << 20, None) == 2
+    assert L.loca_gram_cross_fused(fake, 1, 2, 64, 64, fake, 65, fake, fake, 16, fake, 1, fake, fake, fake,
+                                   1 << 20, None) == 2
+    assert L.loca_gram_cross_fused(fake, 1, 2, 64, 64, fake, 4, fake, fake, 16, fake, 1, P(260), fake, fake,
+                                   1 << 20, None) == 3
+    assert L.loca_gram_cross_fused(fake, 1, 2, 64, 64, None, 4, fake, fake, 16, fake, 1, fake, fake, fake,
+                                   1 << 20, None) == 1
+    assert L.loca_gram_cross_fused(fake, 1, 2, 64, 64, fake, 4, fake, fake, 16, fake, 1, fake, fake, fake,
+                                   8, None) == 7
+    assert L.loca_targets_sq(fake, 64, 4, fake, fake, 2, 33, 64, fake, fake, 1 << 20, None) == 2
+    assert L.loca_targets_sq(fake, 64, 4, fake, fake, 2, 8, 64, None, fake, 1 << 20, None) == 1
+    assert L.loca_targets_sq(fake, 64, 4, fake, fake, 2, 8, 64, fake, fake, 8, None) == 7
+    rc, n = _ws(L.loca_gram_cross_fused_workspace_size, 28, 131072, 16)
+    assert rc == 0 and n >= 256 + 4 * 28 * 131072 * 16
+    rc, _ = _ws(L.loca_gram_cross_fused_workspace_size, 28, 131072, 33)
+    assert rc == 2
+    rc, n = _ws(L.loca_targets_sq_workspace_size, 131072, 4)
+    assert rc == 0 and n >= 8 * 16 * (131072 // 2048) and n % 256 == 0
+    del f
     # host memory: freeing NULL is a no-op; a pointer the library did not hand out is rejected
     assert L.loca_host_free(None) == 0
     assert L.loca_host_free(fake) == 1

@@ -1,7 +1,8 @@
 """The failure path of the bounded device waits, exercised without faulting or hanging the GPU.
 
 A wait limit of 1 microsecond (the loca_set_wait_limit test hook) makes the first wait of the
-tensor-core kernels (targets, k-space statistics, the CTA-pair Gram / cross kernel) that does not
+tensor-core kernels (targets, k-space statistics, the CTA-pair Gram / cross kernel with and
+without generated targets) that does not
 succeed at once give up: the kernel must record
 LOCA_ERR_TIMEOUT in the device status word, let its copies and MMAs in flight land, free its
 tensor memory and return.  The CUDA context must stay usable: with the default limit restored,
@@ -59,6 +60,15 @@ def _gram_call(lc, X, T):
     return gram, cross
 
 
+def _fused_call(lc, X, E, P, Q):
+    L, N, d = X.shape
+    gram = torch.empty((L, d, d), device="cuda")
+    cross = torch.empty((L, d, d), device="cuda")
+    lc.loca_gram_cross_fused(X, E, P, Q, torch.full((L,), 0.25, device="cuda"), gram, cross, zero_first=True)
+    torch.cuda.synchronize()
+    return gram, cross
+
+
 def test_wait_timeout_is_reported_and_the_context_recovers(lc):
     g = torch.Generator(device="cuda")
     g.manual_seed(5)
@@ -74,23 +84,28 @@ def test_wait_timeout_is_reported_and_the_context_recovers(lc):
     ref_k = _kspace_call(lc, X, A, E, P, Q)
     ref_t = _targets_call(lc, E, P, Q, L, N, d)
     ref_g = _gram_call(lc, X, T)
+    ref_f = _fused_call(lc, X, E, P, Q)
     assert lc.loca_device_status() == 0
-    for call in ("kspace", "targets", "gram"):
+    for call in ("kspace", "targets", "gram", "fused"):
         lc.loca_set_wait_limit(1000)  # 1 us: a wait that does not succeed at once gives up
         if call == "kspace":
             _kspace_call(lc, X, A, E, P, Q)
         elif call == "targets":
             _targets_call(lc, E, P, Q, L, N, d)
-        else:
+        elif call == "gram":
             # the CTA-pair kernel: its roles stop at different points, the odd CTA's half of an
             # armed stage may never be issued, and every copy, MMA and bulk store still lands
             # before either CTA of a pair leaves
             _gram_call(lc, X, T)
+        else:
+            # the same kernel generating its targets: more roles (U producer, T conversion)
+            _fused_call(lc, X, E, P, Q)
         assert lc.loca_device_status() == LOCA_ERR_TIMEOUT, call
         lc.loca_set_wait_limit(0)
         again_k = _kspace_call(lc, X, A, E, P, Q)
         again_t = _targets_call(lc, E, P, Q, L, N, d)
         again_g = _gram_call(lc, X, T)
+        again_f = _fused_call(lc, X, E, P, Q)
         assert lc.loca_device_status() == 0, call
-        for a, b in zip(ref_k + ref_t + ref_g, again_k + again_t + again_g):
+        for a, b in zip(ref_k + ref_t + ref_g + ref_f, again_k + again_t + again_g + again_f):
             assert torch.equal(a, b), call
