@@ -2,11 +2,11 @@
 all-linear network check on the GPU path: head error -> calibration -> targets reproduce the
 true backpropagated hidden-state gradients.
 
-Tolerance: the products E^T E and E^T G are formed from fp32 products summed in fp32 over
-32-token chunks and in fp64 across chunks (relative error ~1e-7); the solve and the Jacobi
-eigen-decomposition run in fp64.  The rank-r map P Q is then within 1e-4 relative Frobenius
-when the retained singular values are separated from the rest (planted rank r, gap >> noise),
-and individual factors match under the same sign convention.
+Tolerance: 1e-5 relative Frobenius on P Q and on each factor (the bound the statement of the
+problem sets for fp32 inputs).  ``pq_bound`` derives the worst-case envelope from the arithmetic
+(fp32 chunk sums of E^T E and E^T G, the conditioning of E^T E + beta I and the gap below the
+retained singular values: 3.6e-5 to 4e-4 for these cases); the rounding errors are random in
+sign, and the measured errors (3.5e-8 to 5.7e-8) are printed beside it.
 """
 
 import math
@@ -41,6 +41,25 @@ def _dev(a, dtype=torch.float32):
     return torch.from_numpy(np.ascontiguousarray(a)).to(device="cuda", dtype=dtype)
 
 
+def pq_bound(E, beta, F_hat, r):
+    """First-order bound on the GPU fit's relative error in the rank-r map P Q.
+
+    The inputs are exact fp32 values.  The only inexact steps before the fp64 solve are the sums
+    K = E^T E and R_l = E^T G_l: fp32 products summed in fp32 over 32-token chunks (relative error
+    at most u = 32 * 2^-24 per entry), chunks summed in fp64.  The solve F^T = (K + beta I)^-1 R
+    multiplies a relative perturbation of K and R by at most 2 kappa(K + beta I).  The rank-r
+    truncation moves by at most (1 + 2 sigma_1 / (sigma_r - sigma_{r+1})) times the perturbation
+    of F (Wedin's bound for the singular subspaces, plus the values themselves).  The eigen-
+    decomposition and the rest run in fp64, far below this."""
+    E = np.asarray(E, dtype=np.float64)
+    K = E.T @ E + beta * np.eye(E.shape[1])
+    kappa = float(np.linalg.cond(K))
+    s = np.linalg.svd(F_hat, compute_uv=False)
+    s_next = s[r] if r < s.size else 0.0
+    gap = max(s[r - 1] - s_next, 1e-300)
+    return 2.0 * kappa * (32 * 2.0 ** -24) * (1.0 + 2.0 * s[0] / gap)
+
+
 def _fit(lc, E, G, beta, r):
     L, Np, d = G.shape
     m = E.shape[1]
@@ -65,11 +84,18 @@ def test_calib_parity(lc, Np, m, d, L, rank, r):
     G = pp["G_probe"]
     beta = 1e-3 * float(np.trace(E.astype(np.float64).T @ E)) / m
     P, Q, sig = _fit(lc, E, G, beta, r)
-    Pr, Qr, sr, _ = O.calib_fit(E, G, beta, r)
+    Pr, Qr, sr, Fh = O.calib_fit(E, G, beta, r)
     for l in range(L):
-        assert _rel(P[l] @ Q[l], Pr[l] @ Qr[l]) < 1e-4, l
+        err = _rel(P[l] @ Q[l], Pr[l] @ Qr[l])
+        bound = pq_bound(E, beta, Fh[l], r)
+        print(f"block {l}: P Q rel err {err:.2e}, worst-case bound of the arithmetic {bound:.2e}")
+        # the fp32-input tolerance (1e-5), inside the worst-case envelope: the rounding errors of the
+        # chunk sums are random in sign, so the measured error sits near 4e-8
+        assert err <= min(1e-5, bound), l
         assert _rel(sig[l], sr[l]) < 1e-5
-        assert _rel(Q[l], Qr[l]) < 1e-4 and _rel(P[l], Pr[l]) < 1e-4
+        # the factors under the sign convention
+        print(f"block {l}: factor rel err Q {_rel(Q[l], Qr[l]):.2e} P {_rel(P[l], Pr[l]):.2e}")
+        assert _rel(Q[l], Qr[l]) <= 1e-5 and _rel(P[l], Pr[l]) <= 1e-5
         assert np.allclose(Q[l] @ Q[l].T, np.eye(r), atol=1e-5)
 
 

@@ -5,9 +5,11 @@ against the exact truncated SVD (calib_fit) where the spectrum has a gap.
 Tolerance: as for loca_calib_fit, the products with E and G_l come from fp32 products summed
 in fp32 over 128-term runs and in fp64 across runs (relative error ~1e-7, times the condition
 number of E^T E + beta I in the solves); the factorisation, solves, bases and the
-Rayleigh-Ritz step run in fp64.  The rank-r map P Q is within 1e-4 relative Frobenius when
-the retained singular values are separated from the rest (planted rank r); singular values
-are Weyl-stable (no gap needed) and match to 1e-5 of sigma_1.
+Rayleigh-Ritz step run in fp64.  The rank-r map P Q and each factor are within 1e-5 relative
+Frobenius (the fp32-input tolerance; measured 1.3e-7 to 6.2e-7) when the retained singular
+values are separated from the rest (planted rank r); the worst-case envelope of the arithmetic
+(``pq_bound``) is printed beside each error.  Singular values are Weyl-stable (no gap needed)
+and match to 1e-5 of sigma_1.
 """
 
 import numpy as np
@@ -15,6 +17,7 @@ import pytest
 import torch
 
 from oracle import loca_oracle as O
+from test_calib_gpu import pq_bound
 from synth import inputs as S
 
 pytestmark = pytest.mark.gpu
@@ -76,10 +79,17 @@ def test_rsvd_parity(lc, Np, m, d, L, rank, r, ell, q, esc):
     beta = _beta(E)
     P, Q, sig = _fit(lc, _dev(E), _dev(G), beta, r, _dev(Om), q)
     Pr, Qr, sr = O.calib_fit_rsvd(E, G, beta, r, Om, q)
+    _, _, _, Fh = O.calib_fit(E, G, beta, r)
     for l in range(L):
-        assert _rel(P[l] @ Q[l], Pr[l] @ Qr[l]) < 1e-4, l
+        err = _rel(P[l] @ Q[l], Pr[l] @ Qr[l])
+        print(f"block {l}: P Q rel err {err:.2e} (worst-case bound of the exact fit's arithmetic "
+              f"{pq_bound(E, beta, Fh[l], r):.2e})")
+        # the fp32-input tolerance: measured 1.3e-7 to 6.2e-7 (fp32 power iterations and GEMM
+        # operands, fp64 for the last solve and the Rayleigh-Ritz step)
+        assert err < 1e-5, l
         assert np.max(np.abs(sig[l] - sr[l])) < 1e-5 * sr[l, 0], (sig[l], sr[l])
-        assert _rel(Q[l], Qr[l]) < 1e-4 and _rel(P[l], Pr[l]) < 1e-4, l
+        print(f"block {l}: factor rel err Q {_rel(Q[l], Qr[l]):.2e} P {_rel(P[l], Pr[l]):.2e}")
+        assert _rel(Q[l], Qr[l]) < 1e-5 and _rel(P[l], Pr[l]) < 1e-5, l
         assert np.allclose(Q[l] @ Q[l].T, np.eye(r), atol=1e-5)
     if q >= 1:
         # gapped spectrum: the randomized fit is the exact truncated SVD to rounding
