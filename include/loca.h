@@ -59,8 +59,10 @@ typedef enum loca_status {
   LOCA_ERR_TIMEOUT = 6,            /* a device wait gave up (reported by loca_device_status) */
   LOCA_ERR_WORKSPACE = 7,          /* workspace missing or smaller than required */
   LOCA_ERR_UNSUPPORTED = 8,        /* valid request outside what this library supports */
-  LOCA_ERR_NUMERIC = 9             /* device: a system that should be positive definite was not
+  LOCA_ERR_NUMERIC = 9,            /* device: a system that should be positive definite was not
                                       in floating point (reported by loca_device_status) */
+  LOCA_ERR_BOUNDS = 10             /* device, debug build only: an index left its buffer; the
+                                      access was skipped (reported by loca_device_status) */
 } loca_status;
 
 /* Element type codes. */
@@ -92,6 +94,17 @@ const char* loca_last_error_string(void);
  * then undefined.  Synchronises `stream`.  *host_status receives LOCA_OK or the code.
  */
 int loca_device_status(int32_t* host_status /* host */, void* stream);
+
+/*
+ * Debug build (libloca_debug.so, compiled with -DLOCA_DEBUG; same entry points).  Every kernel
+ * checks the index of each global access it computes, and the coordinates of its TMA stores,
+ * against the extent of the buffer that the sizes of the call give.  A failed check skips the
+ * access and records LOCA_ERR_BOUNDS with the source line; nothing traps.  loca_device_status
+ * then returns LOCA_ERR_BOUNDS (after any code of the status word above) and names the source
+ * file and line in loca_last_error_string().  The release library compiles the checks away.
+ * loca_debug_build returns 1 in the debug build and 0 in the release build.
+ */
+int loca_debug_build(void);
 
 /*
  * loca_error — top-layer error at the frozen head (Eq. 4; Lemma "Top-layer error", S3).

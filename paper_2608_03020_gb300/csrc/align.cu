@@ -64,7 +64,7 @@ __global__ void __launch_bounds__(AL_THREADS) k_align_u(const float* __restrict_
 #pragma unroll
   for (int i = 0; i < SPT; ++i) {
     const int s = sg + SG * i;
-    if (s < r) U[(int64_t(l) * Np + n) * r + s] = acc[i];
+    if (s < r && LOCA_CHECK((int64_t(l) * Np + n) * r + s, int64_t(gridDim.y) * Np * r)) U[(int64_t(l) * Np + n) * r + s] = acc[i];
   }
 }
 
@@ -110,7 +110,7 @@ __global__ void __launch_bounds__(AL_THREADS) k_align_part(const float* __restri
       float tv = 0.f;
 #pragma unroll
       for (int s = 0; s < RP; ++s) tv = fmaf(Us[t][s], Qs[s][tid], tv);
-      const float g = jv ? Gl[(s0 + t) * d + j] : 0.f;
+      const float g = (jv && LOCA_CHECK((s0 + t) * d + j, Np * d)) ? Gl[(s0 + t) * d + j] : 0.f;
       gt = fmaf(g, tv, gt);
       gg = fmaf(g, g, gg);
       tt = fmaf(tv, tv, tt);
@@ -127,7 +127,8 @@ __global__ void __launch_bounds__(AL_THREADS) k_align_part(const float* __restri
   if (tid < 3) {
     double a = 0.0;
     for (int w = 0; w < AL_THREADS / 32; ++w) a += red[tid][w];
-    part[((int64_t(l) * ntile + tile) * nch + ch) * 3 + tid] = a;
+    if (LOCA_CHECK(((int64_t(l) * ntile + tile) * nch + ch) * 3 + tid, int64_t(gridDim.z) * ntile * nch * 3))
+      part[((int64_t(l) * ntile + tile) * nch + ch) * 3 + tid] = a;
   }
 }
 
@@ -141,7 +142,7 @@ __global__ void k_align_final(const double* __restrict__ part, int nparts, doubl
     gg += p[1];
     tt += p[2];
   }
-  alpha[l] = (gg > 0.0 && tt > 0.0) ? gt / sqrt(gg * tt) : 0.0;
+  if (LOCA_CHECK(l, gridDim.x)) alpha[l] = (gg > 0.0 && tt > 0.0) ? gt / sqrt(gg * tt) : 0.0;
 }
 
 }  // namespace

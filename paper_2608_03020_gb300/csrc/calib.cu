@@ -46,7 +46,7 @@ __global__ void __launch_bounds__(256) k_calib_xty(const float* __restrict__ E, 
     for (int e = threadIdx.x; e < XT_TOK * XT_COLS; e += 256) {
       const int nn = e / XT_COLS, c = e % XT_COLS;
       const int64_t jc = int64_t(blockIdx.x) * XT_COLS + c;
-      Ys[nn][c] = (n0 + nn < Np && jc < w) ? Yb[(n0 + nn) * w + jc] : 0.f;
+      Ys[nn][c] = (n0 + nn < Np && jc < w && LOCA_CHECK((n0 + nn) * w + jc, Np * w)) ? Yb[(n0 + nn) * w + jc] : 0.f;
     }
     __syncthreads();
     float part[SPT];
@@ -65,7 +65,7 @@ __global__ void __launch_bounds__(256) k_calib_xty(const float* __restrict__ E, 
 #pragma unroll
   for (int i = 0; i < SPT; ++i) {
     const int s = grp + 4 * i;
-    if (s < m) out[(int64_t(b) * m + s) * w + j] = acc[i];
+    if (s < m && LOCA_CHECK((int64_t(b) * m + s) * w + j, int64_t(gridDim.y) * m * w)) out[(int64_t(b) * m + s) * w + j] = acc[i];
   }
 }
 
@@ -130,6 +130,7 @@ __global__ void __launch_bounds__(256) k_calib_solve(const double* __restrict__ 
   __syncthreads();
   if (s_bad) {
     if (t == 0) atomicExch(status, int32_t(LOCA_ERR_NUMERIC));
+    if (!LOCA_CHECK_SPAN(int64_t(l) * r * d, int64_t(r) * d, int64_t(gridDim.x) * r * d)) return;
     for (int64_t e = t; e < int64_t(r) * d; e += 256) Q[int64_t(l) * r * d + e] = 0.f;
     for (int e = t; e < m * r; e += 256) P[int64_t(l) * m * r + e] = 0.f;
     if (sigma != nullptr)
@@ -189,6 +190,7 @@ __global__ void __launch_bounds__(256) k_calib_solve(const double* __restrict__ 
     double sg = lam > 0.0 ? sqrt(lam) : 0.0;
     if (!(sg > 1e-12 * s1)) sg = 0.0;
     float* qrow = Q + (int64_t(l) * r + i) * d;
+    if (!LOCA_CHECK_SPAN((int64_t(l) * r + i) * d, d, int64_t(gridDim.x) * r * d)) break;
     // Q row = U_i^T F^T / sigma_i ; track the entry of largest magnitude (lowest index on ties)
     double best = -1.0;
     int64_t bj = 0;
@@ -224,7 +226,8 @@ __global__ void __launch_bounds__(256) k_calib_solve(const double* __restrict__ 
     __syncthreads();
     if (sign < 0.f)
       for (int64_t j = t; j < d; j += 256) qrow[j] = -qrow[j];
-    for (int a = t; a < m; a += 256) P[(int64_t(l) * m + a) * r + i] = float(sign * sm.V[a][col] * sg);
+    for (int a = t; a < m; a += 256)
+      if (LOCA_CHECK((int64_t(l) * m + a) * r + i, int64_t(gridDim.x) * m * r)) P[(int64_t(l) * m + a) * r + i] = float(sign * sm.V[a][col] * sg);
     if (sigma != nullptr && t == 0) sigma[int64_t(l) * r + i] = float(sg);
     __syncthreads();
   }

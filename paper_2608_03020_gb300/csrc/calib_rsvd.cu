@@ -154,7 +154,8 @@ __global__ void __launch_bounds__(256) k_cr_gemm(const float* __restrict__ A, in
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const int64_t gi = i0 + ty * 4 + p, gj = j0 + tx * 4 + q;
-      if (gi < M && gj < N) C[gi * ldc + gj] = TC(acc[p][q] + double(run_sum[p][q]));
+      if (gi < M && gj < N && LOCA_CHECK(gi * ldc + gj, (M - 1) * ldc + N))
+        C[gi * ldc + gj] = TC(acc[p][q] + double(run_sum[p][q]));
     }
 }
 
@@ -498,7 +499,7 @@ __global__ void __launch_bounds__(QR_CHUNK) k_cr_qr_apply(double* __restrict__ V
   for (int e = tid; e < ELLP * ELLP; e += QR_CHUNK) F[e / ELLP][e % ELLP] = fac[int64_t(l) * ELLP * ELLP + e];
   __syncthreads();
   const int64_t rrow = int64_t(blockIdx.x) * QR_CHUNK + tid;
-  if (rrow >= rows) return;
+  if (rrow >= rows || !LOCA_CHECK_SPAN(rrow * n + int64_t(l) * ell, ell, rows * n)) return;
   double* v = V + rrow * n + int64_t(l) * ell;
   double x[ELLP];
 #pragma unroll
@@ -609,7 +610,8 @@ __global__ void __launch_bounds__(RZ_CH) k_cr_ritz_out(const double* __restrict_
     for (int i = 0; i < r; ++i) {
       double s = 0.0;
       for (int c = 0; c < ell; ++c) s = fma(row[c], Us[c * r + i], s);
-      P[(int64_t(l) * m + a) * r + i] = (ss[i] > 0.0) ? float(ss[i] * s) : 0.f;
+      if (LOCA_CHECK((int64_t(l) * m + a) * r + i, int64_t(gridDim.y) * m * r))
+        P[(int64_t(l) * m + a) * r + i] = (ss[i] > 0.0) ? float(ss[i] * s) : 0.f;
     }
   }
   const int64_t j = int64_t(ch) * RZ_CH + tid;
@@ -620,7 +622,8 @@ __global__ void __launch_bounds__(RZ_CH) k_cr_ritz_out(const double* __restrict_
       for (int c = 0; c < ell; ++c) v = fma(brow[c], Us[c * r + i], v);
       v /= ss[i];
     }
-    if (j < d) Q[(int64_t(l) * r + i) * d + j] = float(v);
+    if (j < d && LOCA_CHECK((int64_t(l) * r + i) * d + j, int64_t(gridDim.y) * r * d))
+      Q[(int64_t(l) * r + i) * d + j] = float(v);
     double best = (j < d && v == v) ? fabs(v) : -1.0;  // NaN entries never win
     int64_t bj = j;
 #pragma unroll
@@ -637,7 +640,7 @@ __global__ void __launch_bounds__(RZ_CH) k_cr_ritz_out(const double* __restrict_
       bi[wid] = bj;
     }
     __syncthreads();
-    if (tid == 0) {
+    if (tid == 0 && LOCA_CHECK((int64_t(l) * r + i) * nch + ch, int64_t(gridDim.y) * r * nch)) {
       double b0 = bv[0];
       int64_t i0 = bi[0];
       for (int w = 1; w < RZ_CH / 32; ++w)
@@ -672,7 +675,7 @@ __global__ void __launch_bounds__(256) k_cr_ritz_sign(float* __restrict__ P, flo
     s_flip = (j0 >= 0 && j0 < d && Q[(int64_t(l) * r + i) * d + j0] < 0.f) ? 1 : 0;
   }
   __syncthreads();
-  if (!s_flip) return;
+  if (!s_flip || !LOCA_CHECK_SPAN((int64_t(l) * r + i) * d, d, int64_t(gridDim.x) * r * d)) return;
   for (int64_t j = threadIdx.x; j < d; j += blockDim.x) Q[(int64_t(l) * r + i) * d + j] *= -1.f;
   for (int64_t a = threadIdx.x; a < m; a += blockDim.x) P[(int64_t(l) * m + a) * r + i] *= -1.f;
 }

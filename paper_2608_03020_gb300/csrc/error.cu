@@ -99,6 +99,7 @@ __global__ void __launch_bounds__(256) k_head_error(const Tz* __restrict__ z, in
   const int64_t nwarps = (int64_t(gridDim.x) * blockDim.x) >> 5;
   for (int64_t n = warp0; n < N; n += nwarps) {
     const Tz* row = z + n * ldz;
+    if (!LOCA_CHECK_SPAN(n * ldz, V, (N - 1) * ldz + V)) continue;
     RunMax a0, a1;
     if (normaliser == 0) {
       int64_t j0 = 0;
@@ -122,7 +123,10 @@ __global__ void __launch_bounds__(256) k_head_error(const Tz* __restrict__ z, in
       }
       for (int64_t j = j0 + lane; j < V; j += 32) a1.add(to_f(row[j]));
     } else {
-      for (int c = lane; c < C; c += 32) a0.add(to_f(row[cols[c]]));
+      for (int c = lane; c < C; c += 32) {
+        const int32_t col = cols[c];
+        if (LOCA_CHECK(col, V)) a0.add(to_f(row[col]));
+      }
     }
     merge(a0, a1.m, a1.s);
 #pragma unroll
@@ -135,10 +139,18 @@ __global__ void __launch_bounds__(256) k_head_error(const Tz* __restrict__ z, in
     const int yn = y[n];
     const float wn = (yn < 0) ? 0.f : (w ? w[n] : 1.f);
     for (int c = lane; c < C; c += 32) {
-      const float zc = to_f(row[cols[c]]);
-      E[n * C + c] = wn * (expf(zc - lse) - (c == yn ? 1.f : 0.f));
+      const int32_t col = cols[c];
+      const float zc = LOCA_CHECK(col, V) ? to_f(row[col]) : 0.f;
+      if (LOCA_CHECK(n * C + c, N * C)) E[n * C + c] = wn * (expf(zc - lse) - (c == yn ? 1.f : 0.f));
     }
-    if (ce != nullptr && lane == 0) ce[n] = (yn < 0) ? 0.f : wn * (lse - to_f(row[cols[yn]]));
+    if (ce != nullptr && lane == 0 && LOCA_CHECK(n, N)) {
+      float cn = 0.f;
+      if (yn >= 0 && LOCA_CHECK(yn, C)) {
+        const int32_t cy = cols[yn];
+        if (LOCA_CHECK(cy, V)) cn = wn * (lse - to_f(row[cy]));
+      }
+      ce[n] = cn;
+    }
   }
 }
 

@@ -211,6 +211,8 @@ __global__ void __launch_bounds__(256) k_fused_u(const float* __restrict__ E, in
   const int l = blockIdx.y;
   const int64_t n = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
   if (n >= N) return;
+  if (!LOCA_CHECK_SPAN(n * C, C, N * C) || !LOCA_CHECK_SPAN((int64_t(l) * N + n) * rp, rp, int64_t(gridDim.y) * N * rp))
+    return;
   const float* Pl = P + int64_t(l) * C * r;
   float u[32];
 #pragma unroll
@@ -438,6 +440,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Cfg<kFused>::kThread
           const uint32_t bdst = st + 2u * A_BYTES;
           const int tok = kb * BK;
           const int col0 = w.nt * BN + int(rank) * BNC;
+          // the stage is armed: a failed check is recorded, the loads (out-of-range boxes are
+          // filled by the TMA unit) still run so that the barrier completes
+          (void)LOCA_REQUIRE(tok >= 0 && col0 % 64 == 0);
           if (blocked) {
             if (!gen)
               for (int s = 0; s < w.nslots; ++s)
@@ -450,6 +455,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Cfg<kFused>::kThread
                 const CUtensorMap* map = w.kind[s] == 0 ? &tmX : &tmT;
                 const uint32_t dst = st + uint32_t(s) * A_BYTES;
                 const int row0 = w.mt[s] * BMP + int(rank) * BMC;
+                (void)LOCA_REQUIRE(row0 % 64 == 0);
                 tma_load_3d_pair(dst, map, fb, row0, tok, w.l);
                 tma_load_3d_pair(dst + SUB_BYTES, map, fb, row0 + 64, tok, w.l);
               }
@@ -654,10 +660,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Cfg<kFused>::kThread
           const int cl = lane + 32 * i;  // channel of this CTA's 128
           const int c = w.mt[0] * BMP + int(rank) * BMC + cl;
           for (int sidx = 0; sidx < rp; ++sidx) {
-            const float q = (sidx < r && c < g.d) ? __ldg(Ql + int64_t(sidx) * g.d + c) : 0.f;
+            const float q = (sidx < r && c < g.d && LOCA_CHECK(int64_t(w.l) * r * g.d + int64_t(sidx) * g.d + c,
+                                                               int64_t(g.L) * r * g.d))
+                                ? __ldg(Ql + int64_t(sidx) * g.d + c)
+                                : 0.f;
             __nv_bfloat16 h, lo;
             split_bf16(q, h, lo);
             const uint32_t off = kmaj16_off(cl, sidx, rp) >> 1;
+            if (!LOCA_CHECK(off, 4096)) continue;
             qh[off] = h;
             ql[off] = lo;
           }
@@ -682,7 +692,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Cfg<kFused>::kThread
         const int64_t n = int64_t(kb) * BK + int64_t(rank) * U_ROWS + lane;
 #pragma unroll
         for (int qq = 0; qq < 4; ++qq) {
-          const bool in = qq < nq && n < g.N;
+          const bool in = qq < nq && n < g.N && LOCA_CHECK(n * nq + qq, g.N * nq);
           h[qq] = in ? __ldg(Uh + n * nq + qq) : make_uint4(0, 0, 0, 0);
           lo[qq] = in ? __ldg(Ul + n * nq + qq) : make_uint4(0, 0, 0, 0);
         }
@@ -806,8 +816,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Cfg<kFused>::kThread
             __syncwarp();
             if (lane == 0) {
               const uint32_t src = box0_s + buf * EPI_BOX_BYTES;
-              if (store) tma_store_3d(omap, src, j0, i0, w.l);
-              else tma_reduce_add_3d(omap, src, j0, i0, w.l);
+              if (LOCA_REQUIRE(i0 >= 0 && j0 >= 0 && j0 % 4 == 0)) {
+                if (store) tma_store_3d(omap, src, j0, i0, w.l);
+                else tma_reduce_add_3d(omap, src, j0, i0, w.l);
+              }
               bulk_commit_group();
             }
             ++nbox;
@@ -868,12 +880,12 @@ __global__ void __launch_bounds__(256) k_gram_mirror(float* __restrict__ gram, i
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
   for (int r = ty; r < 32; r += 8) {  // source rows j of the upper tile (bj, bi)
     const int i = bj * 32 + r, j = bi * 32 + tx;
-    if (i < d && j < d) tile[r][tx] = G[int64_t(i) * d + j];
+    if (i < d && j < d && LOCA_CHECK(int64_t(i) * d + j, int64_t(d) * d)) tile[r][tx] = G[int64_t(i) * d + j];
   }
   __syncthreads();
   for (int r = ty; r < 32; r += 8) {
     const int i = bi * 32 + r, j = bj * 32 + tx;
-    if (i < d && j < d && i > j) G[int64_t(i) * d + j] = tile[tx][r];
+    if (i < d && j < d && i > j && LOCA_CHECK(int64_t(i) * d + j, int64_t(d) * d)) G[int64_t(i) * d + j] = tile[tx][r];
   }
 }
 

@@ -61,9 +61,10 @@ __global__ void __launch_bounds__(PREP_THREADS) k_kspace_prep(const float* __res
   for (int64_t e = int64_t(part) * PREP_THREADS + threadIdx.x; e < tot; e += int64_t(PREP_SPLIT) * PREP_THREADS) {
     const int s = int(e / d);
     const int64_t j = e - int64_t(s) * d;
-    const float a = (s < k) ? Al[j * k + s] : 0.f;
+    const float a = (s < k && LOCA_CHECK(j * k + s, d * k)) ? Al[j * k + s] : 0.f;
     const __nv_bfloat16 hi = __float2bfloat16_rn(a);
     const __nv_bfloat16 lo = __float2bfloat16_rn(a - __bfloat162float(hi));
+    if (!LOCA_CHECK(int64_t(kp + s) * d + j, int64_t(2) * kp * d)) continue;
     Wl[int64_t(s) * d + j] = hi;
     Wl[int64_t(kp + s) * d + j] = lo;
   }
@@ -77,7 +78,8 @@ __global__ void __launch_bounds__(PREP_THREADS) k_kspace_prep(const float* __res
     double v = double(acc);
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-    if (lane == 0) M[(int64_t(l) * r + a) * r + b] = float(v);
+    if (lane == 0 && LOCA_CHECK((int64_t(l) * r + a) * r + b, int64_t(gridDim.x) * r * r))
+      M[(int64_t(l) * r + a) * r + b] = float(v);
   }
 }
 
@@ -173,6 +175,7 @@ __global__ void __launch_bounds__(xa_threads(KP), 1)
           pending |= 1u << stage;
           pending_par = (pending_par & ~(1u << stage)) | (phase << stage);
           const uint32_t st = sbase + uint32_t(stage) * XA_STAGE;
+          (void)LOCA_REQUIRE((kc * XA_BK) % 8 == 0 && t0 >= 0);
           tma_load_3d(st, &tmX, fb, kc * XA_BK, t0, l);
           tma_load_3d(st + XA_XBYTES, &tmW, fb, kc * XA_BK, 0, l);
           if (++stage == XA_STAGES) { stage = 0; phase ^= 1u; }
@@ -233,7 +236,8 @@ __global__ void __launch_bounds__(xa_threads(KP), 1)
       double a = xs;
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) a += __shfl_xor_sync(0xffffffffu, a, off);
-      if (lane == 0) part[(int64_t(lf) * PS + xe) * nslot + int64_t(blockIdx.x) * 4 + w2] = a;
+      if (lane == 0 && LOCA_CHECK((int64_t(lf) * PS + xe) * nslot + int64_t(blockIdx.x) * 4 + w2, int64_t(L) * PS * nslot))
+        part[(int64_t(lf) * PS + xe) * nslot + int64_t(blockIdx.x) * 4 + w2] = a;
     };
     int stage = 0;
     uint32_t phase = 0;
@@ -335,6 +339,8 @@ __global__ void __launch_bounds__(xa_threads(KP), 1)
     auto flush = [&](int lf) {
       // entry-major: entry e of block lf at part[(lf * PS + e) * nslot + this slot]
       double* slot = part + int64_t(lf) * PS * nslot + int64_t(blockIdx.x) * 4 + q;
+      // every entry index below is < PS - 1 (the last one is the ||x||^2 entry of the other warps)
+      if (!LOCA_CHECK(lf, L) || !LOCA_REQUIRE(NTRI + NS + 1 == PS)) return;
       if constexpr (kBlk) {
 #pragma unroll
         for (int i2 = 0; i2 < NG; ++i2) {
@@ -396,7 +402,7 @@ __global__ void __launch_bounds__(xa_threads(KP), 1)
         }
 #pragma unroll
         for (int c = 0; c < kMaxCk; ++c)
-          if (c < C) es[c * TST + lane] = nv ? E[n * C + c] : 0.f;
+          if (c < C) es[c * TST + lane] = (nv && LOCA_CHECK(n * C + c, N * C)) ? E[n * C + c] : 0.f;
       } else {
         float v[NCOL];
         if constexpr (NCOL == 32) {
@@ -413,7 +419,7 @@ __global__ void __launch_bounds__(xa_threads(KP), 1)
         for (int s2 = 0; s2 < KP; ++s2) ps[lane * PSTR + s2] = v[s2] + v[KP + s2];
 #pragma unroll
         for (int c = 0; c < kMaxCk; ++c)
-          if (c < C) es[lane * ESTR + c] = nv ? E[n * C + c] : 0.f;
+          if (c < C) es[lane * ESTR + c] = (nv && LOCA_CHECK(n * C + c, N * C)) ? E[n * C + c] : 0.f;
       }
       __syncwarp();
       // the tile's sums over this warp's 32 tokens, for the entries this lane owns
@@ -523,7 +529,7 @@ __global__ void __launch_bounds__(ETE_THREADS) k_kspace_ete(const float* __restr
     __syncthreads();
     for (int e = tid; e < ETE_SUB * C; e += ETE_THREADS) {
       const int t = e / C, c = e % C;
-      es[t][c] = (s0 + t < n1) ? E[(s0 + t) * C + c] : 0.f;
+      es[t][c] = (s0 + t < n1 && LOCA_CHECK((s0 + t) * C + c, N * C)) ? E[(s0 + t) * C + c] : 0.f;
     }
     __syncthreads();
     if (a < C && b < C) {
@@ -533,7 +539,8 @@ __global__ void __launch_bounds__(ETE_THREADS) k_kspace_ete(const float* __restr
       acc += double(part);
     }
   }
-  if (a < C && b < C) ete_part[int64_t(ch) * kMaxCk * kMaxCk + a * kMaxCk + b] = acc;
+  if (a < C && b < C && LOCA_CHECK(int64_t(ch) * kMaxCk * kMaxCk + a * kMaxCk + b, int64_t(gridDim.x) * kMaxCk * kMaxCk))
+    ete_part[int64_t(ch) * kMaxCk * kMaxCk + a * kMaxCk + b] = acc;
 }
 
 // ------------------------------------------------------------------ per-block final reduction
@@ -617,7 +624,7 @@ __global__ void __launch_bounds__(FI_THREADS) k_kspace_final(const double* __res
         b = tmp;
       }
       const double v = sum_entry(a * kp - a * (a - 1) / 2 + (b - a), 4);  // row a of the upper triangle
-      if (lane == 0) {
+      if (lane == 0 && LOCA_CHECK(int64_t(l) * k * k + e, int64_t(gridDim.x) * k * k)) {
         float* o = G + int64_t(l) * k * k + e;
         *o = zero_first ? float(v) : float(double(*o) + v);
       }
@@ -625,13 +632,13 @@ __global__ void __launch_bounds__(FI_THREADS) k_kspace_final(const double* __res
       const int e2 = e - k * k;
       const int cc = e2 / k, s2 = e2 % k;
       const double v = sum_entry(nt + cc * kp + s2, 4);
-      if (lane == 0) {
+      if (lane == 0 && LOCA_CHECK(int64_t(l) * C * k + e2, int64_t(gridDim.x) * C * k)) {
         float* o = SC + int64_t(l) * C * k + e2;
         *o = zero_first ? float(al * v) : float(double(*o) + al * v);
       }
     }
   }
-  if (prt == 0 && tid == 0) {
+  if (prt == 0 && tid == 0 && LOCA_CHECK(l, gridDim.x)) {
     xsq_total[l] = zero_first ? xsq_b : xsq_total[l] + xsq_b;
     if (alpha_out) alpha_out[l] = float(al);
   }
@@ -681,11 +688,14 @@ __global__ void __launch_bounds__(KS_THREADS) k_kspace_solve(
   }
   __syncthreads();
   const int inf = chol_factor<KM>(Md, Lf, Linv, &s_info);
-  if (threadIdx.x == 0) info[int64_t(j) * L + l] = inf;
+  if (threadIdx.x == 0 && LOCA_CHECK(int64_t(j) * L + l, int64_t(gridDim.x) * L)) info[int64_t(j) * L + l] = inf;
   float* Bj = B + (int64_t(j) * L + l) * d * k;
   const float* Bp = B_prev ? B_prev + int64_t(l) * d * k : nullptr;
   const float* Ql = Q + int64_t(l) * r * d;
   for (int64_t i = threadIdx.x; i < d; i += KS_THREADS) {
+    if (!LOCA_CHECK_SPAN((int64_t(j) * L + l) * d * k + i * k, k, int64_t(gridDim.x) * L * d * k) ||
+        !LOCA_CHECK_SPAN((int64_t(l) * d + i) * k, k, int64_t(L) * d * k))
+      break;
     float c[KM];
 #pragma unroll
     for (int s = 0; s < KM; ++s) c[s] = 0.f;

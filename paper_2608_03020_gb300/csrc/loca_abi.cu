@@ -7,6 +7,7 @@
 #include <cstring>
 #include <atomic>
 #include <mutex>
+#include <vector>
 
 #include "loca_internal.h"
 
@@ -77,6 +78,28 @@ std::atomic<unsigned long long> g_wait_limit_ns{0};
 unsigned long long wait_limit_ns() {
   const unsigned long long v = g_wait_limit_ns.load(std::memory_order_relaxed);
   return v == 0 ? 4000000000ull : v;
+}
+
+namespace {
+struct DebugWord {
+  DebugWordReader read;
+  const char* file;
+};
+struct DebugWords {
+  std::mutex mu;
+  std::vector<DebugWord> list;  // filled by static initialisers, before any entry point runs
+};
+DebugWords& debug_words() {
+  static DebugWords w;
+  return w;
+}
+}  // namespace
+
+bool register_debug_word(DebugWordReader reader, const char* file) {
+  DebugWords& w = debug_words();
+  std::lock_guard<std::mutex> lock(w.mu);
+  w.list.push_back(DebugWord{reader, file});
+  return true;
 }
 
 int32_t* device_status_word() {
@@ -204,7 +227,25 @@ int loca_device_status(int32_t* host_status, void* stream) {
   if (e == cudaSuccess) e = cudaMemsetAsync(w, 0, sizeof(int32_t), s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(e, "loca_device_status");
+  // debug build: the first failed bounds check of each translation unit (all words are cleared)
+  for (const DebugWord& dw : debug_words().list) {
+    int32_t code = 0, line = 0;
+    e = dw.read(&code, &line);
+    if (e != cudaSuccess) return cuda_fail(e, "loca_device_status (debug word)");
+    if (code != 0 && *host_status == LOCA_OK) {
+      *host_status = code;
+      set_error_message(code, "device: index outside its buffer at %s:%d", dw.file, int(line));
+    }
+  }
   return LOCA_OK;
+}
+
+int loca_debug_build(void) {
+#ifdef LOCA_DEBUG
+  return 1;
+#else
+  return 0;
+#endif
 }
 
 int loca_error(const void* logits, int logit_dtype, int64_t N, int64_t V, int64_t ldz,

@@ -7,6 +7,7 @@
 #include <stdint.h>
 
 #include "../../include/loca.h"
+#include "debug_check.cuh"
 
 namespace loca {
 

@@ -65,7 +65,9 @@ __global__ void __launch_bounds__(PR_THREADS, KM <= 16 ? 3 : 1) k_project_rows(c
     for (int it = 0; it < PR_ALOADS; ++it) {
       const int e = tid + it * PR_THREADS;
       const int jj = e / KM, s = e % KM;
-      apre[it] = (e < PR_JC * KM && jj < jn && s < k) ? __ldg(Al + (j0 + jj) * k + s) : 0.f;
+      apre[it] = (e < PR_JC * KM && jj < jn && s < k && LOCA_CHECK((j0 + jj) * k + s, d * k))
+                     ? __ldg(Al + (j0 + jj) * k + s)
+                     : 0.f;
     }
 #pragma unroll
     for (int it = 0; it < PR_LOADS; ++it) {
@@ -73,7 +75,7 @@ __global__ void __launch_bounds__(PR_THREADS, KM <= 16 ? 3 : 1) k_project_rows(c
       const int rr = e / (PR_JC / 4), c4 = (e % (PR_JC / 4)) * 4;
       const int64_t row = row0 + rr;
       float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (row < 2 * d) {
+      if (row < 2 * d && LOCA_CHECK_SPAN((row < d ? row : row - d) * d + j0 + c4, c4 + 4 <= jn ? 4 : jn - c4, d * d)) {
         const float* M = (row < d ? gram + int64_t(l) * d * d + row * d
                                   : cross + int64_t(l) * d * d + (row - d) * d) + j0 + c4;
         if (vec && c4 + 4 <= jn) {
@@ -126,7 +128,8 @@ __global__ void __launch_bounds__(PR_THREADS, KM <= 16 ? 3 : 1) k_project_rows(c
     float* out = (is_gram ? GA : CA) + part + (int64_t(l) * d + ri) * k;
 #pragma unroll
     for (int s = 0; s < SPT; ++s)
-      if (g * SPT + s < k) out[g * SPT + s] = acc[i][s];
+      if (g * SPT + s < k && LOCA_CHECK(part + (int64_t(l) * d + ri) * k + g * SPT + s, int64_t(PR_SPLIT) * gridDim.y * d * k))
+        out[g * SPT + s] = acc[i][s];
   }
 }
 
@@ -165,7 +168,7 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
     __syncthreads();
     for (int e = threadIdx.x; e < CS_ROWS * KM; e += CS_THREADS) {
       const int ii = e / KM, s = e % KM;
-      const bool ok = (i0 + ii < d) && s < k;
+      const bool ok = (i0 + ii < d) && s < k && LOCA_CHECK((i0 + ii) * k + s, d * k);
       As[ii][s] = ok ? Al[(i0 + ii) * k + s] : 0.f;
       float gsum = 0.f;
       if (ok)
@@ -207,11 +210,12 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
   if (G_out != nullptr && j == 0) {
     for (int e = threadIdx.x; e < k * k; e += CS_THREADS) {
       const int a = e / k, b = e % k;
-      G_out[(int64_t(l) * k + a) * k + b] = float(0.5 * (double(Gf[a][b]) + double(Gf[b][a])));
+      if (LOCA_CHECK((int64_t(l) * k + a) * k + b, int64_t(L) * k * k))
+        G_out[(int64_t(l) * k + a) * k + b] = float(0.5 * (double(Gf[a][b]) + double(Gf[b][a])));
     }
   }
   const int inf = chol_factor<KM>(Md, Lf, Linv, &s_info);
-  if (threadIdx.x == 0) info[int64_t(j) * L + l] = inf;
+  if (threadIdx.x == 0 && LOCA_CHECK(int64_t(j) * L + l, int64_t(gridDim.x) * L)) info[int64_t(j) * L + l] = inf;
 
   float* Bj = B + (int64_t(j) * L + l) * d * k;
   const float* Bp = B_prev ? B_prev + int64_t(l) * d * k : nullptr;
@@ -252,7 +256,8 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
       if (C_out != nullptr && j == 0 && on)
 #pragma unroll
         for (int r = 0; r < RW; ++r)
-          if (i0 + r < d) C_out[(int64_t(l) * d + i0 + r) * k + lane] = c[r];
+          if (i0 + r < d && LOCA_CHECK((int64_t(l) * d + i0 + r) * k + lane, int64_t(L) * d * k))
+            C_out[(int64_t(l) * d + i0 + r) * k + lane] = c[r];
       if (inf != 0) {
 #pragma unroll
         for (int r = 0; r < RW; ++r)
@@ -282,50 +287,53 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
       }
 #pragma unroll
       for (int r = 0; r < RW; ++r)
-        if (on && i0 + r < d) Bj[(i0 + r) * k + lane] = c[r];
+        if (on && i0 + r < d && LOCA_CHECK((i0 + r) * k + lane, d * k)) Bj[(i0 + r) * k + lane] = c[r];
     }
-    return;
-  }
-  for (int64_t i = threadIdx.x; i < d; i += CS_THREADS) {
-    float c[KM];
+  } else {
+    for (int64_t i = threadIdx.x; i < d; i += CS_THREADS) {
+      if (!LOCA_CHECK_SPAN(i * k, k, d * k) || !LOCA_CHECK_SPAN((int64_t(j) * L + l) * d * k + i * k, k,
+                                                               int64_t(gridDim.x) * L * d * k))
+        break;
+      float c[KM];
 #pragma unroll
-    for (int s = 0; s < KM; ++s) c[s] = 0.f;
+      for (int s = 0; s < KM; ++s) c[s] = 0.f;
 #pragma unroll 1
-    for (int z = 0; z < PR_SPLIT; ++z) {
-      const float* cz = CAl + z * zs + i * k;
+      for (int z = 0; z < PR_SPLIT; ++z) {
+        const float* cz = CAl + z * zs + i * k;
 #pragma unroll
-      for (int s = 0; s < KM; ++s)
-        if (s < k) c[s] += cz[s];
-    }
-#pragma unroll
-    for (int s = 0; s < KM; ++s) c[s] *= cs;
-    if (Bp != nullptr) {
-      float b[KM];
-#pragma unroll
-      for (int s = 0; s < KM; ++s) b[s] = (s < k) ? Bp[i * k + s] : 0.f;
-#pragma unroll
-      for (int s = 0; s < KM; ++s) {
-        float a = c[s];
-#pragma unroll
-        for (int t = 0; t < KM; ++t) a = fmaf(b[t], Gf[t][s], a);
-        c[s] = (s < k) ? a : 0.f;
+        for (int s = 0; s < KM; ++s)
+          if (s < k) c[s] += cz[s];
       }
-    }
-    if (C_out != nullptr && j == 0) {
+#pragma unroll
+      for (int s = 0; s < KM; ++s) c[s] *= cs;
+      if (Bp != nullptr) {
+        float b[KM];
+#pragma unroll
+        for (int s = 0; s < KM; ++s) b[s] = (s < k) ? Bp[i * k + s] : 0.f;
+#pragma unroll
+        for (int s = 0; s < KM; ++s) {
+          float a = c[s];
+#pragma unroll
+          for (int t = 0; t < KM; ++t) a = fmaf(b[t], Gf[t][s], a);
+          c[s] = (s < k) ? a : 0.f;
+        }
+      }
+      if (C_out != nullptr && j == 0 && LOCA_CHECK_SPAN((int64_t(l) * d + i) * k, k, int64_t(L) * d * k)) {
+#pragma unroll
+        for (int s = 0; s < KM; ++s)
+          if (s < k) C_out[(int64_t(l) * d + i) * k + s] = c[s];
+      }
+      if (inf != 0) {
+#pragma unroll
+        for (int s = 0; s < KM; ++s)
+          if (s < k) Bj[i * k + s] = 0.f;
+        continue;
+      }
+      chol_solve_row<KM>(Lf, Linv, c);
 #pragma unroll
       for (int s = 0; s < KM; ++s)
-        if (s < k) C_out[(int64_t(l) * d + i) * k + s] = c[s];
+        if (s < k) Bj[i * k + s] = c[s];
     }
-    if (inf != 0) {
-#pragma unroll
-      for (int s = 0; s < KM; ++s)
-        if (s < k) Bj[i * k + s] = 0.f;
-      continue;
-    }
-    chol_solve_row<KM>(Lf, Linv, c);
-#pragma unroll
-    for (int s = 0; s < KM; ++s)
-      if (s < k) Bj[i * k + s] = c[s];
   }
 }
 

@@ -38,10 +38,12 @@ __global__ void __launch_bounds__(256) k_sumsq(const void* __restrict__ Xv, int6
       // 8-element aligned interior
       int64_t vb = (beg + 7) / 8, ve = end / 8;
       for (int64_t e = beg + threadIdx.x; e < vb * 8 && e < end; e += blockDim.x) {
+        if (!LOCA_CHECK(e, n_el)) break;
         const float v = __bfloat162float(X[e]);
         part = fmaf(v, v, part);
       }
       for (int64_t vi = vb + threadIdx.x; vi < ve; vi += blockDim.x) {
+        if (!LOCA_CHECK_SPAN(vi * 8, 8, n_el)) break;
         const uint4 q = __ldg(reinterpret_cast<const uint4*>(X) + vi);
         const uint32_t w[4] = {q.x, q.y, q.z, q.w};
 #pragma unroll
@@ -53,11 +55,13 @@ __global__ void __launch_bounds__(256) k_sumsq(const void* __restrict__ Xv, int6
         if (++cnt == 4) { acc += part; part = 0.f; cnt = 0; }
       }
       for (int64_t e = (ve * 8 > vb * 8 ? ve * 8 : vb * 8) + threadIdx.x; e < end; e += blockDim.x) {
+        if (!LOCA_CHECK(e, n_el)) break;
         const float v = __bfloat162float(X[e]);
         part = fmaf(v, v, part);
       }
     } else {
       for (int64_t e = beg + threadIdx.x; e < end; e += blockDim.x) {
+        if (!LOCA_CHECK(e, n_el)) break;
         const float v = __bfloat162float(X[e]);
         part = fmaf(v, v, part);
         if (++cnt == 32) { acc += part; part = 0.f; cnt = 0; }
@@ -66,6 +70,7 @@ __global__ void __launch_bounds__(256) k_sumsq(const void* __restrict__ Xv, int6
   } else {
     const float* X = static_cast<const float*>(Xv) + int64_t(l) * n_el;
     for (int64_t e = beg + threadIdx.x; e < end; e += blockDim.x) {
+      if (!LOCA_CHECK(e, n_el)) break;
       const double v = X[e];
       acc = fma(v, v, acc);
     }
@@ -79,7 +84,7 @@ __global__ void __launch_bounds__(256) k_sumsq(const void* __restrict__ Xv, int6
   if (threadIdx.x == 0) {
     double a = 0.0;
     for (int i = 0; i < int(blockDim.x >> 5); ++i) a += red[i];
-    partials[int64_t(l) * kMaxPartials + blockIdx.x] = a;
+    if (LOCA_CHECK(blockIdx.x, kMaxPartials)) partials[int64_t(l) * kMaxPartials + blockIdx.x] = a;
   }
 }
 
@@ -87,7 +92,7 @@ __global__ void k_step(const double* __restrict__ partials, int G, int L, const 
                        float eta, int zero_first, double* __restrict__ xsq_total,
                        float* __restrict__ alpha) {
   const int l = blockIdx.x * blockDim.x + threadIdx.x;
-  if (l >= L) return;
+  if (l >= L || !LOCA_CHECK(G, kMaxPartials + 1)) return;
   double xb = 0.0;
   for (int g = 0; g < G; ++g) xb += partials[int64_t(l) * kMaxPartials + g];
   const double ts = tsq[l];
@@ -103,7 +108,8 @@ __global__ void __launch_bounds__(256) k_step_from_gram(const float* __restrict_
   const int l = blockIdx.x;
   const float* Gl = gram + int64_t(l) * d * d;
   double acc = 0.0;
-  for (int64_t j = threadIdx.x; j < d; j += 256) acc += double(Gl[j * (d + 1)]);
+  for (int64_t j = threadIdx.x; j < d; j += 256)
+    if (LOCA_CHECK(j * (d + 1), d * d)) acc += double(Gl[j * (d + 1)]);
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
@@ -141,8 +147,8 @@ __global__ void __launch_bounds__(256) k_gram_cross_f32(const float* __restrict_
     for (int e = threadIdx.x; e < FK * FT; e += 256) {
       const int kk = e / FT, c = e % FT;
       const int64_t n = n0 + kk;
-      As[kk][c] = (n < N && i0 + c < d) ? Rl[n * d + i0 + c] : 0.f;
-      Bs[kk][c] = (n < N && j0 + c < d) ? Xl[n * d + j0 + c] : 0.f;
+      As[kk][c] = (n < N && i0 + c < d && LOCA_CHECK(n * d + i0 + c, N * d)) ? Rl[n * d + i0 + c] : 0.f;
+      Bs[kk][c] = (n < N && j0 + c < d && LOCA_CHECK(n * d + j0 + c, N * d)) ? Xl[n * d + j0 + c] : 0.f;
     }
     __syncthreads();
 #pragma unroll
@@ -170,6 +176,7 @@ __global__ void __launch_bounds__(256) k_gram_cross_f32(const float* __restrict_
       const int64_t c = j0 + tx * 4 + j;
       if (c >= d) continue;
       if (is_gram && r > c) continue;
+      if (!LOCA_CHECK(r * d + c, d * d) || !LOCA_CHECK(c * d + r, d * d)) continue;
       const double v = al * acc[i][j];
       float* p = out + r * d + c;
       *p = zero_first ? float(v) : float(double(*p) + v);

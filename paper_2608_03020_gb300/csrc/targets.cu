@@ -164,11 +164,15 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
             const int s = s4 + u;
-            const float x = (jv && s < r) ? Ql[int64_t(s) * g.d + j0 + j] : 0.f;
+            const float x = (jv && s < r && LOCA_CHECK(int64_t(l) * r * g.d + int64_t(s) * g.d + j0 + j,
+                                                       int64_t(g.L) * r * g.d))
+                                ? Ql[int64_t(s) * g.d + j0 + j]
+                                : 0.f;
             hi[u] = tf32_rna(x);
             lo[u] = tf32_rna(x - __uint_as_float(hi[u]));
           }
           const uint32_t off = kmaj_off(j, s4, rp);
+          if (!LOCA_CHECK_SPAN(off, 16, uint32_t(TCH) * rp * 4)) continue;
           *reinterpret_cast<uint4*>(smem + lay.b_hi + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
           *reinterpret_cast<uint4*>(smem + lay.b_lo + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
         }
@@ -183,7 +187,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         float u[kMaxRP];
 #pragma unroll
         for (int s = 0; s < kMaxRP; ++s) u[s] = 0.f;
-        if (n < nend) {
+        if (n < nend && LOCA_CHECK_SPAN(n * C, C, g.N * C) && LOCA_CHECK_SPAN(int64_t(l) * C * r, C * r, int64_t(g.L) * C * r)) {
           const float* er = E + n * C;
           for (int c = 0; c < C; ++c) {
             const float ec = er[c];
@@ -204,6 +208,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             lo[v] = tf32_rna(u[s4 + v] - __uint_as_float(hi[v]));
           }
           const uint32_t off = kmaj_off(i, s4, rp);
+          if (!LOCA_CHECK_SPAN(off, 16, uint32_t(TM) * rp * 4)) continue;
           *reinterpret_cast<uint4*>(smem + lay.a_hi[buf] + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
           *reinterpret_cast<uint4*>(smem + lay.a_lo[buf] + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
         }
@@ -313,12 +318,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             if (lane == 0) {
               const int rows0 = int(n0) + q * 32;
               if (store_mode == 1) {
-                if (rows0 < nend && j0 + 64 * cp < g.d)
+                if (rows0 < nend && j0 + 64 * cp < g.d && LOCA_REQUIRE(rows0 >= 0 && (j0 + 64 * cp) % 8 == 0))
                   tma_store_3d(&tmT, stage + uint32_t(cp) * (32u * 128u), int(j0) + 64 * cp, rows0, l);
                 bulk_commit_group();
               } else if (cp & 1) {
                 const int h = cp >> 1;  // boxes 2h, 2h+1 leave as one 4-D box of two channel blocks
-                if (rows0 < nend && j0 + 128 * h < g.d)
+                if (rows0 < nend && j0 + 128 * h < g.d && LOCA_REQUIRE(rows0 >= 0 && j0 % 64 == 0))
                   tma_store_4d(&tmT, stage + uint32_t(h) * (64u * 128u), 0, rows0, int(j0 / 64) + 2 * h, l);
                 bulk_commit_group();
               }
@@ -330,6 +335,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             const float* vv = v + 32 * hh;
             const int64_t jb = j0 + cp * 64 + hh * 32;
             if (!nv || jb >= g.d) continue;
+            if (!LOCA_CHECK_SPAN(rbase + jb, jb + 32 <= g.d ? 32 : g.d - jb, int64_t(g.L) * g.N * g.d)) continue;
             const bool whole = (jb + 32 <= g.d) && (g.d % 8 == 0);
             if (whole) {
               if (kBF16) {
@@ -365,7 +371,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         // one partial per (item, epilogue warp): no synchronisation across warps
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) sqd += __shfl_xor_sync(0xffffffffu, sqd, off);
-        if (lane == 0) partials[((int64_t(l) * g.nd + jt) * g.nchunks + ck) * 4 + q] = sqd;
+        if (lane == 0 && LOCA_CHECK(((int64_t(l) * g.nd + jt) * g.nchunks + ck) * 4 + q, int64_t(g.L) * g.nd * g.nchunks * 4))
+          partials[((int64_t(l) * g.nd + jt) * g.nchunks + ck) * 4 + q] = sqd;
       }
     }
   }
@@ -383,7 +390,8 @@ __global__ void __launch_bounds__(256) k_reduce_partials(const double* __restric
   __shared__ double sm[256];
   const int l = blockIdx.x;
   double a = 0.0;
-  for (int64_t i = threadIdx.x; i < nparts; i += 256) a += partials[int64_t(l) * nparts + i];
+  for (int64_t i = threadIdx.x; i < nparts; i += 256)
+    if (LOCA_CHECK(int64_t(l) * nparts + i, int64_t(gridDim.x) * nparts)) a += partials[int64_t(l) * nparts + i];
   sm[threadIdx.x] = a;
   __syncthreads();
   for (int w = 128; w > 0; w >>= 1) {

@@ -26,8 +26,9 @@ __global__ void __launch_bounds__(TSQ_THREADS) k_tsq_ete(const float* __restrict
   for (int e = threadIdx.x; e < C * C; e += TSQ_THREADS) {
     const int a = e / C, b = e % C;
     double acc = 0.0;
-    for (int64_t n = n0; n < n1; ++n) acc += double(E[n * C + a]) * double(E[n * C + b]);
-    out[e] = acc;
+    for (int64_t n = n0; n < n1; ++n)
+      if (LOCA_CHECK(n * C + a, N * C) && LOCA_CHECK(n * C + b, N * C)) acc += double(E[n * C + a]) * double(E[n * C + b]);
+    if (LOCA_CHECK(int64_t(blockIdx.x) * C * C + e, int64_t(gridDim.x) * C * C)) out[e] = acc;
   }
 }
 
@@ -41,7 +42,7 @@ __global__ void __launch_bounds__(TSQ_THREADS) k_tsq_block(const double* __restr
   const int l = blockIdx.x;
   for (int e = threadIdx.x; e < C * C; e += TSQ_THREADS) {
     double acc = 0.0;
-    for (int c = 0; c < nchunks; ++c) acc += part[int64_t(c) * C * C + e];
+    for (int c = 0; c < nchunks; ++c) acc += part[int64_t(c) * C * C + e];  // e < C * C
     ete[e] = acc;
   }
   // M = Q_l Q_l^T: one warp per entry (s, t), lanes over channels, fp32 runs of 32 products
@@ -88,7 +89,7 @@ __global__ void __launch_bounds__(TSQ_THREADS) k_tsq_block(const double* __restr
     if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
     __syncthreads();
   }
-  if (threadIdx.x == 0) tsq[l] = red[0];
+  if (threadIdx.x == 0 && LOCA_CHECK(l, gridDim.x)) tsq[l] = red[0];
 }
 
 }  // namespace

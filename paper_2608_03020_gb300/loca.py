@@ -16,6 +16,7 @@ import torch
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libloca.so")
+LIB_DEBUG_PATH = os.path.join(_PKG, "libloca_debug.so")  # built with -DLOCA_DEBUG (bounds checks)
 
 LOCA_F32 = 0
 LOCA_BF16 = 1
@@ -23,7 +24,7 @@ LOCA_BF16 = 1
 STATUS_NAMES = {
     0: "LOCA_OK", 1: "LOCA_ERR_INVALID_ARG", 2: "LOCA_ERR_SHAPE", 3: "LOCA_ERR_ALIGNMENT",
     4: "LOCA_ERR_UNSUPPORTED_DTYPE", 5: "LOCA_ERR_CUDA", 6: "LOCA_ERR_TIMEOUT",
-    7: "LOCA_ERR_WORKSPACE", 8: "LOCA_ERR_UNSUPPORTED", 9: "LOCA_ERR_NUMERIC",
+    7: "LOCA_ERR_WORKSPACE", 8: "LOCA_ERR_UNSUPPORTED", 9: "LOCA_ERR_NUMERIC", 10: "LOCA_ERR_BOUNDS",
 }
 
 # (name, restype, argtypes) of every exported entry point
@@ -36,6 +37,7 @@ SIGNATURES = [
     ("loca_version", ctypes.c_int, []),
     ("loca_last_error_string", ctypes.c_char_p, []),
     ("loca_device_status", ctypes.c_int, [ctypes.POINTER(_I32), _P]),
+    ("loca_debug_build", ctypes.c_int, []),
     ("loca_set_wait_limit", ctypes.c_int, [ctypes.c_uint64]),
     ("loca_error", ctypes.c_int, [_P, ctypes.c_int, _I64, _I64, _I64, _P, _I32, _P, _P, ctypes.c_int, _P, _P, _P]),
     ("loca_targets_workspace_size", ctypes.c_int, [_I64, _I32, _I64, ctypes.POINTER(_SZ)]),
@@ -87,21 +89,44 @@ class LocaError(RuntimeError):
 
 
 _lib = None
+_loaded = {}
 
 
-def lib() -> ctypes.CDLL:
-    """Load ``libloca.so`` (built in-tree by ``_build.build()``); fails loudly if missing."""
-    global _lib
-    if _lib is None:
-        if not os.path.exists(LIB_PATH):
-            raise RuntimeError(f"{LIB_PATH} is not built: run __graft_entry__.build() (nvcc, sm_103a)")
-        h = ctypes.CDLL(LIB_PATH)
+def _load(path: str) -> ctypes.CDLL:
+    if path not in _loaded:
+        if not os.path.exists(path):
+            raise RuntimeError(f"{path} is not built: run __graft_entry__.build() (nvcc, sm_103a)")
+        h = ctypes.CDLL(path)
         for name, res, args in SIGNATURES:
             fn = getattr(h, name)
             fn.restype = res
             fn.argtypes = args
-        _lib = h
+        _loaded[path] = h
+    return _loaded[path]
+
+
+def lib() -> ctypes.CDLL:
+    """The library every function here calls: ``libloca.so`` (built in-tree by
+    ``_build.build()``) unless :func:`use_debug_library` switched it; fails loudly if missing."""
+    global _lib
+    if _lib is None:
+        _lib = _load(LIB_PATH)
     return _lib
+
+
+def use_debug_library(on: bool = True) -> ctypes.CDLL:
+    """Route every function of this module to ``libloca_debug.so`` (``_build.build(debug=True)``:
+    the same entry points with index bounds checks reported as LOCA_ERR_BOUNDS by
+    :func:`loca_device_status`), or back to ``libloca.so``.  Each library keeps its own device
+    status word; returns the library now in use."""
+    global _lib
+    _lib = _load(LIB_DEBUG_PATH if on else LIB_PATH)
+    return _lib
+
+
+def loca_debug_build() -> bool:
+    """True when the library in use is the LOCA_DEBUG build."""
+    return bool(lib().loca_debug_build())
 
 
 def _check(rc: int, where: str):
@@ -156,10 +181,17 @@ def loca_version() -> int:
 
 
 def loca_device_status(stream=None) -> int:
-    """Read and clear the device status word (LOCA_OK or LOCA_ERR_TIMEOUT)."""
+    """Read and clear the device status word (LOCA_OK or a device-side code: LOCA_ERR_TIMEOUT,
+    LOCA_ERR_NUMERIC, or in the debug build LOCA_ERR_BOUNDS, whose source line
+    :func:`loca_last_error` then names)."""
     out = ctypes.c_int32(0)
     _check(lib().loca_device_status(ctypes.byref(out), _stream(stream)), "loca_device_status")
     return out.value
+
+
+def loca_last_error() -> str:
+    """Message of the last non-OK status of the calling thread (``loca_last_error_string``)."""
+    return lib().loca_last_error_string().decode(errors="replace")
 
 
 def loca_set_wait_limit(ns: int):

@@ -190,3 +190,22 @@ def test_calib_rsvd_validation(L):
     floor = 12 * 3584 * 3584 + (8 * 2 * 3584 + 4 * 3584 + 12 * 3584 + 4 * 8192) * n_cols
     assert rc == 0 and floor <= n < floor + (16 << 20) and n % 256 == 0
     assert _ws(L.loca_calib_fit_rsvd_workspace_size, 8192, 3584, 3584, 28, 33, 32)[0] == 2
+
+
+def test_debug_library_builds_and_exports_every_declared_symbol(L):
+    """The LOCA_DEBUG build (bounds checks in every kernel) has the release library's ABI and says
+    which it is; the release build compiles the checks away."""
+    from paper_2608_03020_gb300 import _build
+    from paper_2608_03020_gb300 import loca
+
+    _build.build(debug=True)
+    D = loca.use_debug_library(True)
+    try:
+        for name in _declared():
+            assert hasattr(D, name), name
+        assert loca.loca_debug_build() and D.loca_version() == L.loca_version()
+    finally:
+        loca.use_debug_library(False)
+    assert not loca.loca_debug_build()
+    # host validation is the same code in both builds
+    assert D.loca_targets_workspace_size(1, 1, 1, None) == 1
