@@ -431,7 +431,7 @@ def measure_workload(lc, name, dev, stream, steps, warmup, peak, hbm, wpeak):
     out["targets_roofline"] = hbm_object(L * N * d * T.element_size(), stages["targets"], "k_targets_tc", hbm,
                                          wpeak)
     out["ridge_solve_roofline"] = hbm_object(2 * L * d * d * 4, stages["ridge_solve"],
-                                             "k_project_rows + k_chol_solve (reads of Gram and cross)", hbm)
+                                             "k_project_tc + k_chol_solve (reads of Gram and cross)", hbm)
     del inp, X, z, T, gram, cross, E, ce, B
     torch.cuda.synchronize()
     torch.cuda.empty_cache()
@@ -573,7 +573,7 @@ def main():
     targets_roofline = hbm_object(L * N * d * T.element_size(), stages["targets"], "k_targets_tc", hbm, wpeak)
     targets_roofline["traffic"] = recorded_traffic(TARGETS_TRAFFIC, "targets.cu", L, N=N, d=d, r=r)
     solve_roofline = hbm_object(2 * L * d * d * 4, stages["ridge_solve"],
-                                "k_project_rows + k_chol_solve (reads of Gram and cross)", hbm)
+                                "k_project_tc + k_chol_solve (reads of Gram and cross)", hbm)
 
     # the paper's own k-space statistics on the same inputs (no T, no d x d statistics):
     # error -> k-space accumulate (X A_l on the tensor cores, one HBM read of X) -> k-space solve

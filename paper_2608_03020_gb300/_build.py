@@ -23,7 +23,7 @@ LIB_DEBUG = os.path.join(PKG, "libloca_debug.so")
 BUILD_DEBUG = os.path.join(PKG, "_build_debug")
 SOURCES = ["loca_abi.cu", "error.cu", "targets.cu", "stats.cu", "gram_tc.cu", "solve.cu", "calib.cu",
            "noalloc.cu", "host_mem.cu", "kspace.cu", "align.cu", "calib_rsvd.cu",
-           "targets_sq.cu"]
+           "targets_sq.cu", "project_tc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVFLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
                   "-I" + os.path.join(ROOT, "include")]

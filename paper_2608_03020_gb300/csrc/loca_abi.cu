@@ -146,14 +146,15 @@ AccumWs accum_ws(int32_t L) {
 }
 
 struct SolveWs {
-  size_t ga, ca, total;
+  size_t ga, ca, flag, total;
 };
 SolveWs solve_ws(int32_t L, int64_t d, int32_t k) {
   SolveWs w{};
   const size_t one = align256(sizeof(float) * size_t(project_split()) * size_t(L) * size_t(d) * size_t(k));
   w.ga = 0;
   w.ca = one;
-  w.total = 2 * one;
+  w.flag = 2 * one;  // abort flag of the tensor-core projection's bounded waits
+  w.total = 2 * one + 256;
   return w;
 }
 
@@ -693,9 +694,20 @@ int loca_ridge_solve(const float* gram, const float* cross, const float* cross_s
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   float* GA = reinterpret_cast<float*>(ws_at(workspace, lay.ga));
   float* CA = reinterpret_cast<float*>(ws_at(workspace, lay.ca));
-  cudaError_t e = launch_project_rows(gram, cross, A, L, d, k, GA, CA, s);
+  cudaError_t e;
+  int nsplit;
+  if (project_tc_supported(gram, cross, A, d, k)) {
+    int32_t* status = device_status_word();
+    if (!status) return fail(LOCA_ERR_CUDA, "cannot resolve the device status word");
+    e = launch_project_tc(gram, cross, A, L, d, k, GA, CA, status,
+                          reinterpret_cast<int32_t*>(ws_at(workspace, lay.flag)), s);
+    nsplit = 1;
+  } else {
+    e = launch_project_rows(gram, cross, A, L, d, k, GA, CA, s);
+    nsplit = project_split();
+  }
   if (e != cudaSuccess) return cuda_fail(e, "loca_ridge_solve: projection");
-  e = launch_chol_solve(GA, CA, A, B_prev, xsq_total, cross_scale, lambda_rel, nl, L, d, k, B, info, G_out,
+  e = launch_chol_solve(GA, CA, nsplit, A, B_prev, xsq_total, cross_scale, lambda_rel, nl, L, d, k, B, info, G_out,
                         C_out, s);
   if (e != cudaSuccess) return cuda_fail(e, "loca_ridge_solve: solve");
   return LOCA_OK;

@@ -122,12 +122,18 @@ cudaError_t launch_kspace_solve(const float* G, const float* SC, const double* x
                                 int64_t d, int k, int C, int r, float* B, int32_t* info, float* C_out,
                                 cudaStream_t s);
 
-// ---- ridge solve (solve.cu)
-// GA / CA are project_split() partial products each (L x d x k fp32 apiece), summed by the solve.
+// ---- ridge solve (solve.cu, project_tc.cu)
+// k_project_rows writes GA / CA as project_split() partial products each (L x d x k fp32 apiece);
+// the tensor-core projection writes one (nsplit = 1).  The solve sums the nsplit partials.
 int project_split();
 cudaError_t launch_project_rows(const float* gram, const float* cross, const float* A, int L,
                                 int64_t d, int k, float* GA, float* CA, cudaStream_t s);
-cudaError_t launch_chol_solve(const float* GA, const float* CA, const float* A, const float* B_prev,
+// Tensor-core projection (tf32 MMAs with the 3xTF32 split): d % 4 == 0, k % 4 == 0, 4 <= k <= 32,
+// 16-byte aligned gram, cross and A.  abort_flag: 4 bytes of launch-local device memory.
+bool project_tc_supported(const float* gram, const float* cross, const float* A, int64_t d, int k);
+cudaError_t launch_project_tc(const float* gram, const float* cross, const float* A, int L, int64_t d, int k,
+                              float* GA, float* CA, int32_t* status, int32_t* abort_flag, cudaStream_t s);
+cudaError_t launch_chol_solve(const float* GA, const float* CA, int nsplit, const float* A, const float* B_prev,
                               const double* xsq_total, const float* cross_scale, const float* lambda_rel,
                               int nl, int L, int64_t d, int k, float* B, int32_t* info, float* G_out,
                               float* C_out, cudaStream_t s);

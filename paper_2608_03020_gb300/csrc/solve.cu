@@ -1,6 +1,8 @@
 // Projected statistics and batched positive-definite solves (Eqs. 8 and 9; Theorem S6; S7).
 //
-// k_project_rows  GA_l = Gram_l A_l, CA_l = Cross_l A_l (d x k each), as PR_SPLIT partial
+// k_project_rows  (shapes the tensor-core projection of project_tc.cu does not take: d or k not a
+//                 multiple of 4, unaligned pointers)
+//                 GA_l = Gram_l A_l, CA_l = Cross_l A_l (d x k each), as PR_SPLIT partial
 //                 products over quarters of the column range (GA = sum_z GA_z, summed in a fixed
 //                 order by k_chol_solve).  A CTA takes 256 rows of the stacked [Gram_l; Cross_l]
 //                 and one column quarter; 32-column slabs of its rows are staged in shared memory
@@ -9,6 +11,7 @@
 //                 RPT rows x SPT columns of the product with A's slab (broadcast reads).  Bound: the
 //                 HBM read of Gram and Cross (8 d^2 bytes per block).
 // k_chol_solve    one thread block per (ridge candidate j, block l):
+//                 GA_l and CA_l summed over their nsplit partial products (fixed order),
 //                 G_l = A_l^T GA_l (k x k), lambda from the trace, Cholesky of G_l + lambda I in
 //                 fp64 in shared memory, then every row i of C_l = B_prev,l G_l + s_l CA_l
 //                 (s_l = cross_scale[l], or 1) is solved
@@ -138,7 +141,7 @@ constexpr int CS_ROWS = 64;  // rows of A / GA staged per step when forming G
 
 template <int KM>
 __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
-    const float* __restrict__ GA, const float* __restrict__ CA, const float* __restrict__ A,
+    const float* __restrict__ GA, const float* __restrict__ CA, int nsplit, const float* __restrict__ A,
     const float* __restrict__ B_prev, const double* __restrict__ xsq_total, const float* __restrict__ cross_scale,
     int64_t d, int k, int L,
     float l0, float l1, float l2, float l3, float l4, float l5, float l6, float l7, float l8,
@@ -157,7 +160,7 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
   const float* Al = A + int64_t(l) * d * k;
   const float* GAl = GA + int64_t(l) * d * k;
   const float* CAl = CA + int64_t(l) * d * k;
-  const int64_t zs = int64_t(L) * d * k;  // stride between the PR_SPLIT partial products
+  const int64_t zs = int64_t(L) * d * k;  // stride between the nsplit partial products
 
   // G_l = A_l^T GA_l: thread owns entries e = t, t + 256, ... of the KM x KM matrix
   constexpr int PER = (KM * KM + CS_THREADS - 1) / CS_THREADS;
@@ -172,7 +175,7 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
       As[ii][s] = ok ? Al[(i0 + ii) * k + s] : 0.f;
       float gsum = 0.f;
       if (ok)
-        for (int z = 0; z < PR_SPLIT; ++z) gsum += GAl[z * zs + (i0 + ii) * k + s];
+        for (int z = 0; z < nsplit; ++z) gsum += GAl[z * zs + (i0 + ii) * k + s];
       Gs[ii][s] = gsum;
     }
     __syncthreads();
@@ -236,7 +239,7 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
         const int64_t i = i0 + r;
         float v = 0.f;
         if (on && i < d)
-          for (int z = 0; z < PR_SPLIT; ++z) v += CAl[z * zs + i * k + lane];
+          for (int z = 0; z < nsplit; ++z) v += CAl[z * zs + i * k + lane];
         c[r] = v * cs;
       }
       if (Bp != nullptr) {
@@ -298,7 +301,7 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
 #pragma unroll
       for (int s = 0; s < KM; ++s) c[s] = 0.f;
 #pragma unroll 1
-      for (int z = 0; z < PR_SPLIT; ++z) {
+      for (int z = 0; z < nsplit; ++z) {
         const float* cz = CAl + z * zs + i * k;
 #pragma unroll
         for (int s = 0; s < KM; ++s)
@@ -349,13 +352,13 @@ cudaError_t project_t(const float* gram, const float* cross, const float* A, int
 }
 
 template <int KM>
-cudaError_t solve_t(const float* GA, const float* CA, const float* A, const float* B_prev,
+cudaError_t solve_t(const float* GA, const float* CA, int nsplit, const float* A, const float* B_prev,
                     const double* xsq_total, const float* cross_scale, const float* lr, int nl, int L,
                     int64_t d, int k, float* B, int32_t* info, float* G_out, float* C_out, cudaStream_t s) {
   float v[16] = {};
   for (int i = 0; i < nl && i < 16; ++i) v[i] = lr[i];
   const dim3 grid = dim3(unsigned(nl), unsigned(L));
-  k_chol_solve<KM><<<grid, CS_THREADS, 0, s>>>(GA, CA, A, B_prev, xsq_total, cross_scale, d, k, L, v[0], v[1],
+  k_chol_solve<KM><<<grid, CS_THREADS, 0, s>>>(GA, CA, nsplit, A, B_prev, xsq_total, cross_scale, d, k, L, v[0], v[1],
                                                v[2], v[3], v[4], v[5], v[6], v[7], v[8], v[9],
                                                v[10], v[11], v[12], v[13], v[14], v[15], B, info,
                                                G_out, C_out);
@@ -375,12 +378,12 @@ cudaError_t launch_project_rows(const float* gram, const float* cross, const flo
   return project_t<64>(gram, cross, A, L, d, k, GA, CA, s);
 }
 
-cudaError_t launch_chol_solve(const float* GA, const float* CA, const float* A, const float* B_prev,
+cudaError_t launch_chol_solve(const float* GA, const float* CA, int nsplit, const float* A, const float* B_prev,
                               const double* xsq_total, const float* cross_scale, const float* lambda_rel,
                               int nl, int L, int64_t d, int k, float* B, int32_t* info, float* G_out,
                               float* C_out, cudaStream_t s) {
 #define LOCA_SOLVE(KM)                                                                               \
-  return solve_t<KM>(GA, CA, A, B_prev, xsq_total, cross_scale, lambda_rel, nl, L, d, k, B, info, G_out, \
+  return solve_t<KM>(GA, CA, nsplit, A, B_prev, xsq_total, cross_scale, lambda_rel, nl, L, d, k, B, info, G_out, \
                      C_out, s)
   if (k <= 4) LOCA_SOLVE(4);
   if (k <= 8) LOCA_SOLVE(8);

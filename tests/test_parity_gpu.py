@@ -381,6 +381,43 @@ def test_ridge_solve_parity(lc, k, d, L, with_prev, relative):
             assert _rel(_np(B)[j, l], B_ref[j, l]) < 1e-5, (j, l)
 
 
+@pytest.mark.parametrize("k,d,L", [
+    (16, 3584, 2),   # the 7B width: tensor-core projection, 28 row tiles and 112 K-slabs per matrix
+    (32, 5120, 1),   # the 14B width (k = 32)
+    (12, 1000, 2),   # k padded to 16, a ragged last row tile (104 rows) and a ragged last K-slab
+    (6, 330, 2),     # k % 4 != 0 and d % 4 != 0: the SIMT projection
+])
+def test_ridge_solve_parity_at_full_width(lc, k, d, L):
+    """Eq. 9 projections and Theorem S6 solves at the widths of the headline workloads: the Gram
+    stand-in is X^T X + diag over 256 rows with LogNormal channel scales (positive definite), the
+    cross product dense; 1e-5 relative Frobenius on G = A^T Gram A, C = B_prev G + Cross A and B."""
+    rng = np.random.default_rng(k + d)
+    Y = rng.standard_normal((L, 256, d)) * rng.lognormal(0, 0.5, (L, 1, d))
+    g = np.transpose(Y, (0, 2, 1)) @ Y
+    g[:, np.arange(d), np.arange(d)] += rng.uniform(0.5, 2.0, (L, d))
+    c = 0.1 * rng.standard_normal((L, d, d)) * rng.lognormal(0, 0.5, (L, 1, d))
+    g32, c32 = g.astype(np.float32), c.astype(np.float32)
+    xs = np.trace(g32.astype(np.float64), axis1=1, axis2=2)
+    A = np.stack([np.linalg.qr(rng.standard_normal((d, k)))[0] for _ in range(L)]).astype(np.float32)
+    Bp = (0.01 * rng.standard_normal((L, d, k))).astype(np.float32)
+    lam_rel = [1e-4, 1e-2]
+    G_ref, C_ref = O.project_stats(g32, c32, A, B_prev=Bp)
+    B_ref, info_ref = O.ridge_solve(G_ref, C_ref, O.ridge_lambdas(lam_rel, xs, d))
+    B = torch.empty((2, L, d, k), device="cuda")
+    info = torch.empty((2, L), dtype=torch.int32, device="cuda")
+    Gout = torch.empty((L, k, k), device="cuda")
+    Cout = torch.empty((L, d, k), device="cuda")
+    lc.loca_ridge_solve(_dev(g32), _dev(c32), _dev(A), lam_rel, B, info, xsq_total=_dev(xs, torch.float64),
+                        B_prev=_dev(Bp), G_out=Gout, C_out=Cout)
+    torch.cuda.synchronize()
+    assert lc.loca_device_status() == 0
+    assert np.array_equal(info.cpu().numpy(), info_ref)
+    eg, ec = _rel(_np(Gout), G_ref), _rel(_np(Cout), C_ref)
+    eb = max(_rel(_np(B)[j, l], B_ref[j, l]) for j in range(2) for l in range(L))
+    print(f"k={k} d={d}: rel err G {eg:.2e} C {ec:.2e} B {eb:.2e}")
+    assert eg < 1e-5 and ec < 1e-5 and eb < 1e-5
+
+
 def test_ridge_solve_reports_not_positive_definite(lc):
     L, d, k = 1, 32, 4
     g = -np.eye(d, dtype=np.float32)[None] * 100.0
