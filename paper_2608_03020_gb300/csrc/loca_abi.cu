@@ -146,15 +146,16 @@ AccumWs accum_ws(int32_t L) {
 }
 
 struct SolveWs {
-  size_t ga, ca, flag, total;
+  size_t ga, ca, fac, flag, total;
 };
 SolveWs solve_ws(int32_t L, int64_t d, int32_t k) {
   SolveWs w{};
   const size_t one = align256(sizeof(float) * size_t(project_split()) * size_t(L) * size_t(d) * size_t(k));
   w.ga = 0;
   w.ca = one;
-  w.flag = 2 * one;  // abort flag of the tensor-core projection's bounded waits
-  w.total = 2 * one + 256;
+  w.fac = 2 * one;  // per-candidate Cholesky factors
+  w.flag = w.fac + align256(chol_workspace_bytes(L));  // abort flag of the tensor-core projection's waits
+  w.total = w.flag + 256;
   return w;
 }
 
@@ -708,7 +709,7 @@ int loca_ridge_solve(const float* gram, const float* cross, const float* cross_s
   }
   if (e != cudaSuccess) return cuda_fail(e, "loca_ridge_solve: projection");
   e = launch_chol_solve(GA, CA, nsplit, A, B_prev, xsq_total, cross_scale, lambda_rel, nl, L, d, k, B, info, G_out,
-                        C_out, s);
+                        C_out, reinterpret_cast<float*>(ws_at(workspace, lay.fac)), s);
   if (e != cudaSuccess) return cuda_fail(e, "loca_ridge_solve: solve");
   return LOCA_OK;
 }

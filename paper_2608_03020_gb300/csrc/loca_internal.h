@@ -133,10 +133,12 @@ cudaError_t launch_project_rows(const float* gram, const float* cross, const flo
 bool project_tc_supported(const float* gram, const float* cross, const float* A, int64_t d, int k);
 cudaError_t launch_project_tc(const float* gram, const float* cross, const float* A, int L, int64_t d, int k,
                               float* GA, float* CA, int32_t* status, int32_t* abort_flag, cudaStream_t s);
+// fac: chol_workspace_bytes(L) of device memory for the per-candidate factors (nl <= 16).
+size_t chol_workspace_bytes(int L);
 cudaError_t launch_chol_solve(const float* GA, const float* CA, int nsplit, const float* A, const float* B_prev,
                               const double* xsq_total, const float* cross_scale, const float* lambda_rel,
                               int nl, int L, int64_t d, int k, float* B, int32_t* info, float* G_out,
-                              float* C_out, cudaStream_t s);
+                              float* C_out, float* fac, cudaStream_t s);
 
 // ---- calibration (calib.cu)
 size_t calib_workspace_bytes(int64_t Np, int m, int64_t d, int L, int r);

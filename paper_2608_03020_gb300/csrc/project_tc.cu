@@ -20,10 +20,11 @@
 // Persistent, one CTA per SM, 448 threads, three rings so that no role waits on another's latency:
 //   warp 0      TMA producer: per K-slab a 128 x 32 fp32 tile of the matrix (128-byte swizzle) and
 //               the 32 x k rows of A_l (plain) into a raw stage (PT_RAW stages).
-//   warps 6-13  two groups of four, taking turns over the stages: split a raw stage into a split
-//               buffer (PT_SPLIT buffers): the tile's hi / mid / lo bf16 parts and A's slab parts,
-//               all K-major without swizzle (8-row x 16-byte core matrices); the raw stage is free
-//               as soon as it is read.
+//   warps 6-13  split a raw stage into a split buffer (PT_SPLIT buffers): the tile's hi / mid / lo
+//               bf16 parts and A's slab parts, all K-major without swizzle (8-row x 16-byte core
+//               matrices); the raw stage is released as soon as its values are in registers.  A
+//               stage's MMAs free its split buffer, so the split of stage t waits for the MMAs of
+//               stage t - PT_SPLIT: the buffers, not the TMA ring, set the loop that bounds the rate.
 //   warp 1      owns the TMEM accumulators (PT_ACC of 128 lanes x 3 KN columns) and issues the
 //               MMAs (kind::f16, M = 128, N = 3 KN, K = 16), one accumulator per K-slab.
 //   warps 2-5   read each slab's accumulator (TMEM lane quarter warp % 4), add its three column
@@ -43,8 +44,8 @@ namespace {
 using namespace tc;
 
 constexpr int PT_THREADS = 448;
-constexpr int PT_RAW = 6;     // raw stages (TMA in flight)
-constexpr int PT_SPLIT = 2;   // split buffers (MMA operands)
+constexpr int PT_RAW = 5;     // raw stages (TMA in flight)
+constexpr int PT_SPLIT = 4;   // split buffers (MMA operands)
 constexpr int PT_ACC = 4;     // TMEM accumulators
 constexpr int PT_CONV_WARPS = 8;
 constexpr int PT_GROUPS = 2;  // split groups: group g takes the stages t with t % PT_GROUPS == g
@@ -289,12 +290,15 @@ __global__ void __launch_bounds__(PT_THREADS, 1)
       }
     }
   } else {
-    // ---------------- warps 6..13: split raw stages into split buffers; the two groups take turns,
-    // so that the latency of one stage's split overlaps the next one's
+    // ---------------- warps 6..13: split raw stages into split buffers (the groups take turns when
+    // there are several, so that one stage's split latency overlaps the next one's)
     const int grp = (warp - 6) / PT_GROUP_WARPS;
     const int ct = threadIdx.x - 6 * 32 - grp * PT_GROUP_WARPS * 32;  // thread within the group
     constexpr int NT = PT_GROUP_WARPS * 32;
-    static_assert(NT == PT_TM, "one row of the tile per thread and 8-column group");
+    constexpr int UPT = PT_TM * (PT_BK / 8) / NT;  // 8-channel chunks of one row per thread
+    static_assert(NT % PT_TM == 0 && UPT >= 1, "whole rows of chunks per thread");
+    const int r = ct % PT_TM;                       // the tile row of this thread
+    const int u0 = (ct / PT_TM) * UPT;              // its first 8-channel chunk
     uint32_t t = 0;
     bool ok = true;
     for (int it = blockIdx.x; it < g.items && ok; it += gridDim.x) {
@@ -310,45 +314,62 @@ __global__ void __launch_bounds__(PT_THREADS, 1)
         }
         const uint8_t* rp = smem + uint32_t(s) * PL::raw_bytes;
         uint8_t* sp = smem + PL::split_base + uint32_t(b) * PL::split_bytes;
-        // the matrix tile: row r, channels 8u .. 8u + 7 are the raw 16-byte chunks 2u and 2u + 1 of
-        // the row, found at positions (2u) ^ (r % 8) and (2u + 1) ^ (r % 8) (128-byte swizzle)
-        const int r = ct;
+        // read everything this thread needs from the raw stage first: row r, channels 8u .. 8u + 7
+        // are the raw 16-byte chunks 2u and 2u + 1 of the row, at positions (2u) ^ (r % 8) and
+        // (2u + 1) ^ (r % 8) (128-byte swizzle); then A's values for the B rows
+        float xv[UPT][8];
+        const uint8_t* row = rp + uint32_t(r) * 128u;
 #pragma unroll
-        for (int u = 0; u < PT_BK / 8; ++u) {
-          const uint8_t* row = rp + uint32_t(r) * 128u;
+        for (int j = 0; j < UPT; ++j) {
+          const int u = u0 + j;
           const float4 x0 = *reinterpret_cast<const float4*>(row + ((uint32_t(2 * u) ^ uint32_t(r & 7)) << 4));
           const float4 x1 = *reinterpret_cast<const float4*>(row + ((uint32_t(2 * u + 1) ^ uint32_t(r & 7)) << 4));
-          const float xv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-          uint4 h, m, lo;
-          split8(xv, h, m, lo);
-          const uint32_t off = kmaj_chunk(r, u);
-          if (!LOCA_CHECK_SPAN(off, 16, PT_PART)) continue;
-          *reinterpret_cast<uint4*>(sp + off) = h;
-          *reinterpret_cast<uint4*>(sp + PT_PART + off) = m;
-          *reinterpret_cast<uint4*>(sp + 2 * PT_PART + off) = lo;
+          xv[j][0] = x0.x; xv[j][1] = x0.y; xv[j][2] = x0.z; xv[j][3] = x0.w;
+          xv[j][4] = x1.x; xv[j][5] = x1.y; xv[j][6] = x1.z; xv[j][7] = x1.w;
         }
-        // A's 32 x k rows -> B rows p KN + s (part p of column s of A), channels 8u .. 8u + 7;
-        // columns s >= k are 0
+        // B rows p KN + s (part p of column s of A), channels 8u .. 8u + 7; columns s >= k are 0
         const float* araw = reinterpret_cast<const float*>(rp + PL::araw_off);
-        for (int c = ct; c < KN * (PT_BK / 8); c += NT) {
-          const int sc = c % KN, u = c / KN;
-          float v[8];
+        constexpr int BPT = (KN * (PT_BK / 8) + NT - 1) / NT;
+        float av[BPT][8];
 #pragma unroll
-          for (int e = 0; e < 8; ++e) v[e] = sc < g.k ? araw[(8 * u + e) * g.k + sc] : 0.f;
-          uint4 h, m, lo;
-          split8(v, h, m, lo);
+        for (int j = 0; j < BPT; ++j) {
+          const int c = ct + j * NT;
+          const int sc = c % KN, u = c / KN;
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            av[j][e] = (c < KN * (PT_BK / 8) && sc < g.k) ? araw[(8 * u + e) * g.k + sc] : 0.f;
+        }
+        uint4 h[UPT], m[UPT], lo[UPT];
+#pragma unroll
+        for (int j = 0; j < UPT; ++j) split8(xv[j], h[j], m[j], lo[j]);
+        uint4 bh[BPT], bm[BPT], bl[BPT];
+#pragma unroll
+        for (int j = 0; j < BPT; ++j) split8(av[j], bh[j], bm[j], bl[j]);
+        // every raw value is consumed: the stage may be refilled
+        __syncwarp();
+        if (lane == 0) mbar_arrive(raw_empty(s));
+#pragma unroll
+        for (int j = 0; j < UPT; ++j) {
+          const uint32_t off = kmaj_chunk(r, u0 + j);
+          if (!LOCA_CHECK_SPAN(off, 16, PT_PART)) continue;
+          *reinterpret_cast<uint4*>(sp + off) = h[j];
+          *reinterpret_cast<uint4*>(sp + PT_PART + off) = m[j];
+          *reinterpret_cast<uint4*>(sp + 2 * PT_PART + off) = lo[j];
+        }
+#pragma unroll
+        for (int j = 0; j < BPT; ++j) {
+          const int c = ct + j * NT;
+          if (c >= KN * (PT_BK / 8)) continue;
+          const int sc = c % KN, u = c / KN;
           const uint32_t o0 = kmaj_chunk(sc, u), o1 = kmaj_chunk(KN + sc, u), o2 = kmaj_chunk(2 * KN + sc, u);
           if (!LOCA_CHECK_SPAN(o2, 16, NB * PT_BK * 2)) continue;
-          *reinterpret_cast<uint4*>(sp + PL::b_off + o0) = h;
-          *reinterpret_cast<uint4*>(sp + PL::b_off + o1) = m;
-          *reinterpret_cast<uint4*>(sp + PL::b_off + o2) = lo;
+          *reinterpret_cast<uint4*>(sp + PL::b_off + o0) = bh[j];
+          *reinterpret_cast<uint4*>(sp + PL::b_off + o1) = bm[j];
+          *reinterpret_cast<uint4*>(sp + PL::b_off + o2) = bl[j];
         }
         fence_proxy_async_smem();  // the split tiles visible to the tensor cores
         __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(raw_empty(s));
-          mbar_arrive(split_full(b));
-        }
+        if (lane == 0) mbar_arrive(split_full(b));
       }
     }
   }

@@ -10,14 +10,15 @@
 //                 lines per request, not 32), then each thread forms a register block of
 //                 RPT rows x SPT columns of the product with A's slab (broadcast reads).  Bound: the
 //                 HBM read of Gram and Cross (8 d^2 bytes per block).
-// k_chol_solve    one thread block per (ridge candidate j, block l):
-//                 GA_l and CA_l summed over their nsplit partial products (fixed order),
-//                 G_l = A_l^T GA_l (k x k), lambda from the trace, Cholesky of G_l + lambda I in
-//                 fp64 in shared memory, then every row i of C_l = B_prev,l G_l + s_l CA_l
-//                 (s_l = cross_scale[l], or 1) is solved
-//                 by a forward and a back substitution:  B[j, l, i] = C_l[i] (G_l + lambda I)^-1.
-//                 k is padded to a compile-time size with an identity block (its solution
-//                 columns are zero), so each row's solve stays in registers.
+// k_chol_factor   one thread block per (ridge candidate j, block l): GA_l summed over its nsplit
+//                 partial products (fixed order), G_l = A_l^T GA_l (k x k), lambda from the trace,
+//                 Cholesky of G_l + lambda I in fp64 in shared memory; the fp32 factor, its
+//                 diagonal reciprocals and G_l go to a per-candidate record in the workspace.
+// k_chol_rows     one thread per row i of C_l = B_prev,l G_l + s_l CA_l (s_l = cross_scale[l], or 1),
+//                 solved by a forward and a back substitution against the staged factor:
+//                 B[j, l, i] = C_l[i] (G_l + lambda I)^-1.  k is padded to a compile-time size with
+//                 an identity block (its solution columns are zero), so each row stays in registers;
+//                 d / 128 x nl x L thread blocks keep the SMs busy.
 #include "chol.cuh"
 #include "loca_internal.h"
 
@@ -137,19 +138,81 @@ __global__ void __launch_bounds__(PR_THREADS, KM <= 16 ? 3 : 1) k_project_rows(c
 }
 
 constexpr int CS_THREADS = 256;
-constexpr int CS_ROWS = 64;  // rows of A / GA staged per step when forming G
+
+// Partial G_l = A_l^T GA_l over one chunk of rows: grid (nch, L); rows staged 128 at a time;
+// a thread owns a 2 x 2 block of entries (KM = 32) or one entry (KM <= 16), fp32 over the chunk.
+constexpr int GP_THREADS = 256;
+constexpr int GP_ROWS = 128;
+constexpr int GP_MAX_CHUNKS = 32;
 
 template <int KM>
-__global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
-    const float* __restrict__ GA, const float* __restrict__ CA, int nsplit, const float* __restrict__ A,
-    const float* __restrict__ B_prev, const double* __restrict__ xsq_total, const float* __restrict__ cross_scale,
+__global__ void __launch_bounds__(GP_THREADS) k_chol_gram(const float* __restrict__ GA, int nsplit,
+                                                          const float* __restrict__ A, int64_t d, int k, int L,
+                                                          float* __restrict__ gpart) {
+  __shared__ __align__(16) float As[GP_ROWS][KM];
+  __shared__ __align__(16) float Gs[GP_ROWS][KM];
+  const int ch = blockIdx.x, l = blockIdx.y, nch = gridDim.x, tid = threadIdx.x;
+  const int64_t per = (d + nch - 1) / nch;
+  const int64_t r0 = int64_t(ch) * per, r1 = r0 + per < d ? r0 + per : d;
+  const float* Al = A + int64_t(l) * d * k;
+  const float* GAl = GA + int64_t(l) * d * k;
+  const int64_t zs = int64_t(L) * d * k;  // stride between the nsplit partial products
+  constexpr bool kBlk = KM == 32;
+  const int a0 = kBlk ? (tid / 16) * 2 : tid / KM, b0 = kBlk ? (tid % 16) * 2 : tid % KM;
+  const bool act = kBlk || tid < KM * KM;
+  float g00 = 0.f, g01 = 0.f, g10 = 0.f, g11 = 0.f;
+  for (int64_t i0 = r0; i0 < r1; i0 += GP_ROWS) {
+    __syncthreads();
+    for (int e = tid; e < GP_ROWS * KM; e += GP_THREADS) {
+      const int ii = e / KM, s2 = e % KM;
+      const bool ok = (i0 + ii < r1) && s2 < k && LOCA_CHECK((i0 + ii) * k + s2, d * k);
+      As[ii][s2] = ok ? Al[(i0 + ii) * k + s2] : 0.f;
+      float gsum = 0.f;
+      if (ok)
+        for (int z = 0; z < nsplit; ++z) gsum += GAl[z * zs + (i0 + ii) * k + s2];
+      Gs[ii][s2] = gsum;
+    }
+    __syncthreads();
+    if (act) {
+      if constexpr (kBlk) {
+#pragma unroll 8
+        for (int ii = 0; ii < GP_ROWS; ++ii) {
+          const float2 av = *reinterpret_cast<const float2*>(&As[ii][a0]);
+          const float2 gv = *reinterpret_cast<const float2*>(&Gs[ii][b0]);
+          g00 = fmaf(av.x, gv.x, g00);
+          g01 = fmaf(av.x, gv.y, g01);
+          g10 = fmaf(av.y, gv.x, g10);
+          g11 = fmaf(av.y, gv.y, g11);
+        }
+      } else {
+#pragma unroll 8
+        for (int ii = 0; ii < GP_ROWS; ++ii) g00 = fmaf(As[ii][a0], Gs[ii][b0], g00);
+      }
+    }
+  }
+  float* out = gpart + (int64_t(l) * nch + ch) * KM * KM;
+  if (kBlk) {
+    out[a0 * KM + b0] = g00;
+    out[a0 * KM + b0 + 1] = g01;
+    out[(a0 + 1) * KM + b0] = g10;
+    out[(a0 + 1) * KM + b0 + 1] = g11;
+  } else if (act) {
+    out[a0 * KM + b0] = g00;
+  }
+}
+
+// Per-candidate factor record in the workspace: Lf (KM x KM fp32 lower factor), Linv (KM), and
+// G_l (KM x KM fp32, symmetrised) for the B_prev term of the rows.
+template <int KM>
+__host__ __device__ constexpr int fac_floats() { return 2 * KM * KM + KM; }
+
+template <int KM>
+__global__ void __launch_bounds__(CS_THREADS) k_chol_factor(
+    const float* __restrict__ gpart, int nch, const double* __restrict__ xsq_total,
     int64_t d, int k, int L,
     float l0, float l1, float l2, float l3, float l4, float l5, float l6, float l7, float l8,
     float l9, float l10, float l11, float l12, float l13, float l14, float l15,
-    float* __restrict__ B, int32_t* __restrict__ info, float* __restrict__ G_out,
-    float* __restrict__ C_out) {
-  __shared__ float As[CS_ROWS][KM];
-  __shared__ float Gs[CS_ROWS][KM];
+    int32_t* __restrict__ info, float* __restrict__ G_out, float* __restrict__ fac) {
   __shared__ float Gf[KM][KM];   // G_l (fp32, symmetrised), padded with identity
   __shared__ double Md[KM][KM];  // G_l + lambda I, then its Cholesky factor (lower)
   __shared__ float Lf[KM][KM];
@@ -157,43 +220,12 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
   __shared__ int s_info;
   const int j = blockIdx.x, l = blockIdx.y;
   const float lam_rel[16] = {l0, l1, l2, l3, l4, l5, l6, l7, l8, l9, l10, l11, l12, l13, l14, l15};
-  const float* Al = A + int64_t(l) * d * k;
-  const float* GAl = GA + int64_t(l) * d * k;
-  const float* CAl = CA + int64_t(l) * d * k;
-  const int64_t zs = int64_t(L) * d * k;  // stride between the nsplit partial products
-
-  // G_l = A_l^T GA_l: thread owns entries e = t, t + 256, ... of the KM x KM matrix
-  constexpr int PER = (KM * KM + CS_THREADS - 1) / CS_THREADS;
-  float g[PER];
-#pragma unroll
-  for (int p = 0; p < PER; ++p) g[p] = 0.f;
-  for (int64_t i0 = 0; i0 < d; i0 += CS_ROWS) {
-    __syncthreads();
-    for (int e = threadIdx.x; e < CS_ROWS * KM; e += CS_THREADS) {
-      const int ii = e / KM, s = e % KM;
-      const bool ok = (i0 + ii < d) && s < k && LOCA_CHECK((i0 + ii) * k + s, d * k);
-      As[ii][s] = ok ? Al[(i0 + ii) * k + s] : 0.f;
-      float gsum = 0.f;
-      if (ok)
-        for (int z = 0; z < nsplit; ++z) gsum += GAl[z * zs + (i0 + ii) * k + s];
-      Gs[ii][s] = gsum;
-    }
-    __syncthreads();
-#pragma unroll
-    for (int p = 0; p < PER; ++p) {
-      const int e = threadIdx.x + p * CS_THREADS;
-      if (e < KM * KM) {
-        const int a = e / KM, b = e % KM;
-        float acc = g[p];
-        for (int ii = 0; ii < CS_ROWS; ++ii) acc = fmaf(As[ii][a], Gs[ii][b], acc);
-        g[p] = acc;
-      }
-    }
-  }
-#pragma unroll
-  for (int p = 0; p < PER; ++p) {
-    const int e = threadIdx.x + p * CS_THREADS;
-    if (e < KM * KM) Gf[e / KM][e % KM] = g[p];
+  // G_l = A_l^T GA_l from the row chunks' partial products, summed in a fixed order in fp64
+  const float* gp = gpart + int64_t(l) * nch * KM * KM;
+  for (int e = threadIdx.x; e < KM * KM; e += CS_THREADS) {
+    double acc = 0.0;
+    for (int c = 0; c < nch; ++c) acc += double(gp[int64_t(c) * KM * KM + e]);
+    Gf[e / KM][e % KM] = float(acc);
   }
   __syncthreads();
   const double lam =
@@ -220,124 +252,82 @@ __global__ void __launch_bounds__(CS_THREADS) k_chol_solve(
   const int inf = chol_factor<KM>(Md, Lf, Linv, &s_info);
   if (threadIdx.x == 0 && LOCA_CHECK(int64_t(j) * L + l, int64_t(gridDim.x) * L)) info[int64_t(j) * L + l] = inf;
 
-  float* Bj = B + (int64_t(j) * L + l) * d * k;
-  const float* Bp = B_prev ? B_prev + int64_t(l) * d * k : nullptr;
+  float* f = fac + (int64_t(j) * L + l) * fac_floats<KM>();
+  for (int e = threadIdx.x; e < KM * KM; e += CS_THREADS) {
+    const int a = e / KM, b = e % KM;
+    f[e] = Lf[a][b];
+    f[KM * KM + KM + e] = (a < k && b < k) ? float(0.5 * (double(Gf[a][b]) + double(Gf[b][a]))) : 0.f;
+  }
+  for (int a = threadIdx.x; a < KM; a += CS_THREADS) f[KM * KM + a] = Linv[a];
+}
+
+// Rows of B for one (ridge candidate j, block l): thread per row i,
+//   c = s_l CA_l[i] (+ B_prev,l[i] G_l),  B[j, l, i] = c (L L^T)^-1
+// with the candidate's factor staged in shared memory (broadcast reads); C_out = c for j = 0.
+constexpr int CR_THREADS = 128;
+
+template <int KM>
+__global__ void __launch_bounds__(CR_THREADS) k_chol_rows(
+    const float* __restrict__ CA, int nsplit, const float* __restrict__ B_prev, const float* __restrict__ cross_scale,
+    int64_t d, int k, int L, const int32_t* __restrict__ info, const float* __restrict__ fac, float* __restrict__ B,
+    float* __restrict__ C_out) {
+  __shared__ float Lf[KM][KM];
+  __shared__ float Linv[KM];
+  __shared__ float Gf[KM][KM];
+  const int j = blockIdx.y, l = blockIdx.z;
+  const float* f = fac + (int64_t(j) * L + l) * fac_floats<KM>();
+  for (int e = threadIdx.x; e < KM * KM; e += CR_THREADS) {
+    Lf[e / KM][e % KM] = f[e];
+    Gf[e / KM][e % KM] = f[KM * KM + KM + e];
+  }
+  for (int a = threadIdx.x; a < KM; a += CR_THREADS) Linv[a] = f[KM * KM + a];
+  __syncthreads();
+  const int inf = info[int64_t(j) * L + l];
+  const int64_t zs = int64_t(L) * d * k;  // stride between the nsplit partial products
   const float cs = cross_scale != nullptr ? cross_scale[l] : 1.f;
-  if constexpr (KM == 32) {
-    // one warp per row, lane s holding entry s: 32 values per thread do not fit in registers
-    // next to the unrolled substitutions, so they move between lanes by shuffles instead
-    __shared__ float Lp[KM][KM + 1];  // Lf with a padded row: column reads without bank conflicts
-    for (int e = threadIdx.x; e < KM * KM; e += CS_THREADS) Lp[e / KM][e % KM] = Lf[e / KM][e % KM];
-    __syncthreads();
-    const int lane = threadIdx.x & 31;
-    const bool on = lane < k;
-    constexpr int RW = 4;  // rows per warp at a time: four independent shuffle chains
-    for (int64_t i0 = int64_t(threadIdx.x >> 5) * RW; i0 < d; i0 += (CS_THREADS / 32) * RW) {
-      float c[RW];
+  float* Bj = B + (int64_t(j) * L + l) * d * k;
+  const int64_t i = int64_t(blockIdx.x) * CR_THREADS + threadIdx.x;
+  if (i >= d) return;
+  if (!LOCA_CHECK_SPAN((int64_t(l) * d + i) * k, k, int64_t(L) * d * k) ||
+      !LOCA_CHECK_SPAN((int64_t(j) * L + l) * d * k + i * k, k, int64_t(gridDim.y) * L * d * k))
+    return;
+  const float* cz = CA + (int64_t(l) * d + i) * k;
+  float c[KM];
 #pragma unroll
-      for (int r = 0; r < RW; ++r) {
-        const int64_t i = i0 + r;
-        float v = 0.f;
-        if (on && i < d)
-          for (int z = 0; z < nsplit; ++z) v += CAl[z * zs + i * k + lane];
-        c[r] = v * cs;
-      }
-      if (Bp != nullptr) {
-        float bl[RW];
+  for (int s2 = 0; s2 < KM; ++s2) c[s2] = 0.f;
+  for (int z = 0; z < nsplit; ++z) {
 #pragma unroll
-        for (int r = 0; r < RW; ++r) bl[r] = (on && i0 + r < d) ? Bp[(i0 + r) * k + lane] : 0.f;
+    for (int s2 = 0; s2 < KM; ++s2)
+      if (s2 < k) c[s2] += cz[z * zs + s2];
+  }
 #pragma unroll
-        for (int t = 0; t < KM; ++t) {
-          const float g = Gf[t][lane];
+  for (int s2 = 0; s2 < KM; ++s2) c[s2] *= cs;
+  if (B_prev != nullptr) {
+    // c += B_prev,l[i] G_l, one entry of the B_prev row at a time (only c stays in registers)
+    const float* bp = B_prev + (int64_t(l) * d + i) * k;
+#pragma unroll 4
+    for (int t = 0; t < k; ++t) {
+      const float bt = bp[t];
 #pragma unroll
-          for (int r = 0; r < RW; ++r) c[r] = fmaf(__shfl_sync(0xffffffffu, bl[r], t), g, c[r]);
-        }
-#pragma unroll
-        for (int r = 0; r < RW; ++r)
-          if (!on) c[r] = 0.f;
-      }
-      if (C_out != nullptr && j == 0 && on)
-#pragma unroll
-        for (int r = 0; r < RW; ++r)
-          if (i0 + r < d && LOCA_CHECK((int64_t(l) * d + i0 + r) * k + lane, int64_t(L) * d * k))
-            C_out[(int64_t(l) * d + i0 + r) * k + lane] = c[r];
-      if (inf != 0) {
-#pragma unroll
-        for (int r = 0; r < RW; ++r)
-          if (on && i0 + r < d) Bj[(i0 + r) * k + lane] = 0.f;
-        continue;
-      }
-      // c <- c (L L^T)^-1: forward L y = c^T, then L^T x = y
-#pragma unroll
-      for (int t = 0; t < KM; ++t) {
-        const float lt = Lp[lane][t], it = Linv[t];
-#pragma unroll
-        for (int r = 0; r < RW; ++r) {
-          if (lane == t) c[r] *= it;
-          const float yt = __shfl_sync(0xffffffffu, c[r], t);
-          if (lane > t) c[r] = fmaf(-lt, yt, c[r]);
-        }
-      }
-#pragma unroll
-      for (int t = KM - 1; t >= 0; --t) {
-        const float lt = Lp[t][lane], it = Linv[t];
-#pragma unroll
-        for (int r = 0; r < RW; ++r) {
-          if (lane == t) c[r] *= it;
-          const float xt = __shfl_sync(0xffffffffu, c[r], t);
-          if (lane < t) c[r] = fmaf(-lt, xt, c[r]);
-        }
-      }
-#pragma unroll
-      for (int r = 0; r < RW; ++r)
-        if (on && i0 + r < d && LOCA_CHECK((i0 + r) * k + lane, d * k)) Bj[(i0 + r) * k + lane] = c[r];
-    }
-  } else {
-    for (int64_t i = threadIdx.x; i < d; i += CS_THREADS) {
-      if (!LOCA_CHECK_SPAN(i * k, k, d * k) || !LOCA_CHECK_SPAN((int64_t(j) * L + l) * d * k + i * k, k,
-                                                               int64_t(gridDim.x) * L * d * k))
-        break;
-      float c[KM];
-#pragma unroll
-      for (int s = 0; s < KM; ++s) c[s] = 0.f;
-#pragma unroll 1
-      for (int z = 0; z < nsplit; ++z) {
-        const float* cz = CAl + z * zs + i * k;
-#pragma unroll
-        for (int s = 0; s < KM; ++s)
-          if (s < k) c[s] += cz[s];
-      }
-#pragma unroll
-      for (int s = 0; s < KM; ++s) c[s] *= cs;
-      if (Bp != nullptr) {
-        float b[KM];
-#pragma unroll
-        for (int s = 0; s < KM; ++s) b[s] = (s < k) ? Bp[i * k + s] : 0.f;
-#pragma unroll
-        for (int s = 0; s < KM; ++s) {
-          float a = c[s];
-#pragma unroll
-          for (int t = 0; t < KM; ++t) a = fmaf(b[t], Gf[t][s], a);
-          c[s] = (s < k) ? a : 0.f;
-        }
-      }
-      if (C_out != nullptr && j == 0 && LOCA_CHECK_SPAN((int64_t(l) * d + i) * k, k, int64_t(L) * d * k)) {
-#pragma unroll
-        for (int s = 0; s < KM; ++s)
-          if (s < k) C_out[(int64_t(l) * d + i) * k + s] = c[s];
-      }
-      if (inf != 0) {
-#pragma unroll
-        for (int s = 0; s < KM; ++s)
-          if (s < k) Bj[i * k + s] = 0.f;
-        continue;
-      }
-      chol_solve_row<KM>(Lf, Linv, c);
-#pragma unroll
-      for (int s = 0; s < KM; ++s)
-        if (s < k) Bj[i * k + s] = c[s];
+      for (int s2 = 0; s2 < KM; ++s2) c[s2] = fmaf(bt, Gf[t][s2], c[s2]);
     }
   }
+  if (C_out != nullptr && j == 0) {
+#pragma unroll
+    for (int s2 = 0; s2 < KM; ++s2)
+      if (s2 < k) C_out[(int64_t(l) * d + i) * k + s2] = c[s2];
+  }
+  float* bj = Bj + i * k;
+  if (inf != 0) {
+#pragma unroll
+    for (int s2 = 0; s2 < KM; ++s2)
+      if (s2 < k) bj[s2] = 0.f;
+    return;
+  }
+  chol_solve_row<KM>(Lf, Linv, c);
+#pragma unroll
+  for (int s2 = 0; s2 < KM; ++s2)
+    if (s2 < k) bj[s2] = c[s2];
 }
 
 template <int KM>
@@ -354,14 +344,27 @@ cudaError_t project_t(const float* gram, const float* cross, const float* A, int
 template <int KM>
 cudaError_t solve_t(const float* GA, const float* CA, int nsplit, const float* A, const float* B_prev,
                     const double* xsq_total, const float* cross_scale, const float* lr, int nl, int L,
-                    int64_t d, int k, float* B, int32_t* info, float* G_out, float* C_out, cudaStream_t s) {
+                    int64_t d, int k, float* B, int32_t* info, float* G_out, float* C_out, float* fac,
+                    cudaStream_t s) {
   float v[16] = {};
   for (int i = 0; i < nl && i < 16; ++i) v[i] = lr[i];
-  const dim3 grid = dim3(unsigned(nl), unsigned(L));
-  k_chol_solve<KM><<<grid, CS_THREADS, 0, s>>>(GA, CA, nsplit, A, B_prev, xsq_total, cross_scale, d, k, L, v[0], v[1],
-                                               v[2], v[3], v[4], v[5], v[6], v[7], v[8], v[9],
-                                               v[10], v[11], v[12], v[13], v[14], v[15], B, info,
-                                               G_out, C_out);
+  float* gpart = fac + size_t(16) * size_t(L) * size_t(fac_floats<32>());
+  int64_t nch = (int64_t(sm_count()) * 2 + L - 1) / L;  // two chunk CTAs per SM over the blocks
+  const int64_t maxch = (d + GP_ROWS - 1) / GP_ROWS;
+  if (nch > maxch) nch = maxch;
+  if (nch > GP_MAX_CHUNKS) nch = GP_MAX_CHUNKS;
+  if (nch < 1) nch = 1;
+  k_chol_gram<KM><<<dim3(unsigned(nch), unsigned(L)), GP_THREADS, 0, s>>>(GA, nsplit, A, d, k, L, gpart);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_chol_factor<KM><<<dim3(unsigned(nl), unsigned(L)), CS_THREADS, 0, s>>>(
+      gpart, int(nch), xsq_total, d, k, L, v[0], v[1], v[2], v[3], v[4], v[5], v[6], v[7], v[8], v[9], v[10], v[11],
+      v[12], v[13], v[14], v[15], info, G_out, fac);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const int64_t rows_per_cta = CR_THREADS;
+  const dim3 grid = dim3(unsigned((d + rows_per_cta - 1) / rows_per_cta), unsigned(nl), unsigned(L));
+  k_chol_rows<KM><<<grid, CR_THREADS, 0, s>>>(CA, nsplit, B_prev, cross_scale, d, k, L, info, fac, B, C_out);
   return cudaGetLastError();
 }
 
@@ -378,13 +381,17 @@ cudaError_t launch_project_rows(const float* gram, const float* cross, const flo
   return project_t<64>(gram, cross, A, L, d, k, GA, CA, s);
 }
 
+size_t chol_workspace_bytes(int L) {
+  return sizeof(float) * size_t(L) * (size_t(16) * size_t(fac_floats<32>()) + size_t(GP_MAX_CHUNKS) * 32 * 32);
+}
+
 cudaError_t launch_chol_solve(const float* GA, const float* CA, int nsplit, const float* A, const float* B_prev,
                               const double* xsq_total, const float* cross_scale, const float* lambda_rel,
                               int nl, int L, int64_t d, int k, float* B, int32_t* info, float* G_out,
-                              float* C_out, cudaStream_t s) {
+                              float* C_out, float* fac, cudaStream_t s) {
 #define LOCA_SOLVE(KM)                                                                               \
   return solve_t<KM>(GA, CA, nsplit, A, B_prev, xsq_total, cross_scale, lambda_rel, nl, L, d, k, B, info, G_out, \
-                     C_out, s)
+                     C_out, fac, s)
   if (k <= 4) LOCA_SOLVE(4);
   if (k <= 8) LOCA_SOLVE(8);
   if (k <= 16) LOCA_SOLVE(16);
