@@ -48,17 +48,21 @@ FALLBACK_SUSTAINED_TFLOPS = 1700.0  # profiling recipe's sustained figure, used 
 # kernel source whose sha256 prefix is given.  Work items and rounds repeat block by block, so
 # the traffic of a launch over L blocks is the capture's times L / L_capture; any other N, d or
 # k, or another source, reports null.
-GRAM_TC_TRAFFIC = {"sha256": "90572b4fced76acd", "L_capture": 2, "N": 131072, "d": 3584,
-                   "read": 8479111000, "write": 1260654000,
+GRAM_TC_TRAFFIC = {"sha256": "1a3b9dd1efc2f8ea", "L_capture": 2, "N": 131072, "d": 3584,
+                   "read": 8480182528, "write": 1255607296,
                    "kernel": "k_gram_cross_tc"}
 # k_kspace_xa (the k-space statistics kernel, which reads X) at k = 16
-KSPACE_TRAFFIC = {"sha256": "0000195dca10d804", "L_capture": 2, "N": 131072, "d": 3584, "k": 16,
-                  "read": 1885318656, "write": 2222848,
+KSPACE_TRAFFIC = {"sha256": "8b7bf4225f8fdb3f", "L_capture": 2, "N": 131072, "d": 3584, "k": 16,
+                  "read": 1885318912, "write": 2275840,
                   "kernel": "k_kspace_xa"}
 # k_targets_tc (writes T) at r = 16, bf16 output
-TARGETS_TRAFFIC = {"sha256": "c16a9c990782675b", "L_capture": 2, "N": 131072, "d": 3584, "r": 16,
-                   "read": 13240832, "write": 1819753728,
+TARGETS_TRAFFIC = {"sha256": "d957ddb952ff0eb1", "L_capture": 2, "N": 131072, "d": 3584, "r": 16,
+                   "read": 13251840, "write": 1816777984,
                    "kernel": "k_targets_tc"}
+# k_project_tc (the ridge solve's projection, which reads Gram and Cross once) at k = 16
+PROJECT_TRAFFIC = {"sha256": "218f1d3db838dccb", "L_capture": 2, "d": 3584, "k": 16,
+                   "read": 206018560, "write": 1268992,
+                   "kernel": "k_project_tc"}
 
 
 def recorded_traffic(rec, source_file, L, **shape):
@@ -431,7 +435,7 @@ def measure_workload(lc, name, dev, stream, steps, warmup, peak, hbm, wpeak):
     out["targets_roofline"] = hbm_object(L * N * d * T.element_size(), stages["targets"], "k_targets_tc", hbm,
                                          wpeak)
     out["ridge_solve_roofline"] = hbm_object(2 * L * d * d * 4, stages["ridge_solve"],
-                                             "k_project_tc + k_chol_solve (reads of Gram and cross)", hbm)
+                                             "k_project_tc + k_chol_gram, k_chol_factor, k_chol_rows (reads of Gram and cross)", hbm)
     del inp, X, z, T, gram, cross, E, ce, B
     torch.cuda.synchronize()
     torch.cuda.empty_cache()
@@ -573,7 +577,9 @@ def main():
     targets_roofline = hbm_object(L * N * d * T.element_size(), stages["targets"], "k_targets_tc", hbm, wpeak)
     targets_roofline["traffic"] = recorded_traffic(TARGETS_TRAFFIC, "targets.cu", L, N=N, d=d, r=r)
     solve_roofline = hbm_object(2 * L * d * d * 4, stages["ridge_solve"],
-                                "k_project_tc + k_chol_solve (reads of Gram and cross)", hbm)
+                                "k_project_tc + k_chol_gram, k_chol_factor, k_chol_rows (reads of Gram and cross)", hbm)
+    solve_roofline["traffic"] = recorded_traffic(PROJECT_TRAFFIC, "project_tc.cu", L, d=d, k=k)
+    solve_roofline["traffic_kernel"] = "k_project_tc"
 
     # the paper's own k-space statistics on the same inputs (no T, no d x d statistics):
     # error -> k-space accumulate (X A_l on the tensor cores, one HBM read of X) -> k-space solve
