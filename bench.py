@@ -86,6 +86,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-kspace", action="store_true", help="skip the k-space statistics measurement")
     ap.add_argument("--no-vocab", action="store_true", help="skip the wide-vocabulary head-error measurement")
+    ap.add_argument("--vocab-N", type=int, default=None,
+                    help="token count of the wide-vocabulary head-error leg (default: the 14B workload's 131072)")
     ap.add_argument("--no-calib", action="store_true", help="skip the one-shot d-wide feedback-fit measurement")
     ap.add_argument("--e2e-group", type=int, default=2, help="blocks per host-to-device copy in the e2e leg")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -696,6 +698,8 @@ def main():
     vocab = None
     if not args.no_vocab and world == 1:
         wv = S.WORKLOADS["qwen2.5-14b"]
+        if args.vocab_N is not None:
+            wv = S.scaled(wv, L=wv.L, N=args.vocab_N)
         gen = torch.Generator(device=dev)
         gen.manual_seed(1234)
         zv = torch.empty((wv.N, wv.V), dtype=torch.bfloat16, device=dev)
