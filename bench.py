@@ -93,6 +93,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-configs", action="store_true", help="skip the other workloads' own-shape measurements")
     ap.add_argument("--no-fused", action="store_true", help="skip the fused-targets pass")
+    ap.add_argument("--ridge-only", action="store_true",
+                    help="time loca_ridge_solve alone on seeded statistics of the workload's shape (for profiling)")
     return ap.parse_args()
 
 
@@ -450,6 +452,41 @@ def V_bytes(z):
 
 # ----------------------------------------------------------------------------- GPU arm
 
+def run_ridge_only(args, w, lc, dev):
+    """loca_ridge_solve alone at the workload's shape: seeded statistics (a Gram stand-in with a
+    dominant diagonal, a dense cross product), W untimed and K timed calls on one stream; one JSON
+    line.  The ridge solve's kernels run exactly as inside the step."""
+    import torch
+
+    L, d, k = w.L, w.d, w.k
+    g = torch.Generator(device=dev)
+    g.manual_seed(5)
+    gram = torch.randn((L, d, d), generator=g, device=dev)
+    gram += float(d) * torch.eye(d, device=dev)
+    cross = torch.randn((L, d, d), generator=g, device=dev)
+    A = torch.randn((L, d, k), generator=g, device=dev) / float(d) ** 0.5
+    nl = len(w.lambda_rel)
+    B = torch.empty((nl, L, d, k), device=dev)
+    info = torch.empty((nl, L), dtype=torch.int32, device=dev)
+    xs = torch.full((L,), float(d) * d, dtype=torch.float64, device=dev)
+    ws = torch.empty(lc.ridge_solve_workspace_size(L, d, k), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        lc.loca_ridge_solve(gram, cross, A, w.lambda_rel, B, info, xsq_total=xs, workspace=ws, stream=stream)
+    torch.cuda.synchronize()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(args.steps):
+        lc.loca_ridge_solve(gram, cross, A, w.lambda_rel, B, info, xsq_total=xs, workspace=ws, stream=stream)
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / args.steps
+    byts = 2.0 * L * d * d * 4
+    print(json.dumps({"ridge_only": w.name, "L": L, "d": d, "k": k, "nl": nl, "ms": ms,
+                      "gbs_of_statistics": byts / (ms / 1e3) / 1e9, "status": lc.loca_device_status()}))
+
+
 def main():
     args = parse()
     from synth import inputs as S
@@ -482,6 +519,9 @@ def main():
 
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
+    if args.ridge_only:
+        run_ridge_only(args, w, lc, dev)
+        return
     inp = S.device_inputs(w, seed=rank, device=dev)
     X, z, y, cols, P, Q, A = (inp[k] for k in ("X", "z", "y", "label_cols", "P", "Q", "A"))
     L, N, d, C, r, k = w.L, w.N, w.d, w.C, w.r, w.k
