@@ -77,8 +77,9 @@ int loca_version(void);
  * when one runs out the kernel records LOCA_ERR_TIMEOUT in the device status word, makes the
  * other waits of its launch give up, lets the copies and MMAs already in flight land, frees its
  * tensor memory and returns, so the context stays usable.  This sets, for the whole process,
- * how long such a wait may take in the tensor-core kernels (loca_targets, loca_kspace_accumulate
- * and the CTA-pair Gram / cross kernel of loca_gram_cross, loca_accumulate and their variants)
+ * how long such a wait may take in the tensor-core kernels (loca_targets, loca_kspace_accumulate,
+ * the CTA-pair Gram / cross kernel of loca_gram_cross, loca_accumulate and their variants, and the
+ * projection of loca_ridge_solve)
  * before it gives up: ns = 0 restores the default of 4 s; a tiny value makes a call time out on
  * purpose, to test that path.
  */
@@ -390,6 +391,11 @@ int loca_step_from_gram(const float* gram, int32_t L, int64_t d, const double* t
  *               the p-th pivot of G_l + lam I is not positive (B[j, l] is then zero)
  * G_out         L x k x k float output or NULL;  C_out  L x d x k float output or NULL
  * 1 <= k <= min(d, 32); 1 <= nl <= 16.
+ * The products gram_l A_l and cross_l A_l run on the tensor cores (an exact three-way bf16 split
+ * of each operand, so every product is exact in fp32; fp32 sums) when d and k are multiples of 4
+ * and gram, cross and A are 16-byte aligned, else on the CUDA cores in fp32.  The tensor-core
+ * path's waits are bounded (loca_set_wait_limit); one that gives up writes LOCA_ERR_TIMEOUT to
+ * the device status word and leaves B undefined.
  */
 int loca_ridge_solve_workspace_size(int32_t L, int64_t d, int32_t k, size_t* bytes /* host */);
 int loca_ridge_solve(const float* gram, const float* cross, const float* cross_scale,

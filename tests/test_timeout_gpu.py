@@ -2,7 +2,7 @@
 
 A wait limit of 1 microsecond (the loca_set_wait_limit test hook) makes the first wait of the
 tensor-core kernels (targets, k-space statistics, the CTA-pair Gram / cross kernel with and
-without generated targets) that does not
+without generated targets, the ridge solve's projection) that does not
 succeed at once give up: the kernel must record
 LOCA_ERR_TIMEOUT in the device status word, let its copies and MMAs in flight land, free its
 tensor memory and return.  The CUDA context must stay usable: with the default limit restored,
@@ -69,6 +69,16 @@ def _fused_call(lc, X, E, P, Q):
     return gram, cross
 
 
+def _ridge_call(lc, gram, cross, A):
+    L, d, _ = gram.shape
+    k = A.shape[2]
+    B = torch.empty((2, L, d, k), device="cuda")
+    info = torch.empty((2, L), dtype=torch.int32, device="cuda")
+    lc.loca_ridge_solve(gram, cross, A, [1e-3, 1e-2], B, info)
+    torch.cuda.synchronize()
+    return B, info
+
+
 def test_wait_timeout_is_reported_and_the_context_recovers(lc):
     g = torch.Generator(device="cuda")
     g.manual_seed(5)
@@ -85,8 +95,9 @@ def test_wait_timeout_is_reported_and_the_context_recovers(lc):
     ref_t = _targets_call(lc, E, P, Q, L, N, d)
     ref_g = _gram_call(lc, X, T)
     ref_f = _fused_call(lc, X, E, P, Q)
+    ref_r = _ridge_call(lc, ref_g[0], ref_g[1], A)
     assert lc.loca_device_status() == 0
-    for call in ("kspace", "targets", "gram", "fused"):
+    for call in ("kspace", "targets", "gram", "fused", "ridge"):
         lc.loca_set_wait_limit(1000)  # 1 us: a wait that does not succeed at once gives up
         if call == "kspace":
             _kspace_call(lc, X, A, E, P, Q)
@@ -97,15 +108,21 @@ def test_wait_timeout_is_reported_and_the_context_recovers(lc):
             # armed stage may never be issued, and every copy, MMA and bulk store still lands
             # before either CTA of a pair leaves
             _gram_call(lc, X, T)
-        else:
+        elif call == "fused":
             # the same kernel generating its targets: more roles (U producer, T conversion)
             _fused_call(lc, X, E, P, Q)
+        else:
+            # the tensor-core projection (d and k multiples of 4): producer, split groups, MMA
+            # and epilogue rings
+            _ridge_call(lc, ref_g[0], ref_g[1], A)
         assert lc.loca_device_status() == LOCA_ERR_TIMEOUT, call
         lc.loca_set_wait_limit(0)
         again_k = _kspace_call(lc, X, A, E, P, Q)
         again_t = _targets_call(lc, E, P, Q, L, N, d)
         again_g = _gram_call(lc, X, T)
         again_f = _fused_call(lc, X, E, P, Q)
+        again_r = _ridge_call(lc, ref_g[0], ref_g[1], A)
         assert lc.loca_device_status() == 0, call
-        for a, b in zip(ref_k + ref_t + ref_g + ref_f, again_k + again_t + again_g + again_f):
+        for a, b in zip(ref_k + ref_t + ref_g + ref_f + ref_r,
+                        again_k + again_t + again_g + again_f + again_r):
             assert torch.equal(a, b), call
