@@ -385,6 +385,8 @@ def test_ridge_solve_parity(lc, k, d, L, with_prev, relative):
     (16, 3584, 2),   # the 7B width: tensor-core projection, 28 row tiles and 112 K-slabs per matrix
     (32, 5120, 1),   # the 14B width (k = 32)
     (12, 1000, 2),   # k padded to 16, a ragged last row tile (104 rows) and a ragged last K-slab
+    (20, 640, 3),    # k padded to 32 (N = 96 with zero columns), five row tiles per matrix
+    (28, 1152, 1),   # k padded to 32, nine row tiles, 36 K-slabs
     (6, 330, 2),     # k % 4 != 0 and d % 4 != 0: the SIMT projection
 ])
 def test_ridge_solve_parity_at_full_width(lc, k, d, L):
