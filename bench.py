@@ -60,7 +60,7 @@ TARGETS_TRAFFIC = {"sha256": "d957ddb952ff0eb1", "L_capture": 2, "N": 131072, "d
                    "read": 13251840, "write": 1816777984,
                    "kernel": "k_targets_tc"}
 # k_project_tc (the ridge solve's projection, which reads Gram and Cross once) at k = 16
-PROJECT_TRAFFIC = {"sha256": "218f1d3db838dccb", "L_capture": 2, "d": 3584, "k": 16,
+PROJECT_TRAFFIC = {"sha256": "d07a68c14390f068", "L_capture": 2, "d": 3584, "k": 16,
                    "read": 206018560, "write": 1268992,
                    "kernel": "k_project_tc"}
 

@@ -20,11 +20,12 @@
 // Persistent, one CTA per SM, 448 threads, three rings so that no role waits on another's latency:
 //   warp 0      TMA producer: per K-slab a 128 x 32 fp32 tile of the matrix (128-byte swizzle) and
 //               the 32 x k rows of A_l (plain) into a raw stage (PT_RAW stages).
-//   warps 6-13  split a raw stage into a split buffer (PT_SPLIT buffers): the tile's hi / mid / lo
-//               bf16 parts and A's slab parts, all K-major without swizzle (8-row x 16-byte core
-//               matrices); the raw stage is released as soon as its values are in registers.  A
-//               stage's MMAs free its split buffer, so the split of stage t waits for the MMAs of
-//               stage t - PT_SPLIT: the buffers, not the TMA ring, set the loop that bounds the rate.
+//   warps 6-13  two groups of four taking turns over the stages: split a raw stage into a split
+//               buffer (PT_SPLIT buffers, two per group): the tile's hi / mid / lo bf16 parts and
+//               A's slab parts, all K-major without swizzle (8-row x 16-byte core matrices); the
+//               raw stage is released as soon as its values are in registers.  A stage's MMAs
+//               free its split buffer, so the split of stage t waits for the MMAs of stage
+//               t - PT_SPLIT: this loop, not the TMA ring, bounds the rate.
 //   warp 1      owns the TMEM accumulators (PT_ACC of 128 lanes x 3 KN columns) and issues the
 //               MMAs (kind::f16, M = 128, N = 3 KN, K = 16), one accumulator per K-slab.
 //   warps 2-5   read each slab's accumulator (TMEM lane quarter warp % 4), add its three column
