@@ -62,6 +62,7 @@ ERROR_CASES = [
     ("pitch_f32", 257, 130, 2, "f32", 0, 6, False),
     ("vocab_row_bf16", 48, 151936, 4, "bf16", 0, 0, True),
     ("single_class", 64, 64, 1, "f32", 0, 0, False),
+    ("wide_labels_bf16", 300, 4096, 64, "bf16", 0, 0, True),
 ]
 
 
@@ -113,6 +114,8 @@ def test_error_parity(lc, case):
     ("f32", 1, 5000, 264, 5, 12),
     ("bf16", 1, 4100, 120, 3, 3),
     ("bf16", 2, 3000, 960, 2, 8),
+    ("bf16", 1, 2000, 256, 64, 32),  # the kernel's limits: C = 64 label columns, r = 32
+    ("f32", 1, 700, 136, 64, 31),
 ])
 def test_targets_parity(lc, tdt, L, N, d, C, r):
     """S3 / S11.  Each output is an fp32 dot product of length r after an fp32 product of length C:
