@@ -48,8 +48,8 @@ FALLBACK_SUSTAINED_TFLOPS = 1700.0  # profiling recipe's sustained figure, used 
 # kernel source whose sha256 prefix is given.  Work items and rounds repeat block by block, so
 # the traffic of a launch over L blocks is the capture's times L / L_capture; any other N, d or
 # k, or another source, reports null.
-GRAM_TC_TRAFFIC = {"sha256": "1a3b9dd1efc2f8ea", "L_capture": 2, "N": 131072, "d": 3584,
-                   "read": 8480182528, "write": 1255607296,
+GRAM_TC_TRAFFIC = {"sha256": "81575fe3750817bb", "L_capture": 2, "N": 131072, "d": 3584,
+                   "read": 8478698496, "write": 1255207936,
                    "kernel": "k_gram_cross_tc"}
 # k_kspace_xa (the k-space statistics kernel, which reads X) at k = 16
 KSPACE_TRAFFIC = {"sha256": "8b7bf4225f8fdb3f", "L_capture": 2, "N": 131072, "d": 3584, "k": 16,

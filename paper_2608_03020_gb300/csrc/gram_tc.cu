@@ -865,9 +865,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Cfg<kFused>::kThread
 }
 
 // Lower triangle of every Gram_l from its upper triangle: element (i, j), i > j, becomes (j, i).
-// One 32 x 32 tile (bi, bj), bi >= bj, per CTA (256 threads), through a padded shared tile.
+// One 64 x 64 tile (bi, bj), bi >= bj, per CTA (256 threads) through a padded shared tile; rows are
+// read and written as 16-byte vectors when d % 4 == 0 (each thread moves 4 consecutive columns).
+constexpr int MIR_T = 64;
+
 __global__ void __launch_bounds__(256) k_gram_mirror(float* __restrict__ gram, int d, int nt) {
-  __shared__ float tile[32][33];
+  __shared__ float tile[MIR_T][MIR_T + 1];
   const int l = blockIdx.y;
   // triangular index t = bi (bi + 1) / 2 + bj, 0 <= bj <= bi < nt
   const int t = blockIdx.x;
@@ -877,15 +880,34 @@ __global__ void __launch_bounds__(256) k_gram_mirror(float* __restrict__ gram, i
   const int bj = t - bi * (bi + 1) / 2;
   (void)nt;
   float* G = gram + int64_t(l) * d * d;
-  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
-  for (int r = ty; r < 32; r += 8) {  // source rows j of the upper tile (bj, bi)
-    const int i = bj * 32 + r, j = bi * 32 + tx;
-    if (i < d && j < d && LOCA_CHECK(int64_t(i) * d + j, int64_t(d) * d)) tile[r][tx] = G[int64_t(i) * d + j];
+  const bool vec = (d & 3) == 0;
+  const int tc4 = (threadIdx.x & 15) * 4, ty = threadIdx.x >> 4;  // 4 columns, 16 rows per pass
+  for (int r = ty; r < MIR_T; r += 16) {  // source rows of the upper tile (bj, bi)
+    const int i = bj * MIR_T + r, j = bi * MIR_T + tc4;
+    if (i >= d) continue;
+    if (vec && j + 3 < d && LOCA_CHECK_SPAN(int64_t(i) * d + j, 4, int64_t(d) * d)) {
+      const float4 v = *reinterpret_cast<const float4*>(G + int64_t(i) * d + j);
+      tile[r][tc4] = v.x;
+      tile[r][tc4 + 1] = v.y;
+      tile[r][tc4 + 2] = v.z;
+      tile[r][tc4 + 3] = v.w;
+    } else {
+      for (int q = 0; q < 4; ++q)
+        if (j + q < d && LOCA_CHECK(int64_t(i) * d + j + q, int64_t(d) * d)) tile[r][tc4 + q] = G[int64_t(i) * d + j + q];
+    }
   }
   __syncthreads();
-  for (int r = ty; r < 32; r += 8) {
-    const int i = bi * 32 + r, j = bj * 32 + tx;
-    if (i < d && j < d && i > j && LOCA_CHECK(int64_t(i) * d + j, int64_t(d) * d)) G[int64_t(i) * d + j] = tile[tx][r];
+  for (int r = ty; r < MIR_T; r += 16) {  // destination rows of the lower tile (bi, bj)
+    const int i = bi * MIR_T + r, j = bj * MIR_T + tc4;
+    if (i >= d) continue;
+    const float4 v = make_float4(tile[tc4][r], tile[tc4 + 1][r], tile[tc4 + 2][r], tile[tc4 + 3][r]);
+    if (vec && bi > bj && j + 3 < d && LOCA_CHECK_SPAN(int64_t(i) * d + j, 4, int64_t(d) * d)) {
+      *reinterpret_cast<float4*>(G + int64_t(i) * d + j) = v;  // off the diagonal: all i > j
+    } else {
+      const float vv[4] = {v.x, v.y, v.z, v.w};
+      for (int q = 0; q < 4; ++q)
+        if (j + q < d && i > j + q && LOCA_CHECK(int64_t(i) * d + j + q, int64_t(d) * d)) G[int64_t(i) * d + j + q] = vv[q];
+    }
   }
 }
 
@@ -1002,7 +1024,7 @@ cudaError_t launch_stats(const void* X, const void* T, int L, int64_t N, int64_t
       reinterpret_cast<uint32_t*>(abort_flag + 1), wait_limit_ns(), sync_ns, fz);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  const int nt = int((d + 31) / 32);
+  const int nt = int((d + MIR_T - 1) / MIR_T);
   k_gram_mirror<<<dim3(unsigned(nt * (nt + 1) / 2), unsigned(L)), 256, 0, s>>>(gram, int(d), nt);
   return cudaGetLastError();
 }
