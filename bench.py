@@ -60,8 +60,8 @@ TARGETS_TRAFFIC = {"sha256": "d957ddb952ff0eb1", "L_capture": 2, "N": 131072, "d
                    "read": 13251840, "write": 1816777984,
                    "kernel": "k_targets_tc"}
 # k_project_tc (the ridge solve's projection, which reads Gram and Cross once) at k = 16
-PROJECT_TRAFFIC = {"sha256": "d07a68c14390f068", "L_capture": 2, "d": 3584, "k": 16,
-                   "read": 206018560, "write": 1268992,
+PROJECT_TRAFFIC = {"sha256": "d41e4a5ac19fe01d", "L_capture": 2, "d": 3584, "k": 16,
+                   "read": 206007296, "write": 1507584,
                    "kernel": "k_project_tc"}
 
 

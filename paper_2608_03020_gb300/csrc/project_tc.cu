@@ -17,18 +17,21 @@
 // width, sets the MMA time: 6 MMAs per 16 KB slab, under the slab's HBM time.
 //
 // Work item = 128 rows of the stacked [Gram_l; Cross_l] (2 d rows per block) over all d columns.
-// Persistent, one CTA per SM, 448 threads, three rings so that no role waits on another's latency:
+// Persistent, one CTA per SM, 512 threads, three rings so that no role waits on another's latency:
 //   warp 0      TMA producer: per K-slab a 128 x 32 fp32 tile of the matrix (128-byte swizzle) and
 //               the 32 x k rows of A_l (plain) into a raw stage (PT_RAW stages).
-//   warps 6-13  two groups of four taking turns over the stages: split a raw stage into a split
-//               buffer (PT_SPLIT buffers, two per group): the tile's hi / mid / lo bf16 parts and
-//               A's slab parts, all K-major without swizzle (8-row x 16-byte core matrices); the
-//               raw stage is released as soon as its values are in registers.  A stage's MMAs
-//               free its split buffer, so the split of stage t waits for the MMAs of stage
-//               t - PT_SPLIT: this loop, not the TMA ring, bounds the rate.
+//   split warps 8, 2, 3, 14 and 12, 10, 11, 15: two groups of four taking turns over the stages:
+//               split a raw stage into a split buffer (PT_SPLIT buffers, two per group): the
+//               tile's hi / mid / lo bf16 parts and A's slab parts, all K-major without swizzle
+//               (8-row x 16-byte core matrices); the raw stage is released as soon as its values
+//               are in registers.  A stage's MMAs free its split buffer, so the split of stage t
+//               waits for the MMAs of stage t - PT_SPLIT: this loop, not the TMA ring, bounds the
+//               rate.  No split warp shares the MMA warp's scheduler (warp % 4 == 1): issuing
+//               the MMAs takes about half of that scheduler's cycles, and a split warp there was
+//               the one that set the pace (warps 9 and 13 stay idle).
 //   warp 1      owns the TMEM accumulators (PT_ACC of 128 lanes x 3 KN columns) and issues the
 //               MMAs (kind::f16, M = 128, N = 3 KN, K = 16), one accumulator per K-slab.
-//   warps 2-5   read each slab's accumulator (TMEM lane quarter warp % 4), add its three column
+//   warps 4-7   read each slab's accumulator (TMEM lane quarter warp % 4), add its three column
 //               groups into their rows' fp32 sums, and write the rows at the end of the item.
 // All waits are bounded (tc_ptx.cuh); a wait that gives up sets the status word, the other roles
 // follow through the launch's abort flag, copies and MMAs in flight land before TMEM is freed.
@@ -44,7 +47,7 @@ namespace {
 
 using namespace tc;
 
-constexpr int PT_THREADS = 448;
+constexpr int PT_THREADS = 512;
 constexpr int PT_RAW = 5;     // raw stages (TMA in flight)
 constexpr int PT_SPLIT = 4;   // split buffers (MMA operands)
 constexpr int PT_ACC = 4;     // TMEM accumulators
@@ -234,8 +237,8 @@ __global__ void __launch_bounds__(PT_THREADS, 1)
       }
     }
     __syncwarp();
-  } else if (warp < 6) {
-    // ---------------- warps 2..5: each slab's three column groups into the rows' sums, then the rows
+  } else if (warp >= 4 && warp < 8) {
+    // ---------------- warps 4..7: each slab's three column groups into the rows' sums, then the rows
     const int q = warp & 3;  // TMEM lane quarter: rows q * 32 + lane of the item
     const uint32_t lane_base = uint32_t(q * 32) << 16;
     uint32_t t = 0;
@@ -290,11 +293,13 @@ __global__ void __launch_bounds__(PT_THREADS, 1)
             *reinterpret_cast<float4*>(out + s4) = make_float4(sum[s4], sum[s4 + 1], sum[s4 + 2], sum[s4 + 3]);
       }
     }
-  } else {
-    // ---------------- warps 6..13: split raw stages into split buffers (the groups take turns when
-    // there are several, so that one stage's split latency overlaps the next one's)
-    const int grp = (warp - 6) / PT_GROUP_WARPS;
-    const int ct = threadIdx.x - 6 * 32 - grp * PT_GROUP_WARPS * 32;  // thread within the group
+  } else if (warp != 9 && warp != 13) {
+    // ---------------- split warps (not on the MMA warp's scheduler): the groups take turns, so that
+    // one stage's split latency overlaps the next one's; each group has a warp on schedulers 0, 2, 3
+    const int cw = warp == 8 ? 0 : warp == 2 ? 1 : warp == 3 ? 2 : warp == 14 ? 3
+                 : warp == 12 ? 4 : warp == 10 ? 5 : warp == 11 ? 6 : 7;  // warp 15
+    const int grp = cw / PT_GROUP_WARPS;
+    const int ct = (cw % PT_GROUP_WARPS) * 32 + lane;  // thread within the group
     constexpr int NT = PT_GROUP_WARPS * 32;
     constexpr int UPT = PT_TM * (PT_BK / 8) / NT;  // 8-channel chunks of one row per thread
     static_assert(NT % PT_TM == 0 && UPT >= 1, "whole rows of chunks per thread");
