@@ -4,16 +4,19 @@
 //                 multiple of 4, unaligned pointers)
 //                 GA_l = Gram_l A_l, CA_l = Cross_l A_l (d x k each), as PR_SPLIT partial
 //                 products over quarters of the column range (GA = sum_z GA_z, summed in a fixed
-//                 order by k_chol_solve).  A CTA takes 256 rows of the stacked [Gram_l; Cross_l]
+//                 order by k_chol_gram and k_chol_rows).  A CTA takes 256 rows of the stacked [Gram_l; Cross_l]
 //                 and one column quarter; 32-column slabs of its rows are staged in shared memory
 //                 by row-contiguous 16-byte loads (a warp request covers 4 rows, so L1 sees 4
 //                 lines per request, not 32), then each thread forms a register block of
 //                 RPT rows x SPT columns of the product with A's slab (broadcast reads).  Bound: the
 //                 HBM read of Gram and Cross (8 d^2 bytes per block).
-// k_chol_factor   one thread block per (ridge candidate j, block l): GA_l summed over its nsplit
-//                 partial products (fixed order), G_l = A_l^T GA_l (k x k), lambda from the trace,
-//                 Cholesky of G_l + lambda I in fp64 in shared memory; the fp32 factor, its
-//                 diagonal reciprocals and G_l go to a per-candidate record in the workspace.
+// k_chol_gram     G_l = A_l^T GA_l (k x k) as partial sums over chunks of the d rows: grid
+//                 (chunks, L), GA_l summed over its nsplit partial products (fixed order) as the
+//                 rows are staged; each chunk's k x k partial sum goes to the workspace.
+// k_chol_factor   one thread block per (ridge candidate j, block l): the chunks' partial sums
+//                 added in chunk order, lambda from the trace, Cholesky of G_l + lambda I in fp64
+//                 in shared memory; the fp32 factor, its diagonal reciprocals and G_l go to a
+//                 per-candidate record in the workspace.
 // k_chol_rows     one thread per row i of C_l = B_prev,l G_l + s_l CA_l (s_l = cross_scale[l], or 1),
 //                 solved by a forward and a back substitution against the staged factor:
 //                 B[j, l, i] = C_l[i] (G_l + lambda I)^-1.  k is padded to a compile-time size with
