@@ -24,11 +24,13 @@
 //               split a raw stage into a split buffer (PT_SPLIT buffers, two per group): the
 //               tile's hi / mid / lo bf16 parts and A's slab parts, all K-major without swizzle
 //               (8-row x 16-byte core matrices); the raw stage is released as soon as its values
-//               are in registers.  A stage's MMAs free its split buffer, so the split of stage t
-//               waits for the MMAs of stage t - PT_SPLIT: this loop, not the TMA ring, bounds the
-//               rate.  No split warp shares the MMA warp's scheduler (warp % 4 == 1): issuing
-//               the MMAs takes about half of that scheduler's cycles, and a split warp there was
-//               the one that set the pace (warps 9 and 13 stay idle).
+//               are in registers.  PT_RAW is a multiple of the group count, so every use of a
+//               raw stage falls to the same group (each barrier phase a group waits for follows
+//               one it has seen).
+//               A stage's MMAs free its split buffer, so the split of stage t waits for the MMAs
+//               of stage t - PT_SPLIT.  No split warp shares the MMA warp's scheduler
+//               (warp % 4 == 1): issuing the MMAs takes about half of that scheduler's cycles,
+//               and a split warp there was the one that set the pace (warps 9 and 13 stay idle).
 //   warp 1      owns the TMEM accumulators (PT_ACC of 128 lanes x 3 KN columns) and issues the
 //               MMAs (kind::f16, M = 128, N = 3 KN, K = 16), one accumulator per K-slab.
 //   warps 4-7   read each slab's accumulator (TMEM lane quarter warp % 4), add its three column
@@ -48,13 +50,17 @@ namespace {
 using namespace tc;
 
 constexpr int PT_THREADS = 512;
-constexpr int PT_RAW = 5;     // raw stages (TMA in flight)
+constexpr int PT_RAW = 4;     // raw stages (TMA in flight)
 constexpr int PT_SPLIT = 4;   // split buffers (MMA operands)
 constexpr int PT_ACC = 4;     // TMEM accumulators
 constexpr int PT_CONV_WARPS = 8;
 constexpr int PT_GROUPS = 2;  // split groups: group g takes the stages t with t % PT_GROUPS == g
 constexpr int PT_GROUP_WARPS = PT_CONV_WARPS / PT_GROUPS;
 static_assert(PT_CONV_WARPS % PT_GROUPS == 0 && PT_SPLIT % PT_GROUPS == 0, "groups own whole split buffers");
+// Every use of a raw stage then falls to the same group, which takes its stages in order: an
+// mbarrier parity wait tells only consecutive phases apart, so with an odd count a group running
+// ahead could take the phase of the other group's earlier use (its copy still landing) for its own.
+static_assert(PT_RAW % PT_GROUPS == 0, "groups own whole raw stages");
 constexpr int PT_TM = 128;    // rows per work item (TMEM lanes)
 constexpr int PT_BK = 32;     // channels per K-slab (128 bytes of fp32: one swizzle row)
 constexpr uint32_t PT_TILE = PT_TM * PT_BK * 4;   // 16 KB fp32 tile
@@ -208,7 +214,8 @@ __global__ void __launch_bounds__(PT_THREADS, 1)
         for (int kb = 0; kb < g.nkb; ++kb, ++t) {
           const int b = int(t % PT_SPLIT);
           const int a = int(t % PT_ACC);
-          if (!mbar_wait(acc_empty(a), ((t / PT_ACC) & 1u) ^ 1u, wc)) { ok = false; break; }
+          const uint32_t pa = ((t / PT_ACC) & 1u) ^ 1u;
+          if (!mbar_try_wait(acc_empty(a), pa) && !mbar_wait(acc_empty(a), pa, wc)) { ok = false; break; }
           if (!mbar_try_wait(split_full(b), (t / PT_SPLIT) & 1u) &&
               !mbar_wait(split_full(b), (t / PT_SPLIT) & 1u, wc)) {
             ok = false;
@@ -251,7 +258,8 @@ __global__ void __launch_bounds__(PT_THREADS, 1)
       for (int i = 0; i < KN; ++i) sum[i] = 0.f;
       for (int kb = 0; kb < g.nkb; ++kb, ++t) {
         const int a = int(t % PT_ACC);
-        const bool w_ok = mbar_wait(acc_full(a), (t / PT_ACC) & 1u, wc);
+        const uint32_t pa = (t / PT_ACC) & 1u;
+        const bool w_ok = mbar_try_wait(acc_full(a), pa) || mbar_wait(acc_full(a), pa, wc);
         if (!__all_sync(0xffffffffu, w_ok)) {
           ok = false;
           break;
@@ -312,8 +320,11 @@ __global__ void __launch_bounds__(PT_THREADS, 1)
         if (int(t % PT_GROUPS) != grp) continue;
         const int s = int(t % PT_RAW);
         const int b = int(t % PT_SPLIT);
-        bool w_ok = mbar_wait(raw_full(s), (t / PT_RAW) & 1u, wc);
-        w_ok = w_ok && mbar_wait(split_empty(b), ((t / PT_SPLIT) & 1u) ^ 1u, wc);
+        // raw stage s: this group's stages only (PT_RAW % PT_GROUPS == 0), taken in order.  The
+        // bounded wait is a call (registers saved around it), so an inline try_wait goes first.
+        const uint32_t pr = (t / PT_RAW) & 1u, pb = ((t / PT_SPLIT) & 1u) ^ 1u;
+        bool w_ok = mbar_try_wait(raw_full(s), pr) || mbar_wait(raw_full(s), pr, wc);
+        w_ok = w_ok && (mbar_try_wait(split_empty(b), pb) || mbar_wait(split_empty(b), pb, wc));
         if (!__all_sync(0xffffffffu, w_ok)) {
           ok = false;
           break;
