@@ -52,16 +52,16 @@ GRAM_TC_TRAFFIC = {"sha256": "81575fe3750817bb", "L_capture": 2, "N": 131072, "d
                    "read": 8478698496, "write": 1255207936,
                    "kernel": "k_gram_cross_tc"}
 # k_kspace_xa (the k-space statistics kernel, which reads X) at k = 16
-KSPACE_TRAFFIC = {"sha256": "8b7bf4225f8fdb3f", "L_capture": 2, "N": 131072, "d": 3584, "k": 16,
-                  "read": 1885318912, "write": 2275840,
+KSPACE_TRAFFIC = {"sha256": "3aba9c60b10e48c0", "L_capture": 2, "N": 131072, "d": 3584, "k": 16,
+                  "read": 1885266176, "write": 2223872,
                   "kernel": "k_kspace_xa"}
 # k_targets_tc (writes T) at r = 16, bf16 output
-TARGETS_TRAFFIC = {"sha256": "d957ddb952ff0eb1", "L_capture": 2, "N": 131072, "d": 3584, "r": 16,
-                   "read": 13251840, "write": 1816777984,
+TARGETS_TRAFFIC = {"sha256": "1796bbc513a2c2d2", "L_capture": 2, "N": 131072, "d": 3584, "r": 16,
+                   "read": 13250816, "write": 1817000448,
                    "kernel": "k_targets_tc"}
 # k_project_tc (the ridge solve's projection, which reads Gram and Cross once) at k = 16
-PROJECT_TRAFFIC = {"sha256": "d41e4a5ac19fe01d", "L_capture": 2, "d": 3584, "k": 16,
-                   "read": 206007296, "write": 1507584,
+PROJECT_TRAFFIC = {"sha256": "ba847e501813d245", "L_capture": 2, "d": 3584, "k": 16,
+                   "read": 206016000, "write": 1437952,
                    "kernel": "k_project_tc"}
 
 

@@ -195,7 +195,10 @@ __global__ void __launch_bounds__(xa_threads(KP), 1)
       for (int it = blockIdx.x; it < total && ok; it += gridDim.x, ++tcount) {
         const int buf = int(tcount & 1u);
         const uint32_t aph = (tcount >> 1) & 1u;
-        if (!mbar_wait(acc_empty(buf), aph ^ 1u, wc)) { ok = false; break; }
+        if (!mbar_try_wait(acc_empty(buf), aph ^ 1u) && !mbar_wait(acc_empty(buf), aph ^ 1u, wc)) {
+          ok = false;
+          break;
+        }
         fence_after();
         const uint32_t dt = tmem_base + uint32_t(buf * NCOL);
         for (int kc = 0; kc < nkc; ++kc) {
@@ -250,7 +253,8 @@ __global__ void __launch_bounds__(xa_threads(KP), 1)
       }
       bool ok = true;
       for (int kc = 0; kc < nkc; ++kc) {
-        const bool w_ok = mbar_wait(full_bar(stage), phase, wc);
+        // the bounded wait is a call (registers saved around it): an inline try_wait goes first
+        const bool w_ok = mbar_try_wait(full_bar(stage), phase) || mbar_wait(full_bar(stage), phase, wc);
         if (!__all_sync(0xffffffffu, w_ok)) { ok = false; break; }
         // squares of the tokens' 64 channels: rows of the swizzled tile (chunk order is irrelevant
         // for a sum, so lane i starts at chunk i % 8 and the 32 lanes' 16-byte reads spread over
@@ -377,7 +381,8 @@ __global__ void __launch_bounds__(xa_threads(KP), 1)
         for (int i2 = 0; i2 < NSM; ++i2) accs[i2] = 0.f;
       }
       const int buf = int(tcount & 1u);
-      const bool a_ok = mbar_wait(acc_full(buf), (tcount >> 1) & 1u, wc);
+      const uint32_t aph = (tcount >> 1) & 1u;
+      const bool a_ok = mbar_try_wait(acc_full(buf), aph) || mbar_wait(acc_full(buf), aph, wc);
       if (!__all_sync(0xffffffffu, a_ok)) break;
       fence_after();
       const uint32_t ta = tmem_base + (uint32_t(q * 32) << 16) + uint32_t(buf * NCOL);

@@ -153,7 +153,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       const int64_t j0 = jt * TCH;
       const int64_t nbeg = ck * CHUNK;
       const int64_t nend = (nbeg + CHUNK < g.N) ? nbeg + CHUNK : g.N;
-      if (!mbar_wait(b_empty, (icount & 1u) ^ 1u, wc)) { ok = false; break; }
+      // the bounded waits are calls (registers saved around them): an inline try_wait goes first
+      if (!mbar_try_wait(b_empty, (icount & 1u) ^ 1u) && !mbar_wait(b_empty, (icount & 1u) ^ 1u, wc)) {
+        ok = false;
+        break;
+      }
       // B = Q_l[:, j0 : j0 + 256] as hi/lo K-major tiles (channel = row, s = k)
       const float* Ql = Q + int64_t(l) * r * g.d;
       for (int h = 0; h < 2; ++h) {
@@ -197,7 +201,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
               if (s < r) u[s] = fmaf(ec, __ldg(pr + s), u[s]);
           }
         }
-        if (!mbar_wait(a_empty(buf), ph ^ 1u, wc)) { ok = false; break; }
+        if (!mbar_try_wait(a_empty(buf), ph ^ 1u) && !mbar_wait(a_empty(buf), ph ^ 1u, wc)) {
+          ok = false;
+          break;
+        }
 #pragma unroll
         for (int s4 = 0; s4 < kMaxRP; s4 += 4) {
           if (s4 >= rp) break;
@@ -228,13 +235,19 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         decode(g, it, l, jt, ck);
         const int64_t nbeg = ck * CHUNK;
         const int64_t nend = (nbeg + CHUNK < g.N) ? nbeg + CHUNK : g.N;
-        if (!mbar_wait(b_full, icount & 1u, wc)) { ok = false; break; }
+        if (!mbar_try_wait(b_full, icount & 1u) && !mbar_wait(b_full, icount & 1u, wc)) {
+          ok = false;
+          break;
+        }
         fence_after();
         for (int64_t n0 = nbeg; n0 < nend; n0 += TM, ++tcount) {
           const int buf = int(tcount & 1u);
           const uint32_t ph = (tcount >> 1) & 1u;
-          if (!mbar_wait(acc_empty(buf), ph ^ 1u, wc)) { ok = false; break; }
-          if (!mbar_wait(a_full(buf), ph, wc)) { ok = false; break; }
+          if ((!mbar_try_wait(acc_empty(buf), ph ^ 1u) && !mbar_wait(acc_empty(buf), ph ^ 1u, wc)) ||
+              (!mbar_try_wait(a_full(buf), ph) && !mbar_wait(a_full(buf), ph, wc))) {
+            ok = false;
+            break;
+          }
           fence_after();
           const uint32_t d_tmem = tmem_base + uint32_t(buf) * TCH;
           for (int kk = 0; kk < rp / 8; ++kk) {
@@ -278,7 +291,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       for (int64_t n0 = nbeg; n0 < nend; n0 += TM, ++tcount) {
         const int buf = int(tcount & 1u);
         const uint32_t ph = (tcount >> 1) & 1u;
-        const bool w_ok = mbar_wait(acc_full(buf), ph, wc);
+        const bool w_ok = mbar_try_wait(acc_full(buf), ph) || mbar_wait(acc_full(buf), ph, wc);
         if (!__all_sync(0xffffffffu, w_ok)) { ok = false; break; }
         fence_after();
         const int64_t n = n0 + row;
