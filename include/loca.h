@@ -391,9 +391,12 @@ int loca_step_from_gram(const float* gram, int32_t L, int64_t d, const double* t
  *               the p-th pivot of G_l + lam I is not positive (B[j, l] is then zero)
  * G_out         L x k x k float output or NULL;  C_out  L x d x k float output or NULL
  * 1 <= k <= min(d, 32); 1 <= nl <= 16.
- * The products gram_l A_l and cross_l A_l run on the tensor cores (an exact three-way bf16 split
- * of each operand, so every product is exact in fp32; fp32 sums) when d and k are multiples of 4
- * and gram, cross and A are 16-byte aligned, else on the CUDA cores in fp32.  The tensor-core
+ * The products gram_l A_l and cross_l A_l run on the tensor cores when d and k are multiples of
+ * 4 and gram, cross and A are 16-byte aligned, else on the CUDA cores in fp32.  On the tensor
+ * cores each operand is split into two fp16 parts after scaling by a power of two per
+ * 32-channel row slice (gram, cross) or column slice (A), which carries every value to within
+ * 2^-22 of itself; the part products are exact in fp32 and summed in fp32, as accurate as an
+ * fp32 FMA evaluation.  The tensor-core
  * path's waits are bounded (loca_set_wait_limit); one that gives up writes LOCA_ERR_TIMEOUT to
  * the device status word and leaves B undefined.
  */

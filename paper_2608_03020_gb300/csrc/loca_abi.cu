@@ -146,7 +146,7 @@ AccumWs accum_ws(int32_t L) {
 }
 
 struct SolveWs {
-  size_t ga, ca, fac, flag, total;
+  size_t ga, ca, fac, arec, flag, total;
 };
 SolveWs solve_ws(int32_t L, int64_t d, int32_t k) {
   SolveWs w{};
@@ -154,7 +154,8 @@ SolveWs solve_ws(int32_t L, int64_t d, int32_t k) {
   w.ga = 0;
   w.ca = one;
   w.fac = 2 * one;  // per-candidate Cholesky factors
-  w.flag = w.fac + align256(chol_workspace_bytes(L));  // abort flag of the tensor-core projection's waits
+  w.arec = w.fac + align256(chol_workspace_bytes(L));  // A's split slabs for the tensor-core projection
+  w.flag = w.arec + align256(project_tc_workspace_bytes(L, d, k));  // abort flag of its waits
   w.total = w.flag + 256;
   return w;
 }
@@ -700,7 +701,7 @@ int loca_ridge_solve(const float* gram, const float* cross, const float* cross_s
   if (project_tc_supported(gram, cross, A, d, k)) {
     int32_t* status = device_status_word();
     if (!status) return fail(LOCA_ERR_CUDA, "cannot resolve the device status word");
-    e = launch_project_tc(gram, cross, A, L, d, k, GA, CA, status,
+    e = launch_project_tc(gram, cross, A, L, d, k, GA, CA, ws_at(workspace, lay.arec), status,
                           reinterpret_cast<int32_t*>(ws_at(workspace, lay.flag)), s);
     nsplit = 1;
   } else {

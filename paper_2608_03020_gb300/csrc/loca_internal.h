@@ -128,11 +128,15 @@ cudaError_t launch_kspace_solve(const float* G, const float* SC, const double* x
 int project_split();
 cudaError_t launch_project_rows(const float* gram, const float* cross, const float* A, int L,
                                 int64_t d, int k, float* GA, float* CA, cudaStream_t s);
-// Tensor-core projection (tf32 MMAs with the 3xTF32 split): d % 4 == 0, k % 4 == 0, 4 <= k <= 32,
-// 16-byte aligned gram, cross and A.  abort_flag: 4 bytes of launch-local device memory.
+// Tensor-core projection (fp16 MMAs on a row- and column-scaled two-part split): d % 4 == 0,
+// k % 4 == 0, 4 <= k <= 32, 16-byte aligned gram, cross and A.  arec: project_tc_workspace_bytes
+// of 16-byte aligned device memory for A's split slabs; abort_flag: 4 bytes of launch-local
+// device memory.
 bool project_tc_supported(const float* gram, const float* cross, const float* A, int64_t d, int k);
+size_t project_tc_workspace_bytes(int L, int64_t d, int k);
 cudaError_t launch_project_tc(const float* gram, const float* cross, const float* A, int L, int64_t d, int k,
-                              float* GA, float* CA, int32_t* status, int32_t* abort_flag, cudaStream_t s);
+                              float* GA, float* CA, void* arec, int32_t* status, int32_t* abort_flag,
+                              cudaStream_t s);
 // fac: chol_workspace_bytes(L) of device memory for the per-candidate factors (nl <= 16).
 size_t chol_workspace_bytes(int L);
 cudaError_t launch_chol_solve(const float* GA, const float* CA, int nsplit, const float* A, const float* B_prev,
