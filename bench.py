@@ -59,9 +59,10 @@ KSPACE_TRAFFIC = {"sha256": "3aba9c60b10e48c0", "L_capture": 2, "N": 131072, "d"
 TARGETS_TRAFFIC = {"sha256": "1796bbc513a2c2d2", "L_capture": 2, "N": 131072, "d": 3584, "r": 16,
                    "read": 13250816, "write": 1817000448,
                    "kernel": "k_targets_tc"}
-# k_project_tc (the ridge solve's projection, which reads Gram and Cross once) at k = 16
-PROJECT_TRAFFIC = {"sha256": "ba847e501813d245", "L_capture": 2, "d": 3584, "k": 16,
-                   "read": 206016000, "write": 1437952,
+# k_project_tc (the ridge solve's projection, which reads Gram and Cross once) at k = 16: taken
+# on the full launch (L = 28, 2.9 GB of statistics), so L_capture = 28
+PROJECT_TRAFFIC = {"sha256": "7771065c47a83799", "L_capture": 28, "d": 3584, "k": 16,
+                   "read": 2886107648, "write": 17300992,
                    "kernel": "k_project_tc"}
 
 
