@@ -544,7 +544,9 @@ def main():
     ws_g = torch.empty(lc.gram_cross_workspace_size(), dtype=torch.uint8, device=dev)
     ws_s = torch.empty(lc.ridge_solve_workspace_size(L, d, k), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
-    launches_per_step = 1 + 2 + 2 + 1 + 2  # error; targets+reduce; gram/cross+mirror; step; project+solve
+    # k_head_error; k_targets_tc + k_reduce_partials; k_gram_cross_tc + k_gram_mirror; k_step_from_gram;
+    # k_project_prep + k_project_tc + k_chol_gram + k_chol_factor + k_chol_rows
+    launches_per_step = 1 + 2 + 2 + 1 + 5
 
     def step(ev=None):
         if ev is not None:
